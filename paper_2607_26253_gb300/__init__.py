@@ -1,0 +1,11 @@
+"""SARA rollout collection on one GB300 (sm_103a): C-ABI library + thin Python binding.
+
+The hot path (batched bf16 decode with tcgen05/TMEM GEMMs, GQA decode attention, fused
+RMSNorm/RoPE epilogues, Gumbel-max sampling, and the on-device Algorithm 1 controller)
+lives in libsara.so, built from csrc/ by build.py.  This package only marshals arguments.
+"""
+from .sara import (ABANDONED, COMMITTED, INCOMPLETE, UNDRAWN, Handle, ModelCfg, SaraError, attention_decode,
+                   gemm_bf16, load, model_cfg, sample, tau_fraction)
+
+__all__ = ["Handle", "ModelCfg", "SaraError", "attention_decode", "gemm_bf16", "load", "model_cfg", "sample",
+           "tau_fraction", "UNDRAWN", "COMMITTED", "ABANDONED", "INCOMPLETE"]

@@ -1,0 +1,473 @@
+// SARA controller on the GPU (Algorithm 1 of arxiv 2607.26253), one CTA of 1024 threads.
+//
+// Runs at the top of every loop iteration of the step graph.  Mid-round (live rows > 0) it
+// only checks the round's step bound.  When a round has finished (or before the probe) it
+//   1. applies the round's verdicts to each issued prompt's posterior counts (n, s);
+//   2. DECIDEs every active prompt with the exact table of Eq. (decide) built from the
+//      closed-form predictor p_eff of Prop. 1 (integer prior, exact 128-bit rationals);
+//   3. funds one more rollout for each continuing prompt while the budget N allows, the
+//      highest p_eff first (ties: lower stream index), the rest become INCOMPLETE;
+//   4. refills the working set toward B - |C| with fresh prompts (n0-rollout probes);
+//   5. (decode) assigns prompt-KV slots and rollout slots, writes the prefill rows of the
+//      fresh prompts and the first decode step's rows, and opens the round-start branch of
+//      the graph; sets the loop condition to 0 once nothing more can be issued.
+#pragma once
+#include <cuda_runtime.h>
+
+#include "device_common.cuh"
+#include "step_state.cuh"
+
+namespace sara {
+
+constexpr int kCtlThreads = 1024;
+
+// ---------------------------------------------------------------------------------------
+// block-wide helpers (blockDim.x == kCtlThreads)
+struct CtlShared {
+    int warp_tot[32];
+    long long warp_tot64[32];
+    int bcast[8];
+    int hist[2 * kMaxK + 2];
+    unsigned pslot_used[256];  // bitmap of prompt slots (<= 8192)
+};
+
+__device__ __forceinline__ int blk_excl_scan(int v, int &total, CtlShared &sh) {
+    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+    int x = v;
+#pragma unroll
+    for (int o = 1; o < 32; o <<= 1) {
+        const int y = __shfl_up_sync(0xffffffffu, x, o);
+        if (lane >= o) x += y;
+    }
+    if (lane == 31) sh.warp_tot[warp] = x;
+    __syncthreads();
+    if (warp == 0) {
+        int w = sh.warp_tot[lane];
+#pragma unroll
+        for (int o = 1; o < 32; o <<= 1) {
+            const int y = __shfl_up_sync(0xffffffffu, w, o);
+            if (lane >= o) w += y;
+        }
+        sh.warp_tot[lane] = w;  // inclusive
+    }
+    __syncthreads();
+    const int before = (warp > 0 ? sh.warp_tot[warp - 1] : 0) + x - v;
+    total = sh.warp_tot[31];
+    __syncthreads();
+    return before;
+}
+
+__device__ __forceinline__ long long blk_sum64(long long v, CtlShared &sh) {
+    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
+    if (lane == 0) sh.warp_tot64[warp] = v;
+    __syncthreads();
+    long long t = 0;
+    for (int w = 0; w < 32; ++w) t += sh.warp_tot64[w];
+    __syncthreads();
+    return t;
+}
+
+__device__ __forceinline__ int blk_max(int v, CtlShared &sh) {
+    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) v = max(v, __shfl_xor_sync(0xffffffffu, v, o));
+    if (lane == 0) sh.warp_tot[warp] = v;
+    __syncthreads();
+    int t = sh.warp_tot[0];
+    for (int w = 1; w < 32; ++w) t = max(t, sh.warp_tot[w]);
+    __syncthreads();
+    return t;
+}
+
+// Stable compaction of list[0..n) by flag(i) into dst; returns the kept count.
+template <typename Flag>
+__device__ __forceinline__ int blk_compact(const int32_t *list, int n, int32_t *dst, Flag flag, CtlShared &sh) {
+    int out = 0;
+    for (int base = 0; base < n; base += kCtlThreads) {
+        const int i = base + threadIdx.x;
+        const int keep = (i < n) ? (flag(i) ? 1 : 0) : 0;
+        int tot;
+        const int off = blk_excl_scan(keep, tot, sh);
+        if (keep) dst[out + off] = list[i];
+        out += tot;
+    }
+    __syncthreads();
+    return out;
+}
+
+// ---------------------------------------------------------------------------------------
+// exact predictor: prod_{i<a} (b+i) / (b+r+i) and p_eff = 1 - that for a saturated prefix
+typedef unsigned __int128 u128;
+
+__device__ __forceinline__ void saturated_ratio(int a, int b, int r, u128 &num, u128 &den) {
+    num = 1;
+    den = 1;
+    for (int i = 0; i < a; ++i) {
+        num *= (u128)(b + i);
+        den *= (u128)(b + r + i);
+    }
+}
+// p_eff(n, s) for n >= 1 as (num, den)
+__device__ __forceinline__ void peff_frac(int n, int s, int k, int a0, int b0, u128 &pn, u128 &pd) {
+    if (s >= 1 && n - s >= 1) { pn = 1; pd = 1; return; }
+    u128 rn, rd;
+    if (s == 0) saturated_ratio(a0, b0 + n, k - n, rn, rd);  // all-fail prefix
+    else saturated_ratio(b0, a0 + n, k - n, rn, rd);         // all-pass prefix
+    pn = rd - rn;
+    pd = rd;
+}
+
+// dec_tab[n][s] (Eq. decide) and rank_tab[n][s] = number of keys (mixed, (m,0), (m,m)) with a
+// strictly larger p_eff, so a smaller rank means a higher priority; 0 = mixed.  1 <= n <= k.
+static __device__ void ctl_build_tables(const StepConst &K, const StepPtrs &c) {
+    const int k = K.k;
+    for (int e = threadIdx.x; e < kTabDim * kTabDim; e += kCtlThreads) {
+        const int n = e / kTabDim, s = e % kTabDim;
+        uint8_t d = D_CONTINUE, rk = 0;
+        if (n >= 1 && n <= k && s <= n) {
+            const bool mixed = s >= 1 && n - s >= 1;
+            u128 pn, pd;
+            peff_frac(n, s, k, K.a0, K.b0, pn, pd);
+            if (mixed) d = (n >= K.commit_min) ? D_COMMIT : D_CONTINUE;
+            else if (n >= k) d = D_ABANDON;
+            else d = (pn * (u128)K.tau_den < (u128)K.tau_num * pd) ? D_ABANDON : D_CONTINUE;
+            int cntg = 0;
+            if (!mixed) {
+                cntg = (pn == pd) ? 0 : 1;  // the mixed class (p_eff = 1)
+                for (int mm = 1; mm <= k; ++mm) {
+                    for (int side = 0; side < 2; ++side) {
+                        u128 qn, qd;
+                        peff_frac(mm, side ? mm : 0, k, K.a0, K.b0, qn, qd);
+                        if (qn * pd > pn * qd) ++cntg;
+                    }
+                }
+            }
+            rk = (uint8_t)min(cntg, 2 * kMaxK + 1);
+        }
+        c.dec_tab[e] = d;
+        c.rank_tab[e] = rk;
+    }
+}
+
+__device__ __forceinline__ int verdict_of(uint64_t seed, int64_t q, int j, uint64_t thr) {
+    return (splitmix_at(seed, (uint64_t)q * 64u + (uint64_t)j + 1u) >> 32) < thr ? 1 : 0;
+}
+
+__device__ __forceinline__ uint64_t sampler_row_seed(uint64_t sample_seed, int64_t uid, int t) {
+    return splitmix_at(sample_seed, (uint64_t)uid * (1ull << 20) + (uint64_t)t + 1u);
+}
+
+// use_handles: bit 0 = the loop handle exists, bit 1 = the round-start handle exists.
+__device__ __forceinline__ void set_conds(cudaGraphConditionalHandle h_loop, cudaGraphConditionalHandle h_round,
+                                          int loop, int round_start, int use_handles) {
+    if (threadIdx.x == 0) {
+        if (use_handles & 1) cudaGraphSetConditional(h_loop, loop ? 1u : 0u);
+        if (use_handles & 2) cudaGraphSetConditional(h_round, round_start ? 1u : 0u);
+    }
+}
+
+// Decode rows of a round's first step and the prefill rows of its fresh prompts.
+static __device__ void ctl_round_setup(const StepConst &K, StepVars &V, const StepPtrs &c, CtlShared &sh,
+                                       int n_funded, int n_fresh, int first_fresh_q) {
+    const int k = K.k, Lp = K.Lp;
+    // prompt slots: continuing prompts keep theirs, fresh prompts take free ones in order
+    for (int w = threadIdx.x; w < 256; w += kCtlThreads) sh.pslot_used[w] = 0u;
+    __syncthreads();
+    for (int i = threadIdx.x; i < n_funded; i += kCtlThreads) {
+        const int ps = c.q_pslot[c.act[i]];
+        atomicOr(&sh.pslot_used[ps >> 5], 1u << (ps & 31));
+    }
+    __syncthreads();
+    int assigned = 0;
+    for (int base = 0; base < c.max_active && assigned < n_fresh; base += kCtlThreads) {
+        const int ps = base + threadIdx.x;
+        const int freeb = (ps < c.max_active) && !((sh.pslot_used[ps >> 5] >> (ps & 31)) & 1u);
+        int tot;
+        const int off = blk_excl_scan(freeb, tot, sh);
+        if (freeb && assigned + off < n_fresh) c.fresh_pslot[assigned + off] = ps;
+        assigned += tot;
+    }
+    __syncthreads();
+    if (assigned < n_fresh) { if (threadIdx.x == 0) report_error(&V.err, ERR_CAPACITY); return; }
+    for (int f = threadIdx.x; f < n_fresh; f += kCtlThreads) c.q_pslot[first_fresh_q + f] = c.fresh_pslot[f];
+    __syncthreads();
+
+    // rollout slots in issue order
+    const int n_iss = V.n_iss;
+    int R = 0;
+    for (int base = 0; base < n_iss; base += kCtlThreads) {
+        const int e = base + threadIdx.x;
+        const int cnt = (e < n_iss) ? c.iss_c[e] : 0;
+        int tot;
+        const int off = blk_excl_scan(cnt, tot, sh);
+        if (e < n_iss) {
+            const int q = c.iss_q[e];
+            const int n_before = c.q_n[q];
+            for (int t = 0; t < cnt; ++t) {
+                const int slot = R + off + t;
+                if (slot >= c.max_seqs) continue;
+                const int j = n_before + t;
+                int L = c.p_len[(int64_t)q * k + j];
+                if (L < 1 || L > K.max_gen) {  // lengths bound the KV cache and the token output
+                    report_error(&V.err, ERR_BOUNDS);
+                    L = L < 1 ? 1 : K.max_gen;
+                }
+                c.seq_q[slot] = q;
+                c.seq_j[slot] = j;
+                c.seq_len[slot] = L;
+                c.seq_gen[slot] = 0;
+                c.seq_pslot[slot] = c.q_pslot[q];
+                c.seq_uid[slot] = (int64_t)q * 64 + j;
+            }
+        }
+        R += tot;
+    }
+    __syncthreads();
+    if (R > c.max_seqs) { if (threadIdx.x == 0) report_error(&V.err, ERR_CAPACITY); return; }
+    // first decode step: input = last prompt token at position Lp - 1
+    const int nsplit = (Lp + K.attn_chunk - 1) / K.attn_chunk;
+    int maxL = 0;
+    for (int r = threadIdx.x; r < R; r += kCtlThreads) {
+        const int q = c.seq_q[r];
+        c.row_slot[r] = r;
+        c.row_pos[r] = Lp - 1;
+        c.row_tok[r] = c.p_tok[(int64_t)q * Lp + Lp - 1];
+        c.row_seed[r] = sampler_row_seed(K.sample_seed, c.seq_uid[r], 0);
+        c.row_item0[r] = r * nsplit;
+        for (int sp = 0; sp < nsplit; ++sp) c.att_items[r * nsplit + sp] = make_int2(r, sp);
+        maxL = max(maxL, c.seq_len[r]);
+    }
+    maxL = blk_max(maxL, sh);
+    // prefill rows: fresh prompt f, token t < Lp - 1, written into prompt slot fresh_pslot[f]
+    const int Lpre = Lp - 1;
+    const int pre_rows = n_fresh * Lpre;
+    if (pre_rows > c.pre_cap) { if (threadIdx.x == 0) report_error(&V.err, ERR_CAPACITY); return; }
+    for (int r = threadIdx.x; r < pre_rows; r += kCtlThreads) {
+        const int f = r / Lpre, t = r - f * Lpre;
+        const int q = first_fresh_q + f;
+        c.pre_slot[r] = c.fresh_pslot[f];
+        c.pre_pos[r] = t;
+        c.pre_tok[r] = c.p_tok[(int64_t)q * Lp + t];
+        c.pre_items[r] = make_int2(r, 0);
+        c.pre_item0[r] = r;
+    }
+    if (threadIdx.x == 0) {
+        V.live = R;
+        V.att_items = R * nsplit;
+        V.pre_rows = pre_rows;
+        V.n_fresh = n_fresh;
+        V.round_maxL = maxL;
+        V.round_steps = 0;
+    }
+}
+
+// One round end + allocation (everything but the decode).
+static __device__ void ctl_round(const StepConst &K, StepVars &V, const StepPtrs &c, CtlShared &sh) {
+    const int k = K.k;
+    const int tid = threadIdx.x;
+    // ---- 1. apply the finished round's verdicts
+    if (V.round >= 0) {
+        const int n_iss = V.n_iss;
+        long long tok = 0;
+        int lmax = 0;
+        for (int e = tid; e < n_iss; e += kCtlThreads) {
+            const int q = c.iss_q[e], cnt = c.iss_c[e];
+            const int n = c.q_n[q];
+            int s = c.q_s[q];
+            for (int t = 0; t < cnt; ++t) {
+                const int j = n + t;
+                s += verdict_of(K.reward_seed, q, j, c.p_thr[q]);
+                const int L = c.p_len[(int64_t)q * k + j];
+                tok += L;
+                lmax = max(lmax, L);
+            }
+            c.q_n[q] = (uint8_t)(n + cnt);
+            c.q_s[q] = (uint8_t)s;
+        }
+        tok = blk_sum64(tok, sh);
+        lmax = blk_max(lmax, sh);
+        if (tid == 0) {
+            V.gen_tokens += tok;
+            V.sched_steps += lmax;
+            V.rounds_done += 1;
+        }
+        __syncthreads();
+        // ---- 2. DECIDE (Eq. decide) for every active prompt
+        const int n_act = V.n_act;
+        long long commits = 0;
+        for (int i = tid; i < n_act; i += kCtlThreads) {
+            const int q = c.act[i];
+            const int d = c.dec_tab[c.q_n[q] * kTabDim + c.q_s[q]];
+            if (d == D_COMMIT) { c.q_status[q] = ST_COMMITTED; c.q_round[q] = (int16_t)V.round; ++commits; }
+            else if (d == D_ABANDON) { c.q_status[q] = ST_ABANDONED; c.q_round[q] = (int16_t)V.round; }
+        }
+        commits = blk_sum64(commits, sh);
+        __syncthreads();
+        const int n_cont = blk_compact(c.act, n_act, c.act_tmp,
+                                       [&](int i) { return c.q_status[c.act[i]] == ST_ACTIVE; }, sh);
+        for (int i = tid; i < n_cont; i += kCtlThreads) c.act[i] = c.act_tmp[i];
+        __syncthreads();
+        if (tid == 0) { V.C += commits; V.n_act = n_cont; }
+        __syncthreads();
+    }
+    const int B = K.B;
+    const int n_cont = V.n_act;
+    // ---- stop once B effective groups are committed
+    if (V.C >= B) {
+        for (int i = tid; i < n_cont; i += kCtlThreads) c.q_status[c.act[i]] = ST_INCOMPLETE;
+        __syncthreads();
+        if (tid == 0) { V.n_act = 0; V.n_iss = 0; V.done = 1; }
+        __syncthreads();
+        return;
+    }
+    // ---- 3. fund continuing prompts by p_eff priority while the budget allows
+    const long long budget = K.N - V.used;
+    int n_funded = n_cont;
+    if ((long long)n_cont > budget) {
+        const int take = (int)max(0ll, budget);
+        for (int b = tid; b < 2 * kMaxK + 2; b += kCtlThreads) sh.hist[b] = 0;
+        __syncthreads();
+        for (int i = tid; i < n_cont; i += kCtlThreads) {
+            const int q = c.act[i];
+            atomicAdd(&sh.hist[c.rank_tab[c.q_n[q] * kTabDim + c.q_s[q]]], 1);
+        }
+        __syncthreads();
+        if (tid == 0) {
+            int acc = 0, rstar = 0;
+            while (rstar < 2 * kMaxK + 2 && acc + sh.hist[rstar] < take) acc += sh.hist[rstar++];
+            sh.bcast[0] = rstar;
+            sh.bcast[1] = take - acc;  // how many of rank rstar, in stream order
+        }
+        __syncthreads();
+        const int rstar = sh.bcast[0], need = sh.bcast[1];
+        int seen = 0;
+        for (int base = 0; base < n_cont; base += kCtlThreads) {
+            const int i = base + tid;
+            int rk = 1 << 30, q = -1;
+            if (i < n_cont) { q = c.act[i]; rk = c.rank_tab[c.q_n[q] * kTabDim + c.q_s[q]]; }
+            const int at = (rk == rstar) ? 1 : 0;
+            int tot;
+            const int off = blk_excl_scan(at, tot, sh);
+            if (i < n_cont) {
+                const bool fund = rk < rstar || (at && seen + off < need);
+                if (!fund) c.q_status[q] = ST_INCOMPLETE;
+            }
+            seen += tot;
+        }
+        __syncthreads();
+        n_funded = blk_compact(c.act, n_cont, c.act_tmp,
+                               [&](int i) { return c.q_status[c.act[i]] == ST_ACTIVE; }, sh);
+        for (int i = tid; i < n_funded; i += kCtlThreads) c.act[i] = c.act_tmp[i];
+        __syncthreads();
+    }
+    // ---- 4. refill toward B - |C| with fresh n0-probes
+    const long long used_after = V.used + n_funded;
+    const long long room = (long long)(B - V.C) - n_funded;
+    const long long by_budget = (K.N - used_after) / K.n0;
+    const long long by_pool = (long long)K.P - V.cursor;
+    const int n_fresh = (int)max(0ll, min(min(room, by_budget), by_pool));
+    const int first_fresh = (int)V.cursor;
+    if (n_funded + n_fresh > c.max_active) {  // cannot happen when B <= max_active
+        if (tid == 0) { report_error(&V.err, ERR_CAPACITY); V.done = 1; }
+        __syncthreads();
+        return;
+    }
+    for (int f = tid; f < n_fresh; f += kCtlThreads) {
+        const int q = first_fresh + f;
+        c.q_status[q] = ST_ACTIVE;
+        c.act[n_funded + f] = q;
+    }
+    const int n_iss = n_funded + n_fresh;
+    __syncthreads();
+    for (int i = tid; i < n_iss; i += kCtlThreads) {
+        c.iss_q[i] = c.act[i];
+        c.iss_c[i] = (i < n_funded) ? 1 : K.n0;
+    }
+    __syncthreads();
+    if (tid == 0) {
+        V.used = used_after + (long long)n_fresh * K.n0;
+        V.drawn += n_fresh;
+        V.cursor += n_fresh;
+        V.n_act = n_iss;
+        V.n_iss = n_iss;
+        V.round += 1;
+        if (n_iss == 0) V.done = 1;
+    }
+    __syncthreads();
+    if (K.decode && n_iss > 0) ctl_round_setup(K, V, c, sh, n_funded, n_fresh, first_fresh);
+    __syncthreads();
+}
+
+// Per-iteration controller kernel of the step graph.
+static __global__ void __launch_bounds__(kCtlThreads, 1)
+ctl_kernel(StepPtrs c, cudaGraphConditionalHandle h_loop, cudaGraphConditionalHandle h_round, int use_handles) {
+    __shared__ CtlShared sh;
+    pdl_wait_prior_grids();
+    const StepConst K = *c.kc;
+    StepVars &V = *c.v;
+    __syncthreads();
+    if (threadIdx.x == 0) V.iters += 1;
+    if (V.err != 0 && !V.done) {  // a kernel reported an error: end the step now
+        __syncthreads();
+        if (threadIdx.x == 0) { V.done = 1; V.live = 0; }
+        set_conds(h_loop, h_round, 0, 0, use_handles);
+        return;
+    }
+    if (V.done) { set_conds(h_loop, h_round, 0, 0, use_handles); return; }
+    if (V.live > 0) {
+        // mid-round: the round may run at most round_maxL decode steps
+        const int stop = V.round_steps > V.round_maxL;
+        if (stop && threadIdx.x == 0) { report_error(&V.err, ERR_ITER_BOUND); V.done = 1; }
+        set_conds(h_loop, h_round, !stop, 0, use_handles);
+        return;
+    }
+    if (K.teacher) {  // teacher forcing runs one prepared round
+        if (threadIdx.x == 0) V.done = 1;
+        set_conds(h_loop, h_round, 0, 0, use_handles);
+        return;
+    }
+    // a round boundary: bound the number of rounds (each issues >= 1 rollout)
+    if (V.rounds_done > K.N + 1) {
+        if (threadIdx.x == 0) { report_error(&V.err, ERR_ITER_BOUND); V.done = 1; }
+        set_conds(h_loop, h_round, 0, 0, use_handles);
+        return;
+    }
+    ctl_round(K, V, c, sh);
+    __syncthreads();
+    if (V.err & (ERR_CAPACITY | ERR_BOUNDS)) { if (threadIdx.x == 0) V.done = 1; }
+    __syncthreads();
+    const int done = V.done;
+    if (done) {
+        // remaining active prompts end INCOMPLETE
+        const int n_act = V.n_act;
+        for (int i = threadIdx.x; i < n_act; i += kCtlThreads)
+            if (c.q_status[c.act[i]] == ST_ACTIVE) c.q_status[c.act[i]] = ST_INCOMPLETE;
+        if (threadIdx.x == 0) { V.live = 0; V.n_act = 0; }
+    }
+    set_conds(h_loop, h_round, !done, !done && K.decode, use_handles);
+}
+
+// Reset the step state and build the decision tables (one CTA).
+static __global__ void __launch_bounds__(kCtlThreads, 1) ctl_init_kernel(StepPtrs c) {
+    pdl_wait_prior_grids();
+    const StepConst K = *c.kc;
+    StepVars &V = *c.v;
+    for (int q = threadIdx.x; q < K.P; q += kCtlThreads) {
+        c.q_status[q] = ST_UNDRAWN;
+        c.q_n[q] = 0;
+        c.q_s[q] = 0;
+        c.q_round[q] = -1;
+        c.q_pslot[q] = -1;
+    }
+    ctl_build_tables(K, c);
+    if (threadIdx.x == 0) {
+        StepVars z;
+        memset(&z, 0, sizeof(z));
+        z.round = -1;
+        V = z;
+    }
+}
+
+}  // namespace sara

@@ -1,0 +1,463 @@
+// Projection GEMM of the decode / prefill path on sm_103a:
+//     Y[r][n] = sum_c X[r][c] * W[n][c]        (X: activations, W: a linear layer's weight)
+// computed "swap-AB" on the 5th-generation tensor core: the weight tile is the MMA's A
+// operand (M = 128 output features), the activation rows are B (N = rows rounded up to
+// 16, <= 128), the fp32 accumulator lives in tensor memory.  Operands are staged in shared
+// memory by TMA (128-byte swizzle) through a multi-stage mbarrier pipeline; one elected
+// thread issues tcgen05.mma; four epilogue warps read the accumulator with tcgen05.ld.
+//
+// Work split: stream-K.  The (tile, k-chunk) units of the whole GEMM are cut into
+// gridDim.x equal contiguous ranges, so every SM streams the same number of weight bytes.
+// A tile whose k-chunks span several CTAs is finished by the CTA that arrives last (a
+// per-tile counter, no spinning): it adds every contributor's fp32 partial in CTA order
+// (deterministic) and runs the epilogue.
+//
+// Warp roles (192 threads): warp 0 = TMA producer, warp 1 = MMA issuer + tensor-memory
+// owner, warps 2..5 = epilogue (warp w reads tensor-memory lanes 32*(w%4) .. +31).
+//
+// In decode mode (one row tile) the producer streams the first pipeline stages of weights
+// before waiting on the preceding grid (programmatic dependent launch), so weight reads
+// overlap the previous kernel's tail.
+#pragma once
+#include "device_common.cuh"
+
+namespace sara {
+
+enum EpiKind : int {
+    EPI_F32 = 0,     // Y fp32 [rows][ld]
+    EPI_QKV = 1,     // RMSNorm scale, RoPE on q/k, q -> q_out, k/v -> KV cache
+    EPI_RESID = 2,   // x += Y; xg = bf16(x * g_next); per-tile sum of squares of x
+    EPI_SWIGLU = 3,  // RMSNorm scale; tile = 64 gate rows + 64 up rows -> h = silu(g) * u
+    EPI_LMHEAD = 4,  // RMSNorm scale; optional fp32 logits; Gumbel-max partial argmax per tile
+};
+
+constexpr int kGemmThreads = 192;
+constexpr int kGemmStages = 5;
+constexpr int kTileM = 128;       // weight rows per tile (MMA M)
+constexpr int kTileK = 64;        // reduction elements per pipeline stage (128 B of bf16)
+constexpr int kTileR = 128;       // activation rows per tile (max MMA N here)
+constexpr int kXBoxRows = 32;     // activation rows per TMA box
+constexpr int kWStageBytes = kTileM * kTileK * 2;   // 16 KB
+constexpr int kXStageBytes = kTileR * kTileK * 2;   // 16 KB
+constexpr int kEpiLd = 33;                          // padded fp32 row of the exchange tile
+
+struct GemmParams {
+    int m_tiles, k_chunks;
+    int rows_cap;              // rows of the activation tensor map
+    const int *rows_dev;       // device count of valid rows (nullptr -> rows_fixed)
+    int rows_fixed;
+    int decode;                // 1: a single row tile, weights prefetched before the PDL wait
+    float *ws_part;            // [gridDim.x][2][kTileR * kTileM] fp32 partials
+    int *ws_cnt;               // [tiles] arrival counters, zero between launches
+    int *err;
+    // outputs / epilogue inputs
+    float *y_f32; int ld;      // EPI_F32 output, EPI_LMHEAD logits (optional); row stride
+    const float *ssq;          // [ssq_tiles][rows_cap] per-128-feature partial sums of x^2
+    int ssq_tiles; float inv_dim; float eps;
+    uint16_t *q_out;           // EPI_QKV: [rows][n_heads * head_dim]
+    int n_heads, n_kv, head_dim;
+    const float2 *rope;        // [positions][head_dim / 2] (cos, sin)
+    const int *row_pos;        // [rows] position of the row's token
+    const int *row_slot;       // [rows] KV slot of the row
+    uint16_t *kv;              // KV cache of this layer: slot s at kv + s * kv_slot_stride,
+    int64_t kv_slot_stride;    //   laid out [2][n_kv][kv_cap][head_dim]
+    int kv_cap;
+    float *x_f32;              // EPI_RESID residual stream [rows][ld]
+    uint16_t *xg_out;          // EPI_RESID bf16(x * g_next) [rows][ld]
+    const uint16_t *g_next;    // EPI_RESID next RMSNorm weight [ld]
+    float *ssq_out;            // EPI_RESID [m_tiles][rows_cap]
+    uint16_t *h_out;           // EPI_SWIGLU [rows][ld]
+    const uint64_t *row_seed;  // EPI_LMHEAD sampler key of the row
+    float *arg_val; int *arg_idx;  // EPI_LMHEAD [rows][m_tiles] partial max / argmax
+};
+
+struct GemmSmem {
+    uint64_t full[kGemmStages];
+    uint64_t empty[kGemmStages];
+    uint64_t acc_full[2];
+    uint64_t acc_empty[2];
+    uint64_t drain;
+    uint32_t tmem_base;
+    int abort_flag;
+    int last_flag;
+    int epi_abort;      // set by an epilogue warp whose bounded wait gave up
+    int epi_decision;   // uniform abort decision of the epilogue warps
+    int skip;           // an earlier kernel of the step reported an error: do nothing
+    float inv_rms[kTileR];
+    float xch[kTileM * kEpiLd];        // exchange tile: 128 features x 32 columns
+};
+
+constexpr size_t kGemmSmemBytes =
+    1024 /* alignment slack */ + (size_t)kGemmStages * (kWStageBytes + kXStageBytes) + sizeof(GemmSmem);
+
+// Stream-K partition: CTA c owns units [unit_begin(c), unit_begin(c+1)).
+__device__ __forceinline__ int64_t unit_begin(int c, int64_t U, int G) { return (int64_t)c * U / G; }
+__device__ __forceinline__ int cta_of_unit(int64_t u, int64_t U, int G) {
+    int c = (int)((u * G) / U);
+    while (c + 1 < G && unit_begin(c + 1, U, G) <= u) ++c;
+    while (c > 0 && unit_begin(c, U, G) > u) --c;
+    return c;
+}
+__device__ __forceinline__ int64_t min64(int64_t a, int64_t b) { return a < b ? a : b; }
+
+
+template <int EPI>
+__device__ __forceinline__ void gemm_epilogue_chunk(const GemmParams &p, GemmSmem &S, float (&v)[32], int m_tile,
+                                                    int r_base, int c0, int rows_in_tile, int mrow, int etid) {
+    const int n = m_tile * kTileM + mrow;  // output feature
+    const int ncols = min(32, rows_in_tile - c0);
+    if constexpr (EPI == EPI_F32) {
+#pragma unroll
+        for (int c = 0; c < 32; ++c)
+            if (c < ncols) p.y_f32[(int64_t)(r_base + c0 + c) * p.ld + n] = v[c];
+        return;
+    }
+    if constexpr (EPI == EPI_QKV || EPI == EPI_SWIGLU || EPI == EPI_LMHEAD) {
+#pragma unroll
+        for (int c = 0; c < 32; ++c) v[c] *= S.inv_rms[c0 + c];
+    }
+    if constexpr (EPI == EPI_RESID) {
+        const float g = bf16_to_f32(p.g_next[n]);
+#pragma unroll
+        for (int c = 0; c < 32; ++c) {
+            if (c < ncols) {
+                const int64_t idx = (int64_t)(r_base + c0 + c) * p.ld + n;
+                const float x = p.x_f32[idx] + v[c];
+                p.x_f32[idx] = x;
+                p.xg_out[idx] = f32_to_bf16(x * g);
+                v[c] = x * x;
+            }
+        }
+    }
+    if constexpr (EPI == EPI_LMHEAD) {
+#pragma unroll
+        for (int c = 0; c < 32; ++c) {
+            if (c < ncols) {
+                const int r = r_base + c0 + c;
+                if (p.y_f32) p.y_f32[(int64_t)r * p.ld + n] = v[c];
+                v[c] += gumbel_from_hash(splitmix_at(p.row_seed[r], (uint64_t)n + 1));
+            }
+        }
+    }
+    // stage the chunk in shared memory for the cross-feature exchanges / reductions
+#pragma unroll
+    for (int c = 0; c < 32; ++c) S.xch[mrow * kEpiLd + c] = v[c];
+    named_bar_sync(1, 128);
+    if constexpr (EPI == EPI_QKV) {
+        const int hd = p.head_dim, half = hd >> 1;
+        const int head = n / hd, i = n - head * hd;
+        const int partner = (i < half) ? mrow + half : mrow - half;
+        const int fi = (i < half) ? i : i - half;
+        const int nq = p.n_heads, nkv = p.n_kv;
+#pragma unroll
+        for (int c = 0; c < 32; ++c) {
+            if (c < ncols) {
+                const int r = r_base + c0 + c;
+                float y = v[c];
+                if (head < nq + nkv) {  // q or k: rotate the pair (i, i + hd/2)
+                    const float2 cs = p.rope[(int64_t)p.row_pos[r] * half + fi];
+                    const float o = S.xch[partner * kEpiLd + c];
+                    y = (i < half) ? (y * cs.x - o * cs.y) : (y * cs.x + o * cs.y);
+                }
+                if (head < nq) {
+                    p.q_out[(int64_t)r * (nq * hd) + n] = f32_to_bf16(y);
+                } else {
+                    const int isv = head >= nq + nkv;
+                    const int kvh = head - nq - isv * nkv;
+                    uint16_t *dst = p.kv + (int64_t)p.row_slot[r] * p.kv_slot_stride +
+                                    ((int64_t)(isv * nkv + kvh) * p.kv_cap + p.row_pos[r]) * hd + i;
+                    *dst = f32_to_bf16(y);
+                }
+            }
+        }
+    } else if constexpr (EPI == EPI_SWIGLU) {
+        if (mrow < 64) {
+            const int f = m_tile * 64 + mrow;
+#pragma unroll
+            for (int c = 0; c < 32; ++c) {
+                if (c < ncols) {
+                    const float g = v[c], u = S.xch[(mrow + 64) * kEpiLd + c];
+                    const float h = g / (1.0f + expf(-g)) * u;
+                    p.h_out[(int64_t)(r_base + c0 + c) * p.ld + f] = f32_to_bf16(h);
+                }
+            }
+        }
+    } else if constexpr (EPI == EPI_RESID || EPI == EPI_LMHEAD) {
+        // thread etid reduces column c = etid / 4 over features [32 * (etid % 4), +32)
+        const int c = etid >> 2, part = etid & 3;
+        if constexpr (EPI == EPI_RESID) {
+            float s = 0.f;
+            for (int f = 0; f < 32; ++f) s += S.xch[(part * 32 + f) * kEpiLd + c];
+            s += __shfl_xor_sync(0xffffffffu, s, 1);
+            s += __shfl_xor_sync(0xffffffffu, s, 2);
+            if (part == 0 && c < ncols) p.ssq_out[(int64_t)m_tile * p.rows_cap + r_base + c0 + c] = s;
+        } else {
+            float best = -INFINITY;
+            int bi = 0x7fffffff;
+            for (int f = 0; f < 32; ++f) {
+                const float z = S.xch[(part * 32 + f) * kEpiLd + c];
+                if (z > best) { best = z; bi = m_tile * kTileM + part * 32 + f; }
+            }
+#pragma unroll
+            for (int o = 1; o <= 2; o <<= 1) {
+                const float ob = __shfl_xor_sync(0xffffffffu, best, o);
+                const int oi = __shfl_xor_sync(0xffffffffu, bi, o);
+                if (ob > best || (ob == best && oi < bi)) { best = ob; bi = oi; }
+            }
+            if (part == 0 && c < ncols) {
+                const int r = r_base + c0 + c;
+                p.arg_val[(int64_t)r * p.m_tiles + m_tile] = best;
+                p.arg_idx[(int64_t)r * p.m_tiles + m_tile] = bi;
+            }
+        }
+    }
+    named_bar_sync(1, 128);  // xch reused by the next chunk
+}
+
+template <int EPI>
+__global__ void __launch_bounds__(kGemmThreads, 1)
+gemm_tc_kernel(const __grid_constant__ CUtensorMap tmW, const __grid_constant__ CUtensorMap tmX, GemmParams p) {
+    extern __shared__ uint8_t smem_raw[];
+    uint8_t *base = reinterpret_cast<uint8_t *>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~(uintptr_t)1023);
+    uint8_t *sW = base;
+    uint8_t *sX = base + (size_t)kGemmStages * kWStageBytes;
+    GemmSmem &S = *reinterpret_cast<GemmSmem *>(sX + (size_t)kGemmStages * kXStageBytes);
+
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const int G = gridDim.x, cta = blockIdx.x;
+
+    if (threadIdx.x == 0) {
+        for (int s = 0; s < kGemmStages; ++s) { mbar_init(&S.full[s], 1); mbar_init(&S.empty[s], 1); }
+        for (int a = 0; a < 2; ++a) { mbar_init(&S.acc_full[a], 1); mbar_init(&S.acc_empty[a], 4); }
+        mbar_init(&S.drain, 1);
+        S.abort_flag = 0;
+        S.epi_abort = 0;
+        S.skip = (p.err != nullptr) && (*(volatile int *)p.err != 0);
+        fence_mbar_init();
+        prefetch_tensormap(&tmW);
+        prefetch_tensormap(&tmX);
+    }
+    if (warp == 1) { tmem_alloc(&S.tmem_base, 256); tmem_relinquish(); }
+    tc_fence_before();
+    __syncthreads();
+    tc_fence_after();
+    const uint32_t tmem = S.tmem_base;
+
+    // Let the next kernel in the stream start its own weight prefetch.
+    pdl_allow_dependents();
+
+    const int m_tiles = p.m_tiles, kch = p.k_chunks;
+    // In decode mode the row count does not change the partition (one row tile).
+    int rows = 0, r_tiles = 1;
+    if (!p.decode) {
+        pdl_wait_prior_grids();
+        rows = p.rows_dev ? min(*p.rows_dev, p.rows_cap) : p.rows_fixed;
+        r_tiles = (rows + kTileR - 1) / kTileR;
+    }
+    const int64_t U = (int64_t)m_tiles * r_tiles * kch;
+    const int64_t u0 = S.skip ? 0 : unit_begin(cta, U, G);
+    const int64_t u1 = S.skip ? 0 : unit_begin(cta + 1, U, G);
+
+    if (warp == 0) {
+        // ------------------------------------------------------------ TMA producer
+        if (p.decode) {
+            if (lane == 0) {
+                // weights of the first stages before the dependency wait
+                const int64_t n_pre = min64(kGemmStages, u1 - u0);
+                for (int64_t i = 0; i < n_pre; ++i) {
+                    const int64_t u = u0 + i;
+                    const int tile = (int)(u / kch), kc = (int)(u % kch);
+                    const int m_tile = tile % m_tiles;
+                    mbar_expect_tx(&S.full[i], (uint32_t)kWStageBytes);
+                    tma_load_2d(sW + i * kWStageBytes, &tmW, &S.full[i], kc * kTileK, m_tile * kTileM,
+                                l2_policy_evict_first());
+                }
+            }
+            pdl_wait_prior_grids();
+            rows = p.rows_dev ? min(*p.rows_dev, p.rows_cap) : p.rows_fixed;
+        }
+        if (lane == 0) {
+            const uint64_t pol_w = l2_policy_evict_first(), pol_x = l2_policy_evict_last();
+            const int64_t n_pre = p.decode ? min64(kGemmStages, u1 - u0) : 0;
+            int64_t i = 0;
+            for (int64_t u = u0; u < u1; ++u, ++i) {
+                const int s = (int)(i % kGemmStages);
+                const uint32_t ph = (uint32_t)((i / kGemmStages) & 1);
+                if (i >= kGemmStages && !mbar_wait(&S.empty[s], ph ^ 1, p.err)) { S.abort_flag = 1; break; }
+                if (*(volatile int *)&S.abort_flag) break;
+                const int tile = (int)(u / kch), kc = (int)(u % kch);
+                const int m_tile = tile % m_tiles, r_tile = tile / m_tiles;
+                const int rin = min(kTileR, max(rows - r_tile * kTileR, 0));
+                const int nbox = max(1, (rin + kXBoxRows - 1) / kXBoxRows);
+                const uint32_t xbytes = (uint32_t)(nbox * kXBoxRows * kTileK * 2);
+                if (i >= n_pre) {
+                    mbar_arrive_expect_tx(&S.full[s], (uint32_t)kWStageBytes + xbytes);
+                    tma_load_2d(sW + (size_t)s * kWStageBytes, &tmW, &S.full[s], kc * kTileK, m_tile * kTileM, pol_w);
+                } else {
+                    mbar_arrive_expect_tx(&S.full[s], xbytes);
+                }
+                for (int b = 0; b < nbox; ++b)
+                    tma_load_2d(sX + (size_t)s * kXStageBytes + b * kXBoxRows * kTileK * 2, &tmX, &S.full[s],
+                                kc * kTileK, r_tile * kTileR + b * kXBoxRows, pol_x);
+            }
+            // On abort, the last load issued on every stage lands before the CTA exits.
+            if (*(volatile int *)&S.abort_flag) {
+                const int64_t issued = i;
+                for (int s = 0; s < kGemmStages && s < issued; ++s) {
+                    const int64_t last = ((issued - 1 - s) / kGemmStages) * kGemmStages + s;
+                    mbar_wait(&S.full[s], (uint32_t)((last / kGemmStages) & 1), p.err);
+                }
+            }
+        }
+    } else if (warp == 1) {
+        // ------------------------------------------------------------ MMA issuer
+        if (p.decode) {
+            pdl_wait_prior_grids();
+            rows = p.rows_dev ? min(*p.rows_dev, p.rows_cap) : p.rows_fixed;
+        }
+        if (lane == 0) {
+            int64_t i = 0;
+            int seg = 0;
+            for (int64_t u = u0; u < u1; ++seg) {
+                const int tile = (int)(u / kch);
+                const int64_t seg_end = min64(u1, (int64_t)(tile + 1) * kch);
+                const int r_tile = tile / m_tiles;
+                const int rin = min(kTileR, max(rows - r_tile * kTileR, 0));
+                const uint32_t N = (uint32_t)max(16, (rin + 15) & ~15);
+                const uint32_t idesc = idesc_bf16_f32(128, N);
+                const int a = seg & 1;
+                if (seg >= 2 && !mbar_wait(&S.acc_empty[a], (uint32_t)(((seg >> 1) - 1) & 1), p.err)) {
+                    S.abort_flag = 1;
+                    break;
+                }
+                tc_fence_after();
+                const uint32_t d = tmem + (uint32_t)(a * kTileR);
+                bool first = true;
+                for (; u < seg_end; ++u, ++i) {
+                    const int s = (int)(i % kGemmStages);
+                    if (!mbar_wait(&S.full[s], (uint32_t)((i / kGemmStages) & 1), p.err) ||
+                        *(volatile int *)&S.abort_flag) {
+                        S.abort_flag = 1;
+                        break;
+                    }
+                    tc_fence_after();
+                    const uint32_t aw = smem_u32(sW + (size_t)s * kWStageBytes);
+                    const uint32_t ax = smem_u32(sX + (size_t)s * kXStageBytes);
+#pragma unroll
+                    for (int kk = 0; kk < kTileK / 16; ++kk) {
+                        tc_mma_bf16(d, sdesc_kmajor_sw128(aw + kk * 32), sdesc_kmajor_sw128(ax + kk * 32), idesc,
+                                    (first && kk == 0) ? 0u : 1u);
+                    }
+                    first = false;
+                    tc_commit(&S.empty[s]);
+                }
+                if (*(volatile int *)&S.abort_flag) break;
+                tc_commit(&S.acc_full[a]);
+            }
+            // every MMA this thread issued has retired before tensor memory is released
+            tc_commit(&S.drain);
+            mbar_wait(&S.drain, 0, p.err);
+        }
+    } else {
+        // ------------------------------------------------------------ epilogue (warps 2..5)
+        pdl_wait_prior_grids();
+        if (p.decode) rows = p.rows_dev ? min(*p.rows_dev, p.rows_cap) : p.rows_fixed;
+        const int quarter = warp & 3;
+        const int mrow = quarter * 32 + lane;
+        const int etid = threadIdx.x - 64;  // 0..127
+        const uint32_t lane_base = (uint32_t)(quarter * 32) << 16;
+        int seg = 0;
+        for (int64_t u = u0; u < u1; ++seg) {
+            const int tile = (int)(u / kch);
+            const int kc_first = (int)(u % kch);
+            const int64_t seg_end = min64(u1, (int64_t)(tile + 1) * kch);
+            const int kc_last = (int)((seg_end - 1) % kch);
+            u = seg_end;
+            const int m_tile = tile % m_tiles, r_tile = tile / m_tiles;
+            const int r_base = r_tile * kTileR;
+            const int rin = min(kTileR, max(rows - r_base, 0));
+            const int a = seg & 1;
+            // every epilogue warp takes the same abort decision, so none is left in a named barrier
+            const bool ok = mbar_wait(&S.acc_full[a], (uint32_t)((seg >> 1) & 1), p.err);
+            if (!ok && lane == 0) atomicOr(&S.epi_abort, 1);
+            named_bar_sync(1, 128);
+            if (etid == 0) S.epi_decision = S.epi_abort | *(volatile int *)&S.abort_flag;
+            named_bar_sync(1, 128);
+            if (S.epi_decision) {
+                S.abort_flag = 1;
+                break;
+            }
+            tc_fence_after();
+            const bool whole = (kc_first == 0) && (kc_last == kch - 1);
+            bool do_epi = whole;
+            int c_a = cta, c_b = cta;
+            if (!whole) {
+                // write this CTA's partial, count arrivals; the last arrival finishes the tile
+                const int slot = (u0 / kch == tile) ? 0 : 1;
+                float *mine = p.ws_part + ((size_t)cta * 2 + slot) * (kTileR * kTileM);
+                for (int c0 = 0; c0 < rin; c0 += 32) {
+                    float v[32];
+                    tmem_ld_32x32b_x32(tmem + lane_base + (uint32_t)(a * kTileR + c0), v);
+#pragma unroll
+                    for (int c = 0; c < 32; ++c) mine[(c0 + c) * kTileM + mrow] = v[c];
+                }
+                __threadfence();
+                named_bar_sync(1, 128);
+                c_a = cta_of_unit((int64_t)tile * kch, U, G);
+                c_b = cta_of_unit((int64_t)(tile + 1) * kch - 1, U, G);
+                if (etid == 0) {
+                    int nseg = 0;
+                    for (int c = c_a; c <= c_b; ++c) nseg += unit_begin(c, U, G) < unit_begin(c + 1, U, G);
+                    const int old = atomicAdd(&p.ws_cnt[tile], 1);
+                    S.last_flag = (old == nseg - 1);
+                    if (S.last_flag) p.ws_cnt[tile] = 0;
+                }
+                named_bar_sync(1, 128);
+                do_epi = S.last_flag != 0;
+                __threadfence();
+            }
+            if (do_epi) {
+                if constexpr (EPI == EPI_QKV || EPI == EPI_SWIGLU || EPI == EPI_LMHEAD) {
+                    if (etid < rin) {
+                        float s = 0.f;
+                        for (int t = 0; t < p.ssq_tiles; ++t)
+                            s += __ldcg(&p.ssq[(int64_t)t * p.rows_cap + r_base + etid]);
+                        S.inv_rms[etid] = rsqrtf(s * p.inv_dim + p.eps);
+                    } else {
+                        S.inv_rms[etid] = 0.f;
+                    }
+                    named_bar_sync(1, 128);
+                }
+                for (int c0 = 0; c0 < rin; c0 += 32) {
+                    float v[32];
+                    if (whole) {
+                        tmem_ld_32x32b_x32(tmem + lane_base + (uint32_t)(a * kTileR + c0), v);
+                    } else {
+#pragma unroll
+                        for (int c = 0; c < 32; ++c) v[c] = 0.f;
+                        for (int cc = c_a; cc <= c_b; ++cc) {
+                            if (!(unit_begin(cc, U, G) < unit_begin(cc + 1, U, G))) continue;
+                            const int first_tile = (int)(unit_begin(cc, U, G) / kch);
+                            const int slot = (first_tile == tile) ? 0 : 1;
+                            const float *src = p.ws_part + ((size_t)cc * 2 + slot) * (kTileR * kTileM);
+#pragma unroll
+                            for (int c = 0; c < 32; ++c) v[c] += __ldcg(&src[(c0 + c) * kTileM + mrow]);
+                        }
+                    }
+                    gemm_epilogue_chunk<EPI>(p, S, v, m_tile, r_base, c0, rin, mrow, etid);
+                }
+            }
+            // release the accumulator buffer
+            tc_fence_before();
+            __syncwarp();
+            if (lane == 0) mbar_arrive(&S.acc_empty[a]);
+        }
+    }
+
+    tc_fence_before();
+    __syncthreads();
+    tc_fence_after();
+    if (warp == 1) tmem_dealloc(tmem, 256);
+}
+
+}  // namespace sara

@@ -1,0 +1,268 @@
+// Small kernels of the step graph: embedding gather (with the first RMSNorm's inputs),
+// prompt-KV fan-out into rollout slots, sampling reduction + per-step bookkeeping, and the
+// teacher-forcing round setup.
+#pragma once
+#include "controller.cuh"
+#include "device_common.cuh"
+#include "step_state.cuh"
+
+namespace sara {
+
+// x_f32[r] = E[tok[r]]; xg[r] = bf16(x * g); ssq[t][r] = sum over features [128t, 128t+128)
+// of x^2.  One CTA (128 threads) per row; rows >= *rows_dev exit.
+static __global__ void __launch_bounds__(128) embed_kernel(const uint16_t *E, const uint16_t *g, const int *rows_dev,
+                                                           const int *row_tok, int d, int rows_cap, int vocab,
+                                                           float *x_f32, uint16_t *xg, float *ssq, int *err) {
+    pdl_wait_prior_grids();
+    pdl_allow_dependents();
+    const int rows = min(*rows_dev, rows_cap);
+    __shared__ float red[4];
+    for (int r = blockIdx.x; r < rows; r += gridDim.x) {
+        int tok = row_tok[r];
+        if (tok < 0 || tok >= vocab) {  // token ids come from the caller: never read outside E
+            if (threadIdx.x == 0) report_error(err, ERR_BOUNDS);
+            tok = 0;
+        }
+        const uint16_t *er = E + (int64_t)tok * d;
+        for (int t = 0; t < d / 128; ++t) {
+            const int f = t * 128 + threadIdx.x;
+            const float x = bf16_to_f32(er[f]);
+            x_f32[(int64_t)r * d + f] = x;
+            xg[(int64_t)r * d + f] = f32_to_bf16(x * bf16_to_f32(g[f]));
+            const float s = warp_sum(x * x);
+            if ((threadIdx.x & 31) == 0) red[threadIdx.x >> 5] = s;
+            __syncthreads();
+            if (threadIdx.x == 0) ssq[(int64_t)t * rows_cap + r] = red[0] + red[1] + red[2] + red[3];
+            __syncthreads();
+        }
+    }
+}
+
+// Copy every layer's prompt KV (positions < Lp - 1) from prompt slot seq_pslot[s] into
+// rollout slot s, for s < live (run once at a round start).
+static __global__ void kv_fanout_kernel(const uint16_t *pkv, uint16_t *kv, const StepPtrs c, int layers, int n_kv,
+                                        int hd, int cap_p, int cap_s, int max_active, int max_seqs) {
+    pdl_wait_prior_grids();
+    pdl_allow_dependents();
+    const int live = c.v->live;
+    const int Lpre = c.kc->Lp - 1;
+    const int vec_per_row = hd / 8;  // 16-byte vectors per position
+    const int64_t per_plane = (int64_t)Lpre * vec_per_row;
+    const int64_t per_slot = 2LL * n_kv * per_plane;
+    const int64_t total = (int64_t)layers * live * per_slot;
+    for (int64_t e = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; e < total; e += (int64_t)gridDim.x * blockDim.x) {
+        const int64_t l = e / ((int64_t)live * per_slot);
+        int64_t rem = e - l * live * per_slot;
+        const int s = (int)(rem / per_slot);
+        rem -= (int64_t)s * per_slot;
+        const int plane = (int)(rem / per_plane);  // 0 .. 2*n_kv-1
+        rem -= (int64_t)plane * per_plane;
+        const int pos = (int)(rem / vec_per_row), v = (int)(rem % vec_per_row);
+        const int ps = c.seq_pslot[s];
+        const uint4 *src =
+            reinterpret_cast<const uint4 *>(pkv + (((l * max_active + ps) * 2LL * n_kv + plane) * cap_p + pos) * hd) + v;
+        uint4 *dst = reinterpret_cast<uint4 *>(kv + (((l * max_seqs + s) * 2LL * n_kv + plane) * cap_s + pos) * hd) + v;
+        *dst = *src;
+    }
+}
+
+// 256-thread exclusive scan helper (blockDim.x == 256): returns the prefix, sets total.
+__device__ __forceinline__ int scan256(int v, int &total, int *warp_tot) {
+    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+    int x = v;
+#pragma unroll
+    for (int o = 1; o < 32; o <<= 1) {
+        const int y = __shfl_up_sync(0xffffffffu, x, o);
+        if (lane >= o) x += y;
+    }
+    if (lane == 31) warp_tot[warp] = x;
+    __syncthreads();
+    int before = 0, tot = 0;
+    for (int w = 0; w < 8; ++w) {
+        if (w < warp) before += warp_tot[w];
+        tot += warp_tot[w];
+    }
+    __syncthreads();
+    total = tot;
+    return before + x - v;
+}
+
+// Sampling reduction + step bookkeeping.  CTA r < live reduces row r's lm_head partial
+// argmax over the vocabulary tiles (ties: lowest token id).  The last CTA to finish then
+// appends each row's token to its rollout, retires rollouts that reached their length,
+// compacts the live rows (order kept) and writes the next step's rows and attention items.
+static __global__ void __launch_bounds__(256) sample_finish_kernel(StepPtrs c) {
+    __shared__ float sv[8];
+    __shared__ int si[8];
+    __shared__ int s_last;
+    __shared__ int warp_tot[8];
+    pdl_wait_prior_grids();
+    pdl_allow_dependents();
+    StepVars &V = *c.v;
+    const int live = V.live;
+    const int r = blockIdx.x;
+    const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+    if (r < live) {
+        float best = -INFINITY;
+        int bi = 0x7fffffff;
+        for (int t = tid; t < c.lm_tiles; t += blockDim.x) {
+            const float v = __ldcg(&c.arg_val[(int64_t)r * c.lm_tiles + t]);
+            const int i = __ldcg(&c.arg_idx[(int64_t)r * c.lm_tiles + t]);
+            if (v > best || (v == best && i < bi)) { best = v; bi = i; }
+        }
+#pragma unroll
+        for (int o = 16; o > 0; o >>= 1) {
+            const float ob = __shfl_xor_sync(0xffffffffu, best, o);
+            const int oi = __shfl_xor_sync(0xffffffffu, bi, o);
+            if (ob > best || (ob == best && oi < bi)) { best = ob; bi = oi; }
+        }
+        if (lane == 0) { sv[warp] = best; si[warp] = bi; }
+        __syncthreads();
+        if (tid == 0) {
+            for (int w = 1; w < 8; ++w)
+                if (sv[w] > best || (sv[w] == best && si[w] < bi)) { best = sv[w]; bi = si[w]; }
+            c.sampled[r] = bi;
+        }
+    }
+    __threadfence();
+    __syncthreads();
+    if (tid == 0) {
+        const int old = atomicAdd(&V.fin_count, 1);
+        s_last = (old == (int)gridDim.x - 1);
+    }
+    __syncthreads();
+    if (!s_last) return;
+    __threadfence();
+    if (tid == 0) V.fin_count = 0;
+    if (live == 0) return;
+    const StepConst &K = *c.kc;
+    const int Lp = K.Lp;
+    // bookkeeping over the live rows (several passes of 256)
+    int out = 0;
+    for (int base = 0; base < live; base += 256) {
+        const int i = base + tid;
+        int keep = 0, slot = 0, gen = 0, next_tok = 0;
+        if (i < live) {
+            slot = c.row_slot[i];
+            gen = c.seq_gen[slot];
+            const int tok = __ldcg(&c.sampled[i]);
+            if (K.teacher) {
+                c.sampled_out[(int64_t)slot * K.T_forced + gen] = tok;
+                next_tok = (gen + 1 < K.T_forced) ? c.forced[(int64_t)slot * K.T_forced + gen] : 0;
+            } else {
+                c.gen_tok[((int64_t)c.seq_q[slot] * K.k + c.seq_j[slot]) * K.max_gen + gen] = tok;
+                next_tok = tok;
+            }
+            gen += 1;
+            c.seq_gen[slot] = gen;
+            keep = gen < c.seq_len[slot];
+        }
+        // stable in-place compaction: a kept row lands at or before its own index
+        int tot;
+        const int before = scan256(keep, tot, warp_tot);
+        if (keep) {
+            const int dst = out + before;
+            c.row_slot[dst] = slot;
+            c.row_pos[dst] = Lp - 1 + gen;
+            c.row_tok[dst] = next_tok;
+            c.row_seed[dst] = sampler_row_seed(K.sample_seed, c.seq_uid[slot], gen);
+        }
+        __syncthreads();
+        out += tot;
+    }
+    // attention items of the next step
+    int items = 0;
+    for (int base = 0; base < out; base += 256) {
+        const int i = base + tid;
+        const int ns = (i < out) ? (c.row_pos[i] + 1 + K.attn_chunk - 1) / K.attn_chunk : 0;
+        int tot;
+        const int before = scan256(ns, tot, warp_tot);
+        if (i < out) {
+            const int i0 = items + before;
+            c.row_item0[i] = i0;
+            for (int sp = 0; sp < ns; ++sp) {
+                if (i0 + sp < c.att_cap) c.att_items[i0 + sp] = make_int2(i, sp);
+                else report_error(&V.err, ERR_CAPACITY);
+            }
+        }
+        items += tot;
+    }
+    if (tid == 0) {
+        V.live = out;
+        V.att_items = min(items, c.att_cap);
+        V.exec_steps += 1;
+        V.round_steps += 1;
+    }
+}
+
+// Teacher forcing: n rollouts, rollout i uses prompt slot i and rollout slot i, lengths T.
+static __global__ void __launch_bounds__(kCtlThreads, 1) teacher_setup_kernel(StepPtrs c, int n, const int64_t *uid) {
+    pdl_wait_prior_grids();
+    const StepConst &K = *c.kc;
+    StepVars &V = *c.v;
+    const int Lp = K.Lp, Lpre = Lp - 1;
+    const int nsplit = (Lp + K.attn_chunk - 1) / K.attn_chunk;
+    for (int r = threadIdx.x; r < n; r += kCtlThreads) {
+        c.seq_q[r] = r;
+        c.seq_j[r] = 0;
+        c.seq_len[r] = K.T_forced;
+        c.seq_gen[r] = 0;
+        c.seq_pslot[r] = r;
+        c.seq_uid[r] = uid[r];
+        c.row_slot[r] = r;
+        c.row_pos[r] = Lp - 1;
+        c.row_tok[r] = c.p_tok[(int64_t)r * Lp + Lp - 1];
+        c.row_seed[r] = sampler_row_seed(K.sample_seed, uid[r], 0);
+        c.row_item0[r] = r * nsplit;
+        for (int sp = 0; sp < nsplit; ++sp) c.att_items[r * nsplit + sp] = make_int2(r, sp);
+    }
+    for (int r = threadIdx.x; r < n * Lpre; r += kCtlThreads) {
+        const int f = r / Lpre, t = r - f * Lpre;
+        c.pre_slot[r] = f;
+        c.pre_pos[r] = t;
+        c.pre_tok[r] = c.p_tok[(int64_t)f * Lp + t];
+        c.pre_items[r] = make_int2(r, 0);
+        c.pre_item0[r] = r;
+    }
+    if (threadIdx.x == 0) {
+        StepVars z;
+        memset(&z, 0, sizeof(z));
+        z.round = 0;
+        z.live = n;
+        z.att_items = n * nsplit;
+        z.pre_rows = n * Lpre;
+        z.n_fresh = n;
+        z.round_maxL = K.T_forced;
+        V = z;
+    }
+}
+
+// Gumbel-max over given fp32 logits (kernel-level entry point): one CTA per row.
+static __global__ void __launch_bounds__(256) sample_rows_kernel(const float *logits, int V, uint64_t sample_seed,
+                                                                 const int64_t *uid, const int *t, int *token) {
+    __shared__ float sv[8];
+    __shared__ int si[8];
+    const int r = blockIdx.x;
+    const uint64_t rs = sampler_row_seed(sample_seed, uid[r], t[r]);
+    float best = -INFINITY;
+    int bi = 0x7fffffff;
+    for (int v = threadIdx.x; v < V; v += blockDim.x) {
+        const float z = logits[(int64_t)r * V + v] + gumbel_from_hash(splitmix_at(rs, (uint64_t)v + 1));
+        if (z > best) { best = z; bi = v; }
+    }
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) {
+        const float ob = __shfl_xor_sync(0xffffffffu, best, o);
+        const int oi = __shfl_xor_sync(0xffffffffu, bi, o);
+        if (ob > best || (ob == best && oi < bi)) { best = ob; bi = oi; }
+    }
+    if ((threadIdx.x & 31) == 0) { sv[threadIdx.x >> 5] = best; si[threadIdx.x >> 5] = bi; }
+    __syncthreads();
+    if (threadIdx.x == 0) {
+        for (int w = 1; w < 8; ++w)
+            if (sv[w] > best || (sv[w] == best && si[w] < bi)) { best = sv[w]; bi = si[w]; }
+        token[r] = bi;
+    }
+}
+
+}  // namespace sara

@@ -1,0 +1,84 @@
+// Device-resident state of one rollout-collection step: per-call constants, scalar
+// progress variables, and the pointers every step kernel reads.  The whole step runs as
+// one CUDA graph whose kernels take their sizes (live rows, items, prefill rows) from here.
+#pragma once
+#include <stdint.h>
+
+namespace sara {
+
+enum : uint8_t { ST_UNDRAWN = 0, ST_ACTIVE = 1, ST_COMMITTED = 2, ST_ABANDONED = 3, ST_INCOMPLETE = 4 };
+enum : uint8_t { D_CONTINUE = 0, D_COMMIT = 1, D_ABANDON = 2 };
+
+constexpr int kMaxK = 64;
+constexpr int kTabDim = kMaxK + 1;  // tables indexed [n][s], 0 <= s <= n <= k
+
+// Per-call constants (host -> device before the graph launch).
+struct StepConst {
+    int32_t P, Lp, k, n0, commit_min, a0, b0, B;
+    int64_t N, tau_num, tau_den;
+    uint64_t reward_seed, sample_seed;
+    int32_t decode;       // 1: decode every issued rollout; 0: controller only
+    int32_t teacher;      // 1: teacher forcing (one round, forced tokens)
+    int32_t T_forced;     // teacher: generated tokens per rollout
+    int32_t max_gen;      // stride of the generated-token output
+    int32_t attn_chunk;   // decode attention positions per split
+    int32_t pad_;
+};
+
+// Scalar progress of the step (device, reset by the init kernel).
+struct StepVars {
+    int32_t live;          // live decode rows
+    int32_t att_items;     // decode attention work items
+    int32_t pre_rows;      // prefill rows (fresh prompts x (Lp - 1))
+    int32_t n_fresh;
+    int32_t done;
+    int32_t round;         // index of the round in flight (-1 before the probe)
+    int32_t round_maxL;    // longest rollout of the round in flight
+    int32_t round_steps;   // decode steps run in the round in flight
+    int32_t n_act, n_iss;
+    int32_t err;
+    int32_t fin_count;     // arrival counter of the sample/finish kernel
+    int32_t iters;         // loop iterations
+    int32_t pad_;
+    int64_t used, C, cursor, drawn, gen_tokens, sched_steps, exec_steps, rounds_done;
+};
+
+struct StepPtrs {
+    StepConst *kc;
+    StepVars *v;
+    // prompt pool
+    const int32_t *p_tok;      // [P][Lp]
+    const uint64_t *p_thr;     // [P]
+    const int32_t *p_len;      // [P][k]
+    // per prompt
+    uint8_t *q_status, *q_n, *q_s;
+    int16_t *q_round;
+    int32_t *q_pslot;
+    // working lists
+    int32_t *act, *act_tmp, *iss_q, *iss_c, *fresh_pslot;
+    // exact decision / priority tables
+    uint8_t *dec_tab, *rank_tab;
+    // sequences (slots)
+    int32_t *seq_q, *seq_j, *seq_len, *seq_gen, *seq_pslot;
+    int64_t *seq_uid;
+    // decode rows of the next step
+    int32_t *row_slot, *row_pos, *row_tok, *row_item0;
+    uint64_t *row_seed;
+    int2 *att_items;
+    int32_t *sampled;          // [max_seqs] token drawn for each row
+    // prefill rows of the round
+    int32_t *pre_slot, *pre_pos, *pre_tok, *pre_item0;
+    int2 *pre_items;
+    // outputs
+    int32_t *gen_tok;          // [P][k][max_gen]
+    // teacher forcing
+    const int32_t *forced;     // [n][T]
+    int32_t *sampled_out;      // [n][T]
+    // lm_head partial argmax
+    const float *arg_val;
+    const int32_t *arg_idx;
+    int32_t lm_tiles;
+    int32_t max_seqs, max_active, pre_cap, att_cap;
+};
+
+}  // namespace sara

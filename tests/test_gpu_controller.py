@@ -1,0 +1,66 @@
+"""The on-device controller (controller-only handle, no decode) against the Algorithm 1
+oracle: every prompt's outcome, n, s and decision round, and every counter, bit-exact."""
+import numpy as np
+import pytest
+
+import synth
+from oracle import controller as oc
+
+pytestmark = pytest.mark.gpu
+
+
+@pytest.fixture(scope="module")
+def handle():
+    import __graft_entry__
+    __graft_entry__.build()
+    import paper_2607_26253_gb300 as pkg
+    cfg = pkg.model_cfg(None, max_prompts=65536, max_active=8192, max_seqs=1, max_prompt_len=1, max_gen_len=1,
+                        max_k=16)
+    with pkg.Handle(cfg) as h:
+        yield h
+
+
+def _compare(h, w, si=None):
+    si = si or synth.step_inputs(w)
+    ref = oc.collect_workload(w, si)
+    out = h.collect_step(thresholds=si.thresholds, lengths=si.lengths, N=w.budget_N, k=w.k, n0=w.n0, tau=w.tau,
+                         target_B=w.target_B, reward_seed=w.reward_seed, prompt_len=w.prompt_len,
+                         commit_min=w.commit_floor, prior=w.prior)
+    assert np.array_equal(out.status, ref.status)
+    assert np.array_equal(out.n, ref.n)
+    assert np.array_equal(out.s, ref.s)
+    assert np.array_equal(out.decided_round, ref.decided_round)
+    for key, v in ref.counters.items():
+        assert out.counters[key] == v, (key, out.counters[key], v)
+    return out
+
+
+@pytest.mark.parametrize("k", synth.SWEEP_K)
+@pytest.mark.parametrize("n0", synth.SWEEP_N0)
+def test_sweep_grid_bit_exact(handle, k, n0):
+    for tau in synth.SWEEP_TAU:
+        for rep in range(3):
+            _compare(handle, synth.sweep_workload(k, n0, tau, rep))
+
+
+def test_budget_binding_priority_and_edge_cases(handle):
+    rng = np.random.default_rng(7)
+    for it in range(60):
+        k = int(rng.integers(2, 17))
+        n0 = int(rng.integers(1, k + 1))
+        P = int(rng.integers(1, 3000))
+        B = int(rng.integers(1, min(P, 8192) + 1))
+        w = synth.Workload("edge", None, n_prompts=P, prompt_len=int(rng.integers(1, 5)), target_B=B, k=k, n0=n0,
+                           tau=float(rng.choice([0.0, 0.3, 0.45, 0.6, 1.0])), budget_N=int(rng.integers(0, 4 * P)),
+                           commit_min=int(rng.integers(2, k + 1)),
+                           prior=(int(rng.integers(1, 9)), int(rng.integers(1, 9))),
+                           lengths=synth.Lengths("uniform", lo=1, hi=50),
+                           seed_latent=it, seed_lengths=it + 1, reward_seed=it + 2)
+        _compare(handle, w)
+
+
+def test_working_set_equal_to_pool(handle):
+    # B = P: the probe round spends the budget (B k > N) and no group reaches the commit floor
+    w = synth.sweep_workload(8, 2, 0.45, 0, n_prompts=8192, target_B=8192)
+    out = _compare(handle, w)
+    assert out.counters["committed"] == 0
