@@ -172,6 +172,19 @@ SARA_API int sara_teacher_force(sara_handle *h, int32_t n_seq, int32_t prompt_le
                                 const int64_t *uid, uint64_t sample_seed, float *logits,
                                 int32_t *sampled, int32_t on_device);
 
+/*
+ * Profiling hook (benchmarks): set `rows` live rollouts at context length `ctx` (synthetic
+ * row state; the step's own state is overwritten) and launch `iters` times, after two
+ * warm-up launches, either one decode kernel of layer 0 or the whole decode step, timing
+ * them with CUDA events on the handle's stream.  *ms_per_launch = elapsed / iters.
+ *   kernel: 0 = whole decode step (eager launches), 1 = QKV projection + RoPE + KV append,
+ *           2 = decode attention, 3 = O projection + residual, 4 = gate/up + SwiGLU,
+ *           5 = down projection + residual, 6 = lm_head + fused sampling partials.
+ * Requires 1 <= rows <= max_seqs, ctx >= 2 and room for the positions the launches use.
+ */
+SARA_API int sara_profile(sara_handle *h, int32_t kernel, int32_t rows, int32_t ctx, int32_t iters,
+                          double *ms_per_launch);
+
 /* Message for the last error on this handle (or of sara_create when h == NULL). */
 SARA_API const char *sara_last_error(const sara_handle *h);
 

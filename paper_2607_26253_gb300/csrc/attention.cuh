@@ -7,7 +7,8 @@
 // the G = n_heads / n_kv query heads that share the KV head once and streams the split's K
 // and V rows (256 contiguous bytes each at hd = 128) exactly once with 16-byte loads.  Each
 // half-warp owns one position at a time, each lane hd/16 dimensions; scores are reduced
-// with xor-shuffles inside the half-warp and folded into an online softmax (base-2,
+// with xor-shuffles inside the half-warp (the warp's two halves always iterate together)
+// and folded into an online softmax (base-2,
 // exp2f) four positions at a time.  The 8 half-warp states are merged in shared memory;
 // rows with several splits write fp32 partials and the last split to arrive (per-row
 // counter, no spinning) merges them in split order.
@@ -87,7 +88,10 @@ attn_rows_kernel(AttnParams p) {
             for (int d = 0; d < DPL; ++d) o[g][d] = 0.f;
         }
 
-        for (int base = p0 + hw * kAttnPPI; base < p1; base += 8 * kAttnPPI) {
+        // The trip count is uniform across the warp (both half-warps iterate together) because
+        // the score reduction below uses full-warp shuffles; positions past p1 are masked.
+        for (int wbase = p0 + warp * 2 * kAttnPPI; wbase < p1; wbase += 8 * kAttnPPI) {
+            const int base = wbase + half * kAttnPPI;
             float kf[kAttnPPI][DPL], vf[kAttnPPI][DPL];
             bool valid[kAttnPPI];
 #pragma unroll

@@ -170,25 +170,22 @@ GemmParams gemm_base(const sara_handle &h, int m_tiles, int k_chunks, const Acts
     return p;
 }
 
-// One forward pass over a row set (decode: live rollouts, KV = rollout slots, lm_head +
-// fused sampling at the end; prefill: fresh prompt tokens, KV = prompt slots, stops after
-// the last layer's K/V).  The first kernel of the sequence is launched without PDL.
-void enqueue_forward(sara_handle &h, cudaStream_t s, bool decode, bool pdl, float *logits_stage) {
+enum Kern { K_QKV = 1, K_ATTN = 2, K_OPROJ = 3, K_GATEUP = 4, K_DOWN = 5, K_LMHEAD = 6 };
+
+// Launch one projection / attention kernel of layer l for a row set (decode: live rollouts,
+// KV = rollout slots; prefill: fresh prompt tokens, KV = prompt slots).
+void enqueue_kernel(sara_handle &h, cudaStream_t s, bool decode, int which, int l, bool pdl, float *logits_stage) {
     const sara_model_cfg &m = h.cfg;
     const StepPtrs &c = h.ptrs;
     Acts &A = decode ? h.dec : h.pre;
     const int *rows_dev = decode ? &h.vars->live : &h.vars->pre_rows;
     const int d = m.d_model, H = m.n_heads, KVH = m.n_kv_heads, hd = m.head_dim, F = m.ffn;
-    const int qkv_out = (H + 2 * KVH) * hd;
     const int G = h.sms;
-    launch(s, false, dim3(A.rows_cap), dim3(128), 0, embed_kernel, (const uint16_t *)h.embed,
-           (const uint16_t *)h.attn_norm[0], rows_dev, decode ? (const int *)c.row_tok : (const int *)c.pre_tok, d,
-           A.rows_cap, m.vocab, A.x_f32, A.xg, A.ssq_a, &h.vars->err);
-    for (int l = 0; l < m.layers; ++l) {
-        const bool last = l == m.layers - 1;
-        uint16_t *kv_l = decode ? h.kv_seq + l * h.kv_seq_layer : h.kv_pr + l * h.kv_pr_layer;
-        {
-            GemmParams p = gemm_base(h, qkv_out / 128, d / 64, A, rows_dev, decode);
+    const bool last = l == m.layers - 1;
+    uint16_t *kv_l = decode ? h.kv_seq + l * h.kv_seq_layer : h.kv_pr + l * h.kv_pr_layer;
+    switch (which) {
+        case K_QKV: {
+            GemmParams p = gemm_base(h, (H + 2 * KVH) * hd / 128, d / 64, A, rows_dev, decode);
             p.ssq = A.ssq_a;
             p.q_out = A.q;
             p.n_heads = H;
@@ -201,9 +198,9 @@ void enqueue_forward(sara_handle &h, cudaStream_t s, bool decode, bool pdl, floa
             p.kv_slot_stride = decode ? h.kv_seq_slot : h.kv_pr_slot;
             p.kv_cap = decode ? h.cap_s : h.cap_p;
             launch_gemm<EPI_QKV>(s, pdl, G, h.tm_qkv[l], A.tm_xg, p);
+            break;
         }
-        if (!decode && last) break;  // the prompt's last hidden state is not needed
-        {
+        case K_ATTN: {
             AttnParams a{};
             a.q = A.q;
             a.out = A.att;
@@ -223,8 +220,9 @@ void enqueue_forward(sara_handle &h, cudaStream_t s, bool decode, bool pdl, floa
             a.cnt = h.attn_cnt;
             a.err = &h.vars->err;
             launch_attention(s, pdl, h.sms, hd, a);
+            break;
         }
-        {
+        case K_OPROJ: {
             GemmParams p = gemm_base(h, d / 128, H * hd / 64, A, rows_dev, decode);
             p.x_f32 = A.x_f32;
             p.xg_out = A.xg;
@@ -232,15 +230,17 @@ void enqueue_forward(sara_handle &h, cudaStream_t s, bool decode, bool pdl, floa
             p.ssq_out = A.ssq_m;
             p.ld = d;
             launch_gemm<EPI_RESID>(s, pdl, G, h.tm_o[l], A.tm_att, p);
+            break;
         }
-        {
+        case K_GATEUP: {
             GemmParams p = gemm_base(h, 2 * F / 128, d / 64, A, rows_dev, decode);
             p.ssq = A.ssq_m;
             p.h_out = A.h;
             p.ld = F;
             launch_gemm<EPI_SWIGLU>(s, pdl, G, h.tm_gu[l], A.tm_xg, p);
+            break;
         }
-        {
+        case K_DOWN: {
             GemmParams p = gemm_base(h, d / 128, F / 64, A, rows_dev, decode);
             p.x_f32 = A.x_f32;
             p.xg_out = A.xg;
@@ -248,19 +248,44 @@ void enqueue_forward(sara_handle &h, cudaStream_t s, bool decode, bool pdl, floa
             p.ssq_out = A.ssq_a;
             p.ld = d;
             launch_gemm<EPI_RESID>(s, pdl, G, h.tm_down[l], A.tm_h, p);
+            break;
         }
+        case K_LMHEAD: {
+            GemmParams p = gemm_base(h, m.vocab / 128, d / 64, A, rows_dev, true);
+            p.ssq = A.ssq_a;
+            p.y_f32 = logits_stage;
+            p.ld = m.vocab;
+            p.row_seed = c.row_seed;
+            p.arg_val = h.lm_val;
+            p.arg_idx = h.lm_idx;
+            launch_gemm<EPI_LMHEAD>(s, pdl, G, h.tm_lm, A.tm_xg, p);
+            break;
+        }
+        default: throw SaraError(SARA_EINVAL, "unknown kernel id");
+    }
+}
+
+// One forward pass over a row set: embedding, every layer, and (decode) lm_head with fused
+// sampling followed by the step bookkeeping.  Prefill stops after the last layer's K/V.
+// The first kernel of the sequence is launched without PDL.
+void enqueue_forward(sara_handle &h, cudaStream_t s, bool decode, bool pdl, float *logits_stage) {
+    const sara_model_cfg &m = h.cfg;
+    const StepPtrs &c = h.ptrs;
+    Acts &A = decode ? h.dec : h.pre;
+    const int *rows_dev = decode ? &h.vars->live : &h.vars->pre_rows;
+    launch(s, false, dim3(A.rows_cap), dim3(128), 0, embed_kernel, (const uint16_t *)h.embed,
+           (const uint16_t *)h.attn_norm[0], rows_dev, decode ? (const int *)c.row_tok : (const int *)c.pre_tok,
+           m.d_model, A.rows_cap, m.vocab, A.x_f32, A.xg, A.ssq_a, &h.vars->err);
+    for (int l = 0; l < m.layers; ++l) {
+        enqueue_kernel(h, s, decode, K_QKV, l, pdl, nullptr);
+        if (!decode && l == m.layers - 1) break;  // the prompt's last hidden state is not needed
+        enqueue_kernel(h, s, decode, K_ATTN, l, pdl, nullptr);
+        enqueue_kernel(h, s, decode, K_OPROJ, l, pdl, nullptr);
+        enqueue_kernel(h, s, decode, K_GATEUP, l, pdl, nullptr);
+        enqueue_kernel(h, s, decode, K_DOWN, l, pdl, nullptr);
     }
     if (!decode) return;
-    {
-        GemmParams p = gemm_base(h, m.vocab / 128, d / 64, A, rows_dev, true);
-        p.ssq = A.ssq_a;
-        p.y_f32 = logits_stage;
-        p.ld = m.vocab;
-        p.row_seed = c.row_seed;
-        p.arg_val = h.lm_val;
-        p.arg_idx = h.lm_idx;
-        launch_gemm<EPI_LMHEAD>(s, pdl, G, h.tm_lm, A.tm_xg, p);
-    }
+    enqueue_kernel(h, s, true, K_LMHEAD, m.layers - 1, pdl, logits_stage);
     launch(s, pdl, dim3(A.rows_cap), dim3(256), 0, sample_finish_kernel, c);
 }
 
@@ -714,6 +739,68 @@ void teacher_impl(sara_handle &h, int n, int Lp, const int32_t *prompts, int T, 
     if (v.live != 0 || v.exec_steps != T) throw SaraError(SARA_EDEVICE, "teacher forcing ran an unexpected number of steps");
 }
 
+// Profiling hook: `rows` live rollouts at context `ctx` (synthetic row state), `iters` launches
+// of one kernel of layer 0 (or of the whole eager decode step, kernel 0) timed with CUDA
+// events on the handle's stream after two warm-up launches.
+void profile_impl(sara_handle &h, int which, int rows, int ctx, int iters, double *ms) {
+    const sara_model_cfg &m = h.cfg;
+    if (!h.has_model) throw SaraError(SARA_EINVAL, "profiling needs a model");
+    if (which < 0 || which > K_LMHEAD) throw SaraError(SARA_EINVAL, "unknown kernel id");
+    if (rows < 1 || rows > m.max_seqs || iters < 1 || !ms) throw SaraError(SARA_EINVAL, "rows / iters out of range");
+    const int steps = which == 0 ? iters + 2 : 0;  // the whole step advances positions
+    if (ctx < 2 || ctx + steps + 1 > h.cap_s || steps + 1 > m.max_gen_len) throw SaraError(SARA_EINVAL, "ctx out of range");
+    cudaStream_t s = h.stream;
+    StepConst K{};
+    K.P = 1; K.Lp = ctx; K.k = 2; K.n0 = 1; K.commit_min = 2; K.a0 = 1; K.b0 = 1; K.B = 1; K.N = 1;
+    K.tau_num = 0; K.tau_den = 1; K.decode = 1; K.max_gen = m.max_gen_len; K.attn_chunk = kDecodeChunk;
+    const int nsplit = (ctx + kDecodeChunk - 1) / kDecodeChunk;
+    std::vector<int> slot(rows), pos(rows, ctx - 1), tok(rows, 0), item0(rows), zero(rows, 0), len(rows, m.max_gen_len);
+    std::vector<uint64_t> seed(rows);
+    std::vector<int64_t> uid(rows);
+    std::vector<int2> items;
+    for (int r = 0; r < rows; ++r) {
+        slot[r] = r;
+        item0[r] = r * nsplit;
+        seed[r] = 0x9E3779B97F4A7C15ull * (r + 1);
+        uid[r] = r;
+        for (int sp = 0; sp < nsplit; ++sp) items.push_back(make_int2(r, sp));
+    }
+    StepVars v{};
+    v.live = rows;
+    v.att_items = rows * nsplit;
+    v.round_maxL = 1 << 30;
+    const StepPtrs &c = h.ptrs;
+    CK(cudaMemcpyAsync(h.kc, &K, sizeof(K), cudaMemcpyHostToDevice, s));
+    CK(cudaMemcpyAsync(h.vars, &v, sizeof(v), cudaMemcpyHostToDevice, s));
+    CK(cudaMemcpyAsync(c.row_slot, slot.data(), rows * 4, cudaMemcpyHostToDevice, s));
+    CK(cudaMemcpyAsync(c.row_pos, pos.data(), rows * 4, cudaMemcpyHostToDevice, s));
+    CK(cudaMemcpyAsync(c.row_tok, tok.data(), rows * 4, cudaMemcpyHostToDevice, s));
+    CK(cudaMemcpyAsync(c.row_item0, item0.data(), rows * 4, cudaMemcpyHostToDevice, s));
+    CK(cudaMemcpyAsync(c.row_seed, seed.data(), rows * 8, cudaMemcpyHostToDevice, s));
+    CK(cudaMemcpyAsync(c.att_items, items.data(), items.size() * sizeof(int2), cudaMemcpyHostToDevice, s));
+    CK(cudaMemcpyAsync(c.seq_q, zero.data(), rows * 4, cudaMemcpyHostToDevice, s));
+    CK(cudaMemcpyAsync(c.seq_j, zero.data(), rows * 4, cudaMemcpyHostToDevice, s));
+    CK(cudaMemcpyAsync(c.seq_gen, zero.data(), rows * 4, cudaMemcpyHostToDevice, s));
+    CK(cudaMemcpyAsync(c.seq_len, len.data(), rows * 4, cudaMemcpyHostToDevice, s));
+    CK(cudaMemcpyAsync(c.seq_uid, uid.data(), rows * 8, cudaMemcpyHostToDevice, s));
+    CK(cudaStreamSynchronize(s));
+    auto one = [&] {
+        if (which == 0) enqueue_forward(h, s, true, h.use_pdl, nullptr);
+        else enqueue_kernel(h, s, true, which, 0, false, nullptr);
+    };
+    one();
+    one();
+    CK(cudaEventRecord(h.ev0, s));
+    for (int i = 0; i < iters; ++i) one();
+    CK(cudaEventRecord(h.ev1, s));
+    CK(cudaStreamSynchronize(s));
+    float t = 0.f;
+    CK(cudaEventElapsedTime(&t, h.ev0, h.ev1));
+    CK(cudaMemcpy(&v, h.vars, sizeof(v), cudaMemcpyDeviceToHost));
+    check_step_error(v);
+    *ms = (double)t / iters;
+}
+
 int guard(sara_handle *h, const std::function<void()> &fn) {
     try {
         fn();
@@ -767,6 +854,11 @@ int sara_teacher_force(sara_handle *h, int32_t n_seq, int32_t prompt_len, const 
     return guard(h, [&] {
         teacher_impl(*h, n_seq, prompt_len, prompts, T, forced, uid, sample_seed, logits, sampled, on_device);
     });
+}
+
+int sara_profile(sara_handle *h, int32_t kernel, int32_t rows, int32_t ctx, int32_t iters, double *ms_per_launch) {
+    if (!h) return SARA_EINVAL;
+    return guard(h, [&] { profile_impl(*h, kernel, rows, ctx, iters, ms_per_launch); });
 }
 
 const char *sara_last_error(const sara_handle *h) { return h ? h->err.c_str() : g_create_error.c_str(); }

@@ -20,7 +20,7 @@ SARA_OK, SARA_EINVAL, SARA_ENOMEM, SARA_ETIMEOUT, SARA_EDEVICE = 0, -1, -2, -3, 
 UNDRAWN, COMMITTED, ABANDONED, INCOMPLETE = 0, 2, 3, 4
 EXPORTED = ("sara_create", "sara_collect_step", "sara_teacher_force", "sara_last_error", "sara_destroy",
             "sara_gemm_workspace_bytes", "sara_gemm_bf16", "sara_attention_workspace_bytes",
-            "sara_attention_decode", "sara_sample")
+            "sara_attention_decode", "sara_sample", "sara_profile")
 
 c_p = ctypes.c_void_p
 
@@ -100,6 +100,9 @@ def load(path: str = LIB_PATH):
     lib.sara_attention_decode.restype = ctypes.c_int
     lib.sara_sample.argtypes = [c_p, ctypes.c_int32, ctypes.c_int32, ctypes.c_uint64, c_p, c_p, c_p, c_p]
     lib.sara_sample.restype = ctypes.c_int
+    lib.sara_profile.argtypes = [c_p, ctypes.c_int32, ctypes.c_int32, ctypes.c_int32, ctypes.c_int32,
+                                 ctypes.POINTER(ctypes.c_double)]
+    lib.sara_profile.restype = ctypes.c_int
     if path == LIB_PATH:
         _lib = lib
     return lib
@@ -231,6 +234,12 @@ class Handle:
                                         ctypes.byref(res)), self._h)
         counters = {name: int(getattr(res, name)) for name in COUNTERS}
         return StepOutput(status, n, s, rnd, toks, counters, float(res.device_ms))
+
+    def profile(self, kernel: int, rows: int, ctx: int, iters: int = 20) -> float:
+        """Milliseconds per launch of one decode kernel (see sara_profile in include/sara.h)."""
+        ms = ctypes.c_double()
+        _check(load().sara_profile(self._h, kernel, rows, ctx, iters, ctypes.byref(ms)), self._h)
+        return ms.value
 
     def teacher_force(self, prompts: np.ndarray, forced: np.ndarray, uids: np.ndarray, sample_seed: int):
         """Logits [n, T, V] (fp32) and sampled tokens [n, T] of teacher-forced decode steps."""
