@@ -43,6 +43,11 @@ def parse():
     ap.add_argument("--impl", default="mine", choices=["mine", "reference"])
     ap.add_argument("--workload", default="1.5b", choices=sorted(synth.WORKLOADS))
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--kernel-profile", type=int, default=None, metavar="KERNEL",
+                    help="profiling mode for ncu: launch one decode kernel (sara_profile ids; 0 = whole "
+                         "eager decode step) on a reduced-capacity handle of the workload's shapes")
+    ap.add_argument("--rows", type=int, default=25, help="live rows in --kernel-profile mode")
+    ap.add_argument("--iters", type=int, default=5, help="launches in --kernel-profile mode")
     return ap.parse_args()
 
 
@@ -343,6 +348,24 @@ def read_traffic(workload: str):
     return None
 
 
+# --------------------------------------------------------------------------------- ncu mode
+def run_kernel_profile(args):
+    """Small-footprint run of the real decode kernels for ncu captures: the workload's model
+    shapes with 32 rollout slots of 512 generated positions (a few GB on the device)."""
+    import torch
+
+    import paper_2607_26253_gb300 as pkg
+    torch.cuda.set_device(0)
+    w = synth.WORKLOADS[args.workload]
+    m = w.model
+    weights = synth.model_weights(m, w.weight_seed)
+    cfg = pkg.model_cfg(m, max_prompts=w.n_prompts, max_active=16, max_seqs=32, max_prompt_len=w.prompt_len,
+                        max_gen_len=512, max_k=w.k)
+    with pkg.Handle(cfg, weights, stream=torch.cuda.current_stream()) as h:
+        ms = h.profile(args.kernel_profile, args.rows, w.prompt_len + 128, iters=args.iters)
+    print(json.dumps({"kernel": args.kernel_profile, "rows": args.rows, "ms_per_launch": ms}))
+
+
 # --------------------------------------------------------------------------------- reference arm
 def run_reference(args):
     rank = int(os.environ.get("RANK", "0"))
@@ -375,7 +398,9 @@ def run_reference(args):
 
 if __name__ == "__main__":
     a = parse()
-    if a.impl == "reference":
+    if a.kernel_profile is not None:
+        run_kernel_profile(a)
+    elif a.impl == "reference":
         run_reference(a)
     else:
         run_mine(a)

@@ -63,11 +63,11 @@ def test_tiny_step_schedule_and_tokens(tiny):
             L = int(si.lengths[q, j])
             toks, margins, _ = o2.generate(W, si.tokens[q], L, w.sample_seed, o2.uid_of(int(q), j))
             got = out.tokens[q, j, :L]
-            low = np.nonzero(margins < 2e-2)[0]
+            low = np.nonzero(margins < 1e-2)[0]
             cut = int(low[0]) if low.size else L  # from a near-tie on, the draws may legitimately differ
             assert np.array_equal(got[:cut], toks[:cut]), (q, j, got[:cut + 1], toks[:cut + 1])
             compared += cut
-    assert compared > 0.8 * out.counters["gen_tokens"]
+    assert compared > 0.7 * out.counters["gen_tokens"]
 
 
 def test_tiny_step_is_deterministic_and_reusable(tiny):
