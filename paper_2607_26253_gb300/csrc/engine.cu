@@ -92,6 +92,7 @@ struct sara_handle {
     int32_t *forced = nullptr, *sampled_out = nullptr;
     int64_t *uid_dev = nullptr;
     size_t forced_cap = 0;
+    uint64_t *stamps = nullptr;  // profiling builds: per-CTA phase timestamps of GEMM launches
     // graph
     cudaGraph_t graph = nullptr;
     cudaGraphExec_t exec = nullptr;
@@ -167,6 +168,7 @@ GemmParams gemm_base(const sara_handle &h, int m_tiles, int k_chunks, const Acts
     p.ssq_tiles = h.cfg.d_model / 128;
     p.inv_dim = 1.0f / (float)h.cfg.d_model;
     p.eps = h.cfg.rms_eps;
+    p.stamps = h.stamps;
     return p;
 }
 
@@ -783,6 +785,10 @@ void profile_impl(sara_handle &h, int which, int rows, int ctx, int iters, doubl
     CK(cudaMemcpyAsync(c.seq_gen, zero.data(), rows * 4, cudaMemcpyHostToDevice, s));
     CK(cudaMemcpyAsync(c.seq_len, len.data(), rows * 4, cudaMemcpyHostToDevice, s));
     CK(cudaMemcpyAsync(c.seq_uid, uid.data(), rows * 8, cudaMemcpyHostToDevice, s));
+#ifdef SARA_STAMPS
+    if (!h.stamps) h.stamps = h.mem.alloc<uint64_t>((size_t)h.sms * 8);
+    CK(cudaMemsetAsync(h.stamps, 0, (size_t)h.sms * 8 * 8, s));
+#endif
     CK(cudaStreamSynchronize(s));
     auto one = [&] {
         if (which == 0) enqueue_forward(h, s, true, h.use_pdl, nullptr);
@@ -799,6 +805,23 @@ void profile_impl(sara_handle &h, int which, int rows, int ctx, int iters, doubl
     CK(cudaMemcpy(&v, h.vars, sizeof(v), cudaMemcpyDeviceToHost));
     check_step_error(v);
     *ms = (double)t / iters;
+#ifdef SARA_STAMPS
+    if (h.stamps && which != 0) {  // phase breakdown of the last launch, relative to the earliest entry
+        std::vector<uint64_t> st((size_t)h.sms * 8);
+        CK(cudaMemcpy(st.data(), h.stamps, st.size() * 8, cudaMemcpyDeviceToHost));
+        uint64_t t0 = ~0ull;
+        for (int c = 0; c < h.sms; ++c) t0 = std::min(t0, st[(size_t)c * 8]);
+        for (int i = 0; i < 8; ++i) {
+            std::vector<double> d;
+            for (int c = 0; c < h.sms; ++c)
+                if (st[(size_t)c * 8 + i]) d.push_back((double)(st[(size_t)c * 8 + i] - t0) * 1e-3);
+            std::sort(d.begin(), d.end());
+            if (!d.empty())
+                fprintf(stderr, "stamp %d: n=%zu min %.2f med %.2f max %.2f us\n", i, d.size(), d.front(), d[d.size() / 2],
+                        d.back());
+        }
+    }
+#endif
 }
 
 int guard(sara_handle *h, const std::function<void()> &fn) {

@@ -69,6 +69,7 @@ struct GemmParams {
     uint16_t *h_out;           // EPI_SWIGLU [rows][ld]
     const uint64_t *row_seed;  // EPI_LMHEAD sampler key of the row
     float *arg_val; int *arg_idx;  // EPI_LMHEAD [rows][m_tiles] partial max / argmax
+    uint64_t *stamps;          // optional [gridDim.x][8] phase timestamps (profiling builds)
 };
 
 struct GemmSmem {
@@ -98,6 +99,11 @@ __device__ __forceinline__ int cta_of_unit(int64_t u, int64_t U, int G) {
     while (c > 0 && unit_begin(c, U, G) > u) --c;
     return c;
 }
+#ifdef SARA_STAMPS
+#define GEMM_STAMP(i) do { if (p.stamps) p.stamps[(size_t)blockIdx.x * 8 + (i)] = globaltimer_ns(); } while (0)
+#else
+#define GEMM_STAMP(i) do { } while (0)
+#endif
 __device__ __forceinline__ int64_t min64(int64_t a, int64_t b) { return a < b ? a : b; }
 
 
@@ -227,6 +233,7 @@ gemm_tc_kernel(const __grid_constant__ CUtensorMap tmW, const __grid_constant__ 
     const int G = gridDim.x, cta = blockIdx.x;
 
     if (threadIdx.x == 0) {
+        GEMM_STAMP(0);
         for (int s = 0; s < kGemmStages; ++s) { mbar_init(&S.full[s], 1); mbar_init(&S.empty[s], 1); }
         for (int a = 0; a < 2; ++a) { mbar_init(&S.acc_full[a], 1); mbar_init(&S.acc_empty[a], 4); }
         mbar_init(&S.drain, 1);
@@ -242,6 +249,7 @@ gemm_tc_kernel(const __grid_constant__ CUtensorMap tmW, const __grid_constant__ 
     __syncthreads();
     tc_fence_after();
     const uint32_t tmem = S.tmem_base;
+    if (threadIdx.x == 0) GEMM_STAMP(1);
 
     // Let the next kernel in the stream start its own weight prefetch.
     pdl_allow_dependents();
@@ -341,6 +349,7 @@ gemm_tc_kernel(const __grid_constant__ CUtensorMap tmW, const __grid_constant__ 
                         break;
                     }
                     tc_fence_after();
+                    if (i == 0) GEMM_STAMP(2);
                     const uint32_t aw = smem_u32(sW + (size_t)s * kWStageBytes);
                     const uint32_t ax = smem_u32(sX + (size_t)s * kXStageBytes);
 #pragma unroll
@@ -354,6 +363,7 @@ gemm_tc_kernel(const __grid_constant__ CUtensorMap tmW, const __grid_constant__ 
                 if (*(volatile int *)&S.abort_flag) break;
                 tc_commit(&S.acc_full[a]);
             }
+            GEMM_STAMP(3);
             // every MMA this thread issued has retired before tensor memory is released
             tc_commit(&S.drain);
             mbar_wait(&S.drain, 0, p.err);
@@ -388,6 +398,7 @@ gemm_tc_kernel(const __grid_constant__ CUtensorMap tmW, const __grid_constant__ 
                 break;
             }
             tc_fence_after();
+            if (seg == 0 && etid == 0) GEMM_STAMP(4);
             const bool whole = (kc_first == 0) && (kc_last == kch - 1);
             bool do_epi = whole;
             int c_a = cta, c_b = cta;
@@ -416,6 +427,7 @@ gemm_tc_kernel(const __grid_constant__ CUtensorMap tmW, const __grid_constant__ 
                 do_epi = S.last_flag != 0;
                 __threadfence();
             }
+            if (etid == 0) GEMM_STAMP(5);
             if (do_epi) {
                 if constexpr (EPI == EPI_QKV || EPI == EPI_SWIGLU || EPI == EPI_LMHEAD) {
                     if (etid < rin) {
@@ -454,10 +466,12 @@ gemm_tc_kernel(const __grid_constant__ CUtensorMap tmW, const __grid_constant__ 
         }
     }
 
+    if (threadIdx.x == 64) GEMM_STAMP(6);
     tc_fence_before();
     __syncthreads();
     tc_fence_after();
     if (warp == 1) tmem_dealloc(tmem, 256);
+    if (threadIdx.x == 32) GEMM_STAMP(7);
 }
 
 }  // namespace sara
