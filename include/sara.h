@@ -58,7 +58,7 @@ typedef struct {
     int32_t layers;          /* decoder layers; 0 creates a controller-only handle */
     int32_t d_model;         /* multiple of 128 */
     int32_t n_heads;         /* query heads */
-    int32_t n_kv_heads;      /* key/value heads; n_heads % n_kv_heads == 0, group <= 8 */
+    int32_t n_kv_heads;      /* key/value heads; n_heads / n_kv_heads in {1, 2, 4, 6, 8} */
     int32_t head_dim;        /* 32, 64 or 128 */
     int32_t ffn;             /* SwiGLU width, multiple of 64 */
     int32_t vocab;           /* multiple of 128 */
@@ -68,7 +68,8 @@ typedef struct {
     int32_t max_active;      /* largest target B (working-set size) per step, <= 8192 */
     int32_t max_seqs;        /* largest number of rollouts in one round (>= B * n0), <= 128 */
     int32_t max_prompt_len;  /* largest prompt length Lp */
-    int32_t max_gen_len;     /* largest generated length of one rollout */
+    int32_t max_gen_len;     /* largest generated length of one rollout
+                                (max_prompt_len + max_gen_len <= 12288) */
     int32_t max_k;           /* largest group size k (<= 64) */
 } sara_model_cfg;
 
@@ -201,8 +202,9 @@ SARA_API void sara_destroy(sara_handle *h);
  * tcgen05 MMA with the accumulator in tensor memory, TMA-fed, stream-K over the weight).
  * X: [R][K] bf16, W: [Nout][K] bf16, Y: [R][Nout] fp32, all device, 16-byte aligned.
  * Shapes: 1 <= R <= 128, Nout % 128 == 0, K % 64 == 0, K >= 64.
- * workspace: device scratch of at least sara_gemm_workspace_bytes(R, Nout, K) bytes whose
- * counter area is zero on first use (the kernel leaves it zero again).
+ * workspace: device scratch of at least sara_gemm_workspace_bytes(R, Nout, K) bytes, all zero
+ * on first use (the kernel leaves it zero again): per-CTA fixed-point tile sums and per-tile
+ * arrival counters of the stream-K split.  Calls sharing a workspace must not overlap.
  */
 SARA_API size_t sara_gemm_workspace_bytes(int32_t R, int32_t Nout, int32_t K);
 SARA_API int sara_gemm_bf16(const uint16_t *X, const uint16_t *W, float *Y, int32_t R,
@@ -213,8 +215,9 @@ SARA_API int sara_gemm_bf16(const uint16_t *X, const uint16_t *W, float *Y, int3
  * Decode attention for b sequences, one new query each (softmax(q K^T / sqrt(hd)) V with
  * grouped-query heads): q [b][n_heads][hd] bf16; kv cache of sequence i at kv + i*kv_stride
  * elements, laid out [2 (K,V)][n_kv_heads][cap][hd] bf16, valid for positions < ctx[i];
- * out [b][n_heads][hd] bf16.  Split over the context in chunks of 256 positions with an
- * fp32 log-sum-exp combine.  hd in {32, 64, 128}; n_heads / n_kv_heads <= 8.
+ * out [b][n_heads][hd] bf16.  Split over the context in chunks of 128 positions with an
+ * fp32 log-sum-exp combine.  hd in {32, 64, 128}; n_heads / n_kv_heads in {1, 2, 4, 6, 8};
+ * max_ctx <= 96 * 128.
  * workspace: >= sara_attention_workspace_bytes(b, n_heads, hd, max_ctx), counter area zero.
  */
 SARA_API size_t sara_attention_workspace_bytes(int32_t b, int32_t n_heads, int32_t head_dim,

@@ -5,13 +5,13 @@
 //
 // Work item = (row, split of `chunk` positions) for one KV head (blockIdx.y): the CTA loads
 // the G = n_heads / n_kv query heads that share the KV head once and streams the split's K
-// and V rows (256 contiguous bytes each at hd = 128) exactly once with 16-byte loads.  Each
-// half-warp owns one position at a time, each lane hd/16 dimensions; scores are reduced
-// with xor-shuffles inside the half-warp (the warp's two halves always iterate together)
-// and folded into an online softmax (base-2,
-// exp2f) four positions at a time.  The 8 half-warp states are merged in shared memory;
-// rows with several splits write fp32 partials and the last split to arrive (per-row
-// counter, no spinning) merges them in split order.
+// and V rows (256 contiguous bytes each at hd = 128) exactly once with 16-byte loads, the
+// next iteration's rows in flight while the current ones are used.  Each half-warp owns
+// one position at a time, each lane hd/16 dimensions; scores are reduced with xor-shuffles
+// inside the half-warp (the warp's two halves always iterate together) and folded into an
+// online softmax (base-2, exp2f) four positions at a time.  The 8 half-warp states are
+// merged in shared memory; rows with several splits write fp32 partials and the last split
+// to arrive (per-row counter, no spinning) merges them in split order.
 #pragma once
 #include "device_common.cuh"
 
@@ -19,7 +19,8 @@ namespace sara {
 
 constexpr int kAttnThreads = 128;
 constexpr int kAttnMaxG = 8;
-constexpr int kAttnPPI = 4;  // positions per half-warp per iteration
+constexpr int kAttnPPI = 4;         // positions per half-warp per iteration
+constexpr int kAttnMaxSplits = 96;  // largest split count the merge handles in shared memory
 
 struct AttnParams {
     const uint16_t *q;        // [rows][n_heads][hd]
@@ -40,25 +41,41 @@ struct AttnParams {
     int *err;
 };
 
-template <int HD>
+template <int DPL>
+__device__ __forceinline__ void attn_load_words(const uint16_t *p, uint32_t (&w)[DPL / 2]) {
+    if constexpr (DPL == 8) {
+        const uint4 x = *reinterpret_cast<const uint4 *>(p);
+        w[0] = x.x; w[1] = x.y; w[2] = x.z; w[3] = x.w;
+    } else if constexpr (DPL == 4) {
+        const uint2 x = *reinterpret_cast<const uint2 *>(p);
+        w[0] = x.x; w[1] = x.y;
+    } else {
+        w[0] = *reinterpret_cast<const uint32_t *>(p);
+    }
+}
+
+template <int HD, int G>
 __global__ void __launch_bounds__(kAttnThreads)
 attn_rows_kernel(AttnParams p) {
     constexpr int DPL = HD / 16;  // dims per lane
+    constexpr int NW = DPL / 2;   // packed bf16 words per lane and position
     static_assert(DPL == 2 || DPL == 4 || DPL == 8, "head_dim must be 32, 64 or 128");
-    __shared__ float s_m[8][kAttnMaxG], s_l[8][kAttnMaxG];
-    __shared__ float s_o[8][kAttnMaxG][HD];
-    __shared__ float s_fin_m[kAttnMaxG], s_fin_l[kAttnMaxG];
+    static_assert(G >= 1 && G <= kAttnMaxG, "query group must be 1..8");
+    __shared__ float s_m[8][G], s_l[8][G];
+    __shared__ float s_o[8][G][HD];
+    __shared__ float s_fin_m[G], s_fin_l[G];
+    __shared__ float s_w[G][kAttnMaxSplits];
     __shared__ int s_last;
 
     pdl_wait_prior_grids();
     pdl_allow_dependents();
     const int n_items = p.n_items_dev ? *p.n_items_dev : p.n_items_fixed;
     const int kvh = blockIdx.y;
-    const int G = p.n_heads / p.n_kv;
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const int half = lane >> 4, dl = lane & 15;
     const int hw = warp * 2 + half;  // half-warp id 0..7
     const unsigned fmask = 0xffffffffu;
+    constexpr int kStride = 8 * kAttnPPI;  // positions per CTA iteration
 
     for (int item = blockIdx.x; item < n_items; item += gridDim.x) {
         const int2 it = p.items[item];
@@ -66,67 +83,60 @@ attn_rows_kernel(AttnParams p) {
         const int ctx = p.row_pos[row] + 1;
         const int p0 = split * p.chunk, p1 = min(ctx, p0 + p.chunk);
         const int nsplit = (ctx + p.chunk - 1) / p.chunk;
-        const uint16_t *Kb = p.kv + (int64_t)p.row_slot[row] * p.slot_stride + (int64_t)kvh * p.cap * HD;
+        const uint16_t *Kb = p.kv + (int64_t)p.row_slot[row] * p.slot_stride + (int64_t)kvh * p.cap * HD + dl * DPL;
         const uint16_t *Vb = Kb + (int64_t)p.n_kv * p.cap * HD;
 
         // q slice of every head in the group, pre-scaled by log2(e)/sqrt(hd)
-        float q[kAttnMaxG][DPL];
+        float q[G][DPL];
 #pragma unroll
-        for (int g = 0; g < kAttnMaxG; ++g) {
+        for (int g = 0; g < G; ++g) {
+            uint32_t w[NW];
+            attn_load_words<DPL>(p.q + ((int64_t)row * p.n_heads + kvh * G + g) * HD + dl * DPL, w);
 #pragma unroll
-            for (int d = 0; d < DPL; ++d)
-                q[g][d] = (g < G) ? bf16_to_f32(p.q[((int64_t)row * p.n_heads + kvh * G + g) * HD + dl * DPL + d]) *
-                                        p.scale_log2
-                                  : 0.f;
+            for (int i = 0; i < NW; ++i) {
+                q[g][2 * i] = __uint_as_float(w[i] << 16) * p.scale_log2;
+                q[g][2 * i + 1] = __uint_as_float(w[i] & 0xffff0000u) * p.scale_log2;
+            }
         }
-        float m[kAttnMaxG], l[kAttnMaxG], o[kAttnMaxG][DPL];
+        float m[G], l[G], o[G][DPL];
 #pragma unroll
-        for (int g = 0; g < kAttnMaxG; ++g) {
+        for (int g = 0; g < G; ++g) {
             m[g] = -INFINITY;
             l[g] = 0.f;
 #pragma unroll
             for (int d = 0; d < DPL; ++d) o[g][d] = 0.f;
         }
 
-        // The trip count is uniform across the warp (both half-warps iterate together) because
-        // the score reduction below uses full-warp shuffles; positions past p1 are masked.
-        for (int wbase = p0 + warp * 2 * kAttnPPI; wbase < p1; wbase += 8 * kAttnPPI) {
-            const int base = wbase + half * kAttnPPI;
-            float kf[kAttnPPI][DPL], vf[kAttnPPI][DPL];
-            bool valid[kAttnPPI];
+        // the trip count is uniform across the warp (full-warp shuffles below)
+        const int wstart = p0 + warp * 2 * kAttnPPI;
+        uint32_t kw[kAttnPPI][NW], vw[kAttnPPI][NW];
+        auto load_rows = [&](int wb, uint32_t (&K)[kAttnPPI][NW], uint32_t (&V)[kAttnPPI][NW]) {
 #pragma unroll
             for (int j = 0; j < kAttnPPI; ++j) {
-                const int pp = base + j;
-                valid[j] = pp < p1;
-                const int pc = valid[j] ? pp : p0;
-                const uint16_t *kr = Kb + (int64_t)pc * HD + dl * DPL;
-                const uint16_t *vr = Vb + (int64_t)pc * HD + dl * DPL;
-                uint32_t kw[DPL / 2], vw[DPL / 2];
-                if constexpr (DPL == 8) {
-                    const uint4 kk = *reinterpret_cast<const uint4 *>(kr);
-                    const uint4 vv = *reinterpret_cast<const uint4 *>(vr);
-                    kw[0] = kk.x; kw[1] = kk.y; kw[2] = kk.z; kw[3] = kk.w;
-                    vw[0] = vv.x; vw[1] = vv.y; vw[2] = vv.z; vw[3] = vv.w;
-                } else if constexpr (DPL == 4) {
-                    const uint2 kk = *reinterpret_cast<const uint2 *>(kr);
-                    const uint2 vv = *reinterpret_cast<const uint2 *>(vr);
-                    kw[0] = kk.x; kw[1] = kk.y;
-                    vw[0] = vv.x; vw[1] = vv.y;
-                } else {
-                    kw[0] = *reinterpret_cast<const uint32_t *>(kr);
-                    vw[0] = *reinterpret_cast<const uint32_t *>(vr);
-                }
-#pragma unroll
-                for (int w = 0; w < DPL / 2; ++w) {
-                    kf[j][2 * w] = __uint_as_float(kw[w] << 16);
-                    kf[j][2 * w + 1] = __uint_as_float(kw[w] & 0xffff0000u);
-                    vf[j][2 * w] = __uint_as_float(vw[w] << 16);
-                    vf[j][2 * w + 1] = __uint_as_float(vw[w] & 0xffff0000u);
-                }
+                const int pp = wb + half * kAttnPPI + j;
+                const int pc = pp < p1 ? pp : p0;
+                attn_load_words<DPL>(Kb + (int64_t)pc * HD, K[j]);
+                attn_load_words<DPL>(Vb + (int64_t)pc * HD, V[j]);
             }
+        };
+        if (wstart < p1) load_rows(wstart, kw, vw);
+        for (int wbase = wstart; wbase < p1; wbase += kStride) {
+            uint32_t nk[kAttnPPI][NW], nv[kAttnPPI][NW];
+            const bool more = wbase + kStride < p1;
+            if (more) load_rows(wbase + kStride, nk, nv);
+            const int base = wbase + half * kAttnPPI;
+            float kf[kAttnPPI][DPL], vf[kAttnPPI][DPL];
 #pragma unroll
-            for (int g = 0; g < kAttnMaxG; ++g) {
-                if (g >= G) break;
+            for (int j = 0; j < kAttnPPI; ++j)
+#pragma unroll
+                for (int i = 0; i < NW; ++i) {
+                    kf[j][2 * i] = __uint_as_float(kw[j][i] << 16);
+                    kf[j][2 * i + 1] = __uint_as_float(kw[j][i] & 0xffff0000u);
+                    vf[j][2 * i] = __uint_as_float(vw[j][i] << 16);
+                    vf[j][2 * i + 1] = __uint_as_float(vw[j][i] & 0xffff0000u);
+                }
+#pragma unroll
+            for (int g = 0; g < G; ++g) {
                 float sc[kAttnPPI];
 #pragma unroll
                 for (int j = 0; j < kAttnPPI; ++j) {
@@ -137,7 +147,7 @@ attn_rows_kernel(AttnParams p) {
                     s += __shfl_xor_sync(fmask, s, 4);
                     s += __shfl_xor_sync(fmask, s, 2);
                     s += __shfl_xor_sync(fmask, s, 1);
-                    sc[j] = valid[j] ? s : -INFINITY;
+                    sc[j] = (base + j < p1) ? s : -INFINITY;
                 }
                 float mn = m[g];
 #pragma unroll
@@ -157,15 +167,19 @@ attn_rows_kernel(AttnParams p) {
                     o[g][d] = acc;
                 }
             }
+            if (more) {
+#pragma unroll
+                for (int j = 0; j < kAttnPPI; ++j)
+#pragma unroll
+                    for (int i = 0; i < NW; ++i) { kw[j][i] = nk[j][i]; vw[j][i] = nv[j][i]; }
+            }
         }
         // merge the 8 half-warp states
 #pragma unroll
-        for (int g = 0; g < kAttnMaxG; ++g) {
-            if (g < G) {
-                if (dl == 0) { s_m[hw][g] = m[g]; s_l[hw][g] = l[g]; }
+        for (int g = 0; g < G; ++g) {
+            if (dl == 0) { s_m[hw][g] = m[g]; s_l[hw][g] = l[g]; }
 #pragma unroll
-                for (int d = 0; d < DPL; ++d) s_o[hw][g][dl * DPL + d] = o[g][d];
-            }
+            for (int d = 0; d < DPL; ++d) s_o[hw][g][dl * DPL + d] = o[g][d];
         }
         __syncthreads();
         if (threadIdx.x < G) {
@@ -178,12 +192,13 @@ attn_rows_kernel(AttnParams p) {
             s_fin_l[g] = L;
         }
         __syncthreads();
-        const int per = G * HD;
+        constexpr int per = G * HD;
         if (nsplit == 1) {
             for (int e = threadIdx.x; e < per; e += kAttnThreads) {
                 const int g = e / HD, d = e - g * HD;
                 const float M = s_fin_m[g];
                 float acc = 0.f;
+#pragma unroll
                 for (int h = 0; h < 8; ++h)
                     if (s_m[h][g] != -INFINITY) acc += s_o[h][g][d] * exp2f(s_m[h][g] - M);
                 p.out[((int64_t)row * p.n_heads + kvh * G + g) * HD + d] = f32_to_bf16(acc / s_fin_l[g]);
@@ -194,6 +209,7 @@ attn_rows_kernel(AttnParams p) {
                 const int g = e / HD, d = e - g * HD;
                 const float M = s_fin_m[g];
                 float acc = 0.f;
+#pragma unroll
                 for (int h = 0; h < 8; ++h)
                     if (s_m[h][g] != -INFINITY) acc += s_o[h][g][d] * exp2f(s_m[h][g] - M);
                 mine[g * (HD + 2) + 2 + d] = acc;
@@ -213,21 +229,33 @@ attn_rows_kernel(AttnParams p) {
             if (s_last) {
                 __threadfence();
                 const int i0 = p.row_item0[row];
+                const float *base = p.part + ((int64_t)i0 * p.n_kv + kvh) * G * (HD + 2);
+                const int64_t sp_stride = (int64_t)p.n_kv * G * (HD + 2);
+                // per head: M = max_s m_s, weights w_s = 2^(m_s - M), L = sum_s w_s l_s (warp g)
+                for (int g = warp; g < G; g += kAttnThreads / 32) {
+                    float M = -INFINITY;
+                    for (int sp = lane; sp < nsplit; sp += 32) M = fmaxf(M, __ldcg(base + sp * sp_stride + g * (HD + 2)));
+#pragma unroll
+                    for (int o2 = 16; o2 > 0; o2 >>= 1) M = fmaxf(M, __shfl_xor_sync(fmask, M, o2));
+                    float L = 0.f;
+                    for (int sp = lane; sp < nsplit; sp += 32) {
+                        const float ms = __ldcg(base + sp * sp_stride + g * (HD + 2));
+                        const float w = (ms == -INFINITY) ? 0.f : exp2f(ms - M);
+                        if (sp < kAttnMaxSplits) s_w[g][sp] = w;
+                        L += w * __ldcg(base + sp * sp_stride + g * (HD + 2) + 1);
+                    }
+#pragma unroll
+                    for (int o2 = 16; o2 > 0; o2 >>= 1) L += __shfl_xor_sync(fmask, L, o2);
+                    if (lane == 0) s_fin_l[g] = L;
+                }
+                __syncthreads();
                 for (int e = threadIdx.x; e < per; e += kAttnThreads) {
                     const int g = e / HD, d = e - g * HD;
-                    float M = -INFINITY;
-                    for (int sp = 0; sp < nsplit; ++sp)
-                        M = fmaxf(M, __ldcg(p.part + ((int64_t)(i0 + sp) * p.n_kv + kvh) * G * (HD + 2) + g * (HD + 2)));
-                    float L = 0.f, acc = 0.f;
-                    for (int sp = 0; sp < nsplit; ++sp) {
-                        const float *src = p.part + ((int64_t)(i0 + sp) * p.n_kv + kvh) * G * (HD + 2) + g * (HD + 2);
-                        const float ms = __ldcg(src);
-                        if (ms == -INFINITY) continue;
-                        const float w = exp2f(ms - M);
-                        L += __ldcg(src + 1) * w;
-                        acc += __ldcg(src + 2 + d) * w;
-                    }
-                    p.out[((int64_t)row * p.n_heads + kvh * G + g) * HD + d] = f32_to_bf16(acc / L);
+                    float acc = 0.f;
+                    const float *src = base + g * (HD + 2) + 2 + d;
+#pragma unroll 4
+                    for (int sp = 0; sp < nsplit; ++sp) acc += s_w[g][sp] * __ldcg(src + sp * sp_stride);
+                    p.out[((int64_t)row * p.n_heads + kvh * G + g) * HD + d] = f32_to_bf16(acc / s_fin_l[g]);
                 }
             }
         }

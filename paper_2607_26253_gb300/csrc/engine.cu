@@ -24,7 +24,7 @@ using namespace sara;
 
 namespace {
 
-constexpr int kDecodeChunk = 256;  // decode attention positions per split
+constexpr int kDecodeChunk = 128;  // decode attention positions per split
 
 struct DeviceBuf {
     std::vector<void *> ptrs;
@@ -74,7 +74,7 @@ struct sara_handle {
     Acts dec, pre;
     int pre_cap = 0, att_cap = 0;
     // workspaces
-    float *gemm_part = nullptr;
+    unsigned long long *gemm_acc = nullptr;
     int *gemm_cnt = nullptr;
     float *attn_part = nullptr;
     int *attn_cnt = nullptr;
@@ -145,12 +145,25 @@ void launch_gemm(cudaStream_t s, bool pdl, int grid, const CUtensorMap &tw, cons
     launch(s, pdl, dim3(grid), dim3(kGemmThreads), kGemmSmemBytes, gemm_tc_kernel<EPI>, tw, tx, p);
 }
 
+template <int HD>
+void launch_attention_hd(cudaStream_t s, bool pdl, dim3 grid, int G, const AttnParams &p) {
+    switch (G) {
+        case 1: launch(s, pdl, grid, dim3(kAttnThreads), 0, attn_rows_kernel<HD, 1>, p); break;
+        case 2: launch(s, pdl, grid, dim3(kAttnThreads), 0, attn_rows_kernel<HD, 2>, p); break;
+        case 4: launch(s, pdl, grid, dim3(kAttnThreads), 0, attn_rows_kernel<HD, 4>, p); break;
+        case 6: launch(s, pdl, grid, dim3(kAttnThreads), 0, attn_rows_kernel<HD, 6>, p); break;
+        case 8: launch(s, pdl, grid, dim3(kAttnThreads), 0, attn_rows_kernel<HD, 8>, p); break;
+        default: throw SaraError(SARA_EINVAL, "n_heads / n_kv_heads must be 1, 2, 4, 6 or 8");
+    }
+}
+
 void launch_attention(cudaStream_t s, bool pdl, int sms, int hd, const AttnParams &p) {
     dim3 grid(std::max(1, (sms * 4) / std::max(1, p.n_kv)), p.n_kv);
+    const int G = p.n_heads / p.n_kv;
     switch (hd) {
-        case 32: launch(s, pdl, grid, dim3(kAttnThreads), 0, attn_rows_kernel<32>, p); break;
-        case 64: launch(s, pdl, grid, dim3(kAttnThreads), 0, attn_rows_kernel<64>, p); break;
-        case 128: launch(s, pdl, grid, dim3(kAttnThreads), 0, attn_rows_kernel<128>, p); break;
+        case 32: launch_attention_hd<32>(s, pdl, grid, G, p); break;
+        case 64: launch_attention_hd<64>(s, pdl, grid, G, p); break;
+        case 128: launch_attention_hd<128>(s, pdl, grid, G, p); break;
         default: throw SaraError(SARA_EINVAL, "head_dim must be 32, 64 or 128");
     }
 }
@@ -162,7 +175,7 @@ GemmParams gemm_base(const sara_handle &h, int m_tiles, int k_chunks, const Acts
     p.rows_cap = A.rows_cap;
     p.rows_dev = rows_dev;
     p.decode = decode ? 1 : 0;
-    p.ws_part = h.gemm_part;
+    p.ws_acc = h.gemm_acc;
     p.ws_cnt = h.gemm_cnt;
     p.err = &h.vars->err;
     p.ssq_tiles = h.cfg.d_model / 128;
@@ -457,8 +470,14 @@ void validate_cfg(const sara_model_cfg &m) {
     if (m.layers == 0) return;
     if (m.d_model % 128 || m.d_model < 128) bad("d_model must be a positive multiple of 128");
     if (m.head_dim != 32 && m.head_dim != 64 && m.head_dim != 128) bad("head_dim must be 32, 64 or 128");
-    if (m.n_kv_heads < 1 || m.n_heads % m.n_kv_heads || m.n_heads / m.n_kv_heads > kAttnMaxG)
-        bad("n_heads / n_kv_heads must be an integer <= 8");
+    if (m.n_kv_heads < 1 || m.n_heads % m.n_kv_heads)
+        bad("n_heads must be a multiple of n_kv_heads");
+    {
+        const int G = m.n_heads / m.n_kv_heads;
+        if (G != 1 && G != 2 && G != 4 && G != 6 && G != 8) bad("n_heads / n_kv_heads must be 1, 2, 4, 6 or 8");
+    }
+    if ((m.max_prompt_len + m.max_gen_len + kDecodeChunk - 1) / kDecodeChunk > kAttnMaxSplits)
+        bad("max_prompt_len + max_gen_len exceeds the attention split capacity (96 x 128 positions)");
     if ((m.n_heads * m.head_dim) % 128 || ((m.n_heads + 2 * m.n_kv_heads) * m.head_dim) % 128)
         bad("head dims must tile by 128");
     if (m.ffn % 64 || m.ffn < 64) bad("ffn must be a multiple of 64");
@@ -559,8 +578,8 @@ void create_impl(sara_handle &h, const sara_model_cfg *cfgp, const sara_weights 
         CK(cudaMemcpy(h.rope, rope.data(), rope.size() * sizeof(float2), cudaMemcpyHostToDevice));
         alloc_acts(h, h.dec, S);
         alloc_acts(h, h.pre, h.pre_cap);
-        // GEMM stream-K workspace: two partial tiles per CTA + per-tile counters
-        h.gemm_part = h.mem.alloc<float>((size_t)h.sms * 2 * kTileR * kTileM, false);
+        // GEMM stream-K workspace: one fixed-point tile sum per CTA + per-tile counters (zeroed)
+        h.gemm_acc = h.mem.alloc<unsigned long long>((size_t)h.sms * kTileR * kTileM);
         const int max_m = std::max({(m.n_heads + 2 * KVH) * hd, d, 2 * m.ffn, m.vocab}) / 128;
         h.gemm_cnt = h.mem.alloc<int>((size_t)max_m * ((h.pre_cap + kTileR - 1) / kTileR + 1));
         const int Gq = m.n_heads / KVH;

@@ -8,9 +8,10 @@
 //
 // Work split: stream-K.  The (tile, k-chunk) units of the whole GEMM are cut into
 // gridDim.x equal contiguous ranges, so every SM streams the same number of weight bytes.
-// A tile whose k-chunks span several CTAs is finished by the CTA that arrives last (a
-// per-tile counter, no spinning): it adds every contributor's fp32 partial in CTA order
-// (deterministic) and runs the epilogue.
+// A tile whose k-chunks span several CTAs is folded into a 64-bit fixed-point accumulator
+// (value * 2^32) with fire-and-forget integer atomic adds -- integer addition is
+// associative, so the sum does not depend on arrival order -- and the CTA that arrives
+// last (a per-tile counter, no spinning) reads it once, clears it, and runs the epilogue.
 //
 // Warp roles (192 threads): warp 0 = TMA producer, warp 1 = MMA issuer + tensor-memory
 // owner, warps 2..5 = epilogue (warp w reads tensor-memory lanes 32*(w%4) .. +31).
@@ -47,7 +48,7 @@ struct GemmParams {
     const int *rows_dev;       // device count of valid rows (nullptr -> rows_fixed)
     int rows_fixed;
     int decode;                // 1: a single row tile, weights prefetched before the PDL wait
-    float *ws_part;            // [gridDim.x][2][kTileR * kTileM] fp32 partials
+    unsigned long long *ws_acc;  // [gridDim.x][kTileR * kTileM] fixed-point tile sums, zero between launches
     int *ws_cnt;               // [tiles] arrival counters, zero between launches
     int *err;
     // outputs / epilogue inputs
@@ -403,19 +404,21 @@ gemm_tc_kernel(const __grid_constant__ CUtensorMap tmW, const __grid_constant__ 
             bool do_epi = whole;
             int c_a = cta, c_b = cta;
             if (!whole) {
-                // write this CTA's partial, count arrivals; the last arrival finishes the tile
-                const int slot = (u0 / kch == tile) ? 0 : 1;
-                float *mine = p.ws_part + ((size_t)cta * 2 + slot) * (kTileR * kTileM);
+                // fold this CTA's share into the tile's fixed-point sum; the last arrival finishes
+                c_a = cta_of_unit((int64_t)tile * kch, U, G);
+                c_b = cta_of_unit((int64_t)(tile + 1) * kch - 1, U, G);
+                unsigned long long *acc = p.ws_acc + (size_t)c_a * (kTileR * kTileM);
                 for (int c0 = 0; c0 < rin; c0 += 32) {
                     float v[32];
                     tmem_ld_32x32b_x32(tmem + lane_base + (uint32_t)(a * kTileR + c0), v);
 #pragma unroll
-                    for (int c = 0; c < 32; ++c) mine[(c0 + c) * kTileM + mrow] = v[c];
+                    for (int c = 0; c < 32; ++c)
+                        if (c0 + c < rin)
+                            atomicAdd(&acc[(c0 + c) * kTileM + mrow],
+                                      (unsigned long long)__float2ll_rn(v[c] * 4294967296.0f));
                 }
                 __threadfence();
                 named_bar_sync(1, 128);
-                c_a = cta_of_unit((int64_t)tile * kch, U, G);
-                c_b = cta_of_unit((int64_t)(tile + 1) * kch - 1, U, G);
                 if (etid == 0) {
                     int nseg = 0;
                     for (int c = c_a; c <= c_b; ++c) nseg += unit_begin(c, U, G) < unit_begin(c + 1, U, G);
@@ -427,7 +430,6 @@ gemm_tc_kernel(const __grid_constant__ CUtensorMap tmW, const __grid_constant__ 
                 do_epi = S.last_flag != 0;
                 __threadfence();
             }
-            if (etid == 0) GEMM_STAMP(5);
             if (do_epi) {
                 if constexpr (EPI == EPI_QKV || EPI == EPI_SWIGLU || EPI == EPI_LMHEAD) {
                     if (etid < rin) {
@@ -445,15 +447,12 @@ gemm_tc_kernel(const __grid_constant__ CUtensorMap tmW, const __grid_constant__ 
                     if (whole) {
                         tmem_ld_32x32b_x32(tmem + lane_base + (uint32_t)(a * kTileR + c0), v);
                     } else {
+                        unsigned long long *acc = p.ws_acc + (size_t)c_a * (kTileR * kTileM);
 #pragma unroll
-                        for (int c = 0; c < 32; ++c) v[c] = 0.f;
-                        for (int cc = c_a; cc <= c_b; ++cc) {
-                            if (!(unit_begin(cc, U, G) < unit_begin(cc + 1, U, G))) continue;
-                            const int first_tile = (int)(unit_begin(cc, U, G) / kch);
-                            const int slot = (first_tile == tile) ? 0 : 1;
-                            const float *src = p.ws_part + ((size_t)cc * 2 + slot) * (kTileR * kTileM);
-#pragma unroll
-                            for (int c = 0; c < 32; ++c) v[c] += __ldcg(&src[(c0 + c) * kTileM + mrow]);
+                        for (int c = 0; c < 32; ++c) {
+                            const size_t idx = (size_t)(c0 + c) * kTileM + mrow;
+                            v[c] = (float)(long long)__ldcg(&acc[idx]) * 2.3283064365386963e-10f;  // 2^-32
+                            if (c0 + c < rin) acc[idx] = 0ull;
                         }
                     }
                     gemm_epilogue_chunk<EPI>(p, S, v, m_tile, r_base, c0, rin, mrow, etid);

@@ -32,9 +32,20 @@ struct GemmWs {
 };
 GemmWs gemm_ws_layout(int Nout, int sms) {
     GemmWs w;
-    w.part_bytes = align_up((size_t)sms * 2 * kTileR * kTileM * sizeof(float), 256);
+    w.part_bytes = align_up((size_t)sms * kTileR * kTileM * sizeof(unsigned long long), 256);
     w.cnt_bytes = align_up((size_t)(Nout / kTileM) * sizeof(int), 256);
     return w;
+}
+
+template <int HD>
+void launch_g(dim3 grid, int G, cudaStream_t s, const AttnParams &a) {
+    switch (G) {
+        case 1: attn_rows_kernel<HD, 1><<<grid, kAttnThreads, 0, s>>>(a); break;
+        case 2: attn_rows_kernel<HD, 2><<<grid, kAttnThreads, 0, s>>>(a); break;
+        case 4: attn_rows_kernel<HD, 4><<<grid, kAttnThreads, 0, s>>>(a); break;
+        case 6: attn_rows_kernel<HD, 6><<<grid, kAttnThreads, 0, s>>>(a); break;
+        default: attn_rows_kernel<HD, 8><<<grid, kAttnThreads, 0, s>>>(a); break;
+    }
 }
 
 template <typename F>
@@ -86,7 +97,7 @@ int sara_gemm_bf16(const uint16_t *X, const uint16_t *W, float *Y, int32_t R, in
         p.rows_dev = nullptr;
         p.rows_fixed = R;
         p.decode = 1;
-        p.ws_part = reinterpret_cast<float *>(workspace);
+        p.ws_acc = reinterpret_cast<unsigned long long *>(workspace);
         p.ws_cnt = reinterpret_cast<int *>(reinterpret_cast<uint8_t *>(workspace) + w.part_bytes);
         p.err = nullptr;
         p.y_f32 = Y;
@@ -98,7 +109,7 @@ int sara_gemm_bf16(const uint16_t *X, const uint16_t *W, float *Y, int32_t R, in
 
 size_t sara_attention_workspace_bytes(int32_t b, int32_t n_heads, int32_t head_dim, int32_t max_ctx) {
     if (b < 1 || n_heads < 1 || head_dim < 1 || max_ctx < 1) return 0;
-    const size_t splits = (size_t)(max_ctx + 255) / 256;
+    const size_t splits = (size_t)(max_ctx + 127) / 128;
     const size_t items = (size_t)b * splits;
     // partials (<= items * n_heads * (hd + 2) floats), counters [b][n_kv], items, 3 row arrays
     return align_up(items * n_heads * (head_dim + 2) * sizeof(float), 256) +
@@ -112,12 +123,12 @@ int sara_attention_decode(const uint16_t *q, const uint16_t *kv, int64_t kv_stri
     if (!q || !kv || !ctx || !out || !workspace) return SARA_EINVAL;
     if (b < 1 || n_kv_heads < 1 || n_heads % n_kv_heads || n_heads / n_kv_heads > kAttnMaxG) return SARA_EINVAL;
     if (head_dim != 32 && head_dim != 64 && head_dim != 128) return SARA_EINVAL;
-    if (max_ctx < 1 || max_ctx > cap) return SARA_EINVAL;
+    if (max_ctx < 1 || max_ctx > cap || (max_ctx + 127) / 128 > kAttnMaxSplits) return SARA_EINVAL;
     return op_guard([&] {
         if (workspace_bytes < sara_attention_workspace_bytes(b, n_heads, head_dim, max_ctx))
             throw SaraError(SARA_EINVAL, "workspace too small");
         cudaStream_t s = static_cast<cudaStream_t>(stream);
-        const size_t splits = (size_t)(max_ctx + 255) / 256;
+        const size_t splits = (size_t)(max_ctx + 127) / 128;
         const size_t items_cap = (size_t)b * splits;
         uint8_t *ws = reinterpret_cast<uint8_t *>(workspace);
         float *part = reinterpret_cast<float *>(ws);
@@ -139,7 +150,7 @@ int sara_attention_decode(const uint16_t *q, const uint16_t *kv, int64_t kv_stri
             hpos[i] = hctx[i] - 1;
             hi0[i] = (int)hitems.size();
             slots[i] = i;
-            for (int sp = 0; sp < (hctx[i] + 255) / 256; ++sp) hitems.push_back(make_int2(i, sp));
+            for (int sp = 0; sp < (hctx[i] + 127) / 128; ++sp) hitems.push_back(make_int2(i, sp));
         }
         CK(cudaMemcpyAsync(items, hitems.data(), hitems.size() * sizeof(int2), cudaMemcpyHostToDevice, s));
         CK(cudaMemcpyAsync(row_pos, hpos.data(), b * sizeof(int), cudaMemcpyHostToDevice, s));
@@ -159,16 +170,18 @@ int sara_attention_decode(const uint16_t *q, const uint16_t *kv, int64_t kv_stri
         a.row_item0 = row_item0;
         a.n_heads = n_heads;
         a.n_kv = n_kv_heads;
-        a.chunk = 256;
+        a.chunk = 128;
         a.scale_log2 = (float)(1.4426950408889634 / std::sqrt((double)head_dim));
         a.part = part;
         a.cnt = cnt;
         a.err = nullptr;
         const int sms = sm_count();
         dim3 grid(std::max(1, sms * 4 / n_kv_heads), n_kv_heads);
-        if (head_dim == 32) attn_rows_kernel<32><<<grid, kAttnThreads, 0, s>>>(a);
-        else if (head_dim == 64) attn_rows_kernel<64><<<grid, kAttnThreads, 0, s>>>(a);
-        else attn_rows_kernel<128><<<grid, kAttnThreads, 0, s>>>(a);
+        const int G = n_heads / n_kv_heads;
+        if (G != 1 && G != 2 && G != 4 && G != 6 && G != 8) throw SaraError(SARA_EINVAL, "query group must be 1, 2, 4, 6 or 8");
+        if (head_dim == 32) launch_g<32>(grid, G, s, a);
+        else if (head_dim == 64) launch_g<64>(grid, G, s, a);
+        else launch_g<128>(grid, G, s, a);
         CK(cudaGetLastError());
         CK(cudaStreamSynchronize(s));  // the host vectors above back in-flight copies
     });
