@@ -805,8 +805,8 @@ void profile_impl(sara_handle &h, int which, int rows, int ctx, int iters, doubl
     CK(cudaMemcpyAsync(c.seq_len, len.data(), rows * 4, cudaMemcpyHostToDevice, s));
     CK(cudaMemcpyAsync(c.seq_uid, uid.data(), rows * 8, cudaMemcpyHostToDevice, s));
 #ifdef SARA_STAMPS
-    if (!h.stamps) h.stamps = h.mem.alloc<uint64_t>((size_t)h.sms * 8);
-    CK(cudaMemsetAsync(h.stamps, 0, (size_t)h.sms * 8 * 8, s));
+    if (!h.stamps) h.stamps = h.mem.alloc<uint64_t>((size_t)h.sms * 16);
+    CK(cudaMemsetAsync(h.stamps, 0, (size_t)h.sms * 16 * 8, s));
 #endif
     CK(cudaStreamSynchronize(s));
     auto one = [&] {
@@ -826,14 +826,14 @@ void profile_impl(sara_handle &h, int which, int rows, int ctx, int iters, doubl
     *ms = (double)t / iters;
 #ifdef SARA_STAMPS
     if (h.stamps && which != 0) {  // phase breakdown of the last launch, relative to the earliest entry
-        std::vector<uint64_t> st((size_t)h.sms * 8);
+        std::vector<uint64_t> st((size_t)h.sms * 16);
         CK(cudaMemcpy(st.data(), h.stamps, st.size() * 8, cudaMemcpyDeviceToHost));
         uint64_t t0 = ~0ull;
-        for (int c = 0; c < h.sms; ++c) t0 = std::min(t0, st[(size_t)c * 8]);
-        for (int i = 0; i < 8; ++i) {
+        for (int c = 0; c < h.sms; ++c) t0 = std::min(t0, st[(size_t)c * 16]);
+        for (int i = 0; i < 16; ++i) {
             std::vector<double> d;
             for (int c = 0; c < h.sms; ++c)
-                if (st[(size_t)c * 8 + i]) d.push_back((double)(st[(size_t)c * 8 + i] - t0) * 1e-3);
+                if (st[(size_t)c * 16 + i]) d.push_back((double)(st[(size_t)c * 16 + i] - t0) * 1e-3);
             std::sort(d.begin(), d.end());
             if (!d.empty())
                 fprintf(stderr, "stamp %d: n=%zu min %.2f med %.2f max %.2f us\n", i, d.size(), d.front(), d[d.size() / 2],

@@ -70,7 +70,7 @@ struct GemmParams {
     uint16_t *h_out;           // EPI_SWIGLU [rows][ld]
     const uint64_t *row_seed;  // EPI_LMHEAD sampler key of the row
     float *arg_val; int *arg_idx;  // EPI_LMHEAD [rows][m_tiles] partial max / argmax
-    uint64_t *stamps;          // optional [gridDim.x][8] phase timestamps (profiling builds)
+    uint64_t *stamps;          // optional [gridDim.x][16] phase timestamps (profiling builds)
 };
 
 struct GemmSmem {
@@ -86,6 +86,9 @@ struct GemmSmem {
     int epi_decision;   // uniform abort decision of the epilogue warps
     int skip;           // an earlier kernel of the step reported an error: do nothing
     float inv_rms[kTileR];
+    int row_pos[kTileR];               // per-row metadata of the tile being finished
+    int row_slot[kTileR];
+    unsigned long long row_seed[kTileR];
     float xch[kTileM * kEpiLd];        // exchange tile: 128 features x 32 columns
 };
 
@@ -101,7 +104,7 @@ __device__ __forceinline__ int cta_of_unit(int64_t u, int64_t U, int G) {
     return c;
 }
 #ifdef SARA_STAMPS
-#define GEMM_STAMP(i) do { if (p.stamps) p.stamps[(size_t)blockIdx.x * 8 + (i)] = globaltimer_ns(); } while (0)
+#define GEMM_STAMP(i) do { if (p.stamps) p.stamps[(size_t)blockIdx.x * 16 + (i)] = globaltimer_ns(); } while (0)
 #else
 #define GEMM_STAMP(i) do { } while (0)
 #endif
@@ -125,11 +128,15 @@ __device__ __forceinline__ void gemm_epilogue_chunk(const GemmParams &p, GemmSme
     }
     if constexpr (EPI == EPI_RESID) {
         const float g = bf16_to_f32(p.g_next[n]);
+        float xo[32];
+#pragma unroll
+        for (int c = 0; c < 32; ++c)  // every load before any store (the stores may alias)
+            xo[c] = (c < ncols) ? __ldcg(&p.x_f32[(int64_t)(r_base + c0 + c) * p.ld + n]) : 0.f;
 #pragma unroll
         for (int c = 0; c < 32; ++c) {
             if (c < ncols) {
                 const int64_t idx = (int64_t)(r_base + c0 + c) * p.ld + n;
-                const float x = p.x_f32[idx] + v[c];
+                const float x = xo[c] + v[c];
                 p.x_f32[idx] = x;
                 p.xg_out[idx] = f32_to_bf16(x * g);
                 v[c] = x * x;
@@ -142,7 +149,7 @@ __device__ __forceinline__ void gemm_epilogue_chunk(const GemmParams &p, GemmSme
             if (c < ncols) {
                 const int r = r_base + c0 + c;
                 if (p.y_f32) p.y_f32[(int64_t)r * p.ld + n] = v[c];
-                v[c] += gumbel_from_hash(splitmix_at(p.row_seed[r], (uint64_t)n + 1));
+                v[c] += gumbel_from_hash(splitmix_at(S.row_seed[c0 + c], (uint64_t)n + 1));
             }
         }
     }
@@ -156,23 +163,27 @@ __device__ __forceinline__ void gemm_epilogue_chunk(const GemmParams &p, GemmSme
         const int partner = (i < half) ? mrow + half : mrow - half;
         const int fi = (i < half) ? i : i - half;
         const int nq = p.n_heads, nkv = p.n_kv;
+        const bool rot = head < nq + nkv;  // q or k: rotate the pair (i, i + hd/2)
+        float2 cs[32];
+#pragma unroll
+        for (int c = 0; c < 32; ++c)  // every table load before any store
+            cs[c] = (rot && c < ncols) ? __ldg(&p.rope[(int64_t)S.row_pos[c0 + c] * half + fi]) : make_float2(1.f, 0.f);
 #pragma unroll
         for (int c = 0; c < 32; ++c) {
             if (c < ncols) {
                 const int r = r_base + c0 + c;
                 float y = v[c];
-                if (head < nq + nkv) {  // q or k: rotate the pair (i, i + hd/2)
-                    const float2 cs = p.rope[(int64_t)p.row_pos[r] * half + fi];
+                if (rot) {
                     const float o = S.xch[partner * kEpiLd + c];
-                    y = (i < half) ? (y * cs.x - o * cs.y) : (y * cs.x + o * cs.y);
+                    y = (i < half) ? (y * cs[c].x - o * cs[c].y) : (y * cs[c].x + o * cs[c].y);
                 }
                 if (head < nq) {
                     p.q_out[(int64_t)r * (nq * hd) + n] = f32_to_bf16(y);
                 } else {
                     const int isv = head >= nq + nkv;
                     const int kvh = head - nq - isv * nkv;
-                    uint16_t *dst = p.kv + (int64_t)p.row_slot[r] * p.kv_slot_stride +
-                                    ((int64_t)(isv * nkv + kvh) * p.kv_cap + p.row_pos[r]) * hd + i;
+                    uint16_t *dst = p.kv + (int64_t)S.row_slot[c0 + c] * p.kv_slot_stride +
+                                    ((int64_t)(isv * nkv + kvh) * p.kv_cap + S.row_pos[c0 + c]) * hd + i;
                     *dst = f32_to_bf16(y);
                 }
             }
@@ -417,8 +428,10 @@ gemm_tc_kernel(const __grid_constant__ CUtensorMap tmW, const __grid_constant__ 
                             atomicAdd(&acc[(c0 + c) * kTileM + mrow],
                                       (unsigned long long)__float2ll_rn(v[c] * 4294967296.0f));
                 }
+                if (etid == 0) GEMM_STAMP(8);
                 __threadfence();
                 named_bar_sync(1, 128);
+                if (etid == 0) GEMM_STAMP(9);
                 if (etid == 0) {
                     int nseg = 0;
                     for (int c = c_a; c <= c_b; ++c) nseg += unit_begin(c, U, G) < unit_begin(c + 1, U, G);
@@ -432,13 +445,28 @@ gemm_tc_kernel(const __grid_constant__ CUtensorMap tmW, const __grid_constant__ 
             }
             if (do_epi) {
                 if constexpr (EPI == EPI_QKV || EPI == EPI_SWIGLU || EPI == EPI_LMHEAD) {
+                    // per-row values of this tile, staged once: 1/rms, position, slot, sampler key
                     if (etid < rin) {
+                        const int r = r_base + etid;
+                        float part[16];
+#pragma unroll
+                        for (int t = 0; t < 16; ++t)
+                            part[t] = (t < p.ssq_tiles) ? __ldcg(&p.ssq[(int64_t)t * p.rows_cap + r]) : 0.f;
                         float s = 0.f;
-                        for (int t = 0; t < p.ssq_tiles; ++t)
-                            s += __ldcg(&p.ssq[(int64_t)t * p.rows_cap + r_base + etid]);
+#pragma unroll
+                        for (int t = 0; t < 16; ++t) s += part[t];
+                        for (int t = 16; t < p.ssq_tiles; ++t) s += __ldcg(&p.ssq[(int64_t)t * p.rows_cap + r]);
                         S.inv_rms[etid] = rsqrtf(s * p.inv_dim + p.eps);
+                        if constexpr (EPI == EPI_QKV) {
+                            S.row_pos[etid] = p.row_pos[r];
+                            S.row_slot[etid] = p.row_slot[r];
+                        }
+                        if constexpr (EPI == EPI_LMHEAD) S.row_seed[etid] = p.row_seed[r];
                     } else {
                         S.inv_rms[etid] = 0.f;
+                        S.row_pos[etid] = 0;
+                        S.row_slot[etid] = 0;
+                        S.row_seed[etid] = 0ull;
                     }
                     named_bar_sync(1, 128);
                 }
@@ -455,7 +483,9 @@ gemm_tc_kernel(const __grid_constant__ CUtensorMap tmW, const __grid_constant__ 
                             if (c0 + c < rin) acc[idx] = 0ull;
                         }
                     }
+                    if (etid == 0) GEMM_STAMP(10);
                     gemm_epilogue_chunk<EPI>(p, S, v, m_tile, r_base, c0, rin, mrow, etid);
+                    if (etid == 0) GEMM_STAMP(11);
                 }
             }
             // release the accumulator buffer
