@@ -140,8 +140,16 @@ void launch(cudaStream_t s, bool pdl, dim3 grid, dim3 block, size_t smem, Kern k
     CK(cudaLaunchKernelEx(&cfg, kern, args...));
 }
 
+// Grid of a decode GEMM: one whole tile per CTA when the tile count nearly fills the SMs
+// (no split reduction at all), else one CTA per SM with the stream-K split.
+int gemm_grid(int sms, int tiles, bool decode) {
+    if (decode && tiles <= sms && tiles * 20 >= sms * 17) return tiles;
+    return sms;
+}
+
 template <int EPI>
 void launch_gemm(cudaStream_t s, bool pdl, int grid, const CUtensorMap &tw, const CUtensorMap &tx, const GemmParams &p) {
+    grid = gemm_grid(grid, p.m_tiles, p.decode != 0);
     launch(s, pdl, dim3(grid), dim3(kGemmThreads), kGemmSmemBytes, gemm_tc_kernel<EPI>, tw, tx, p);
 }
 

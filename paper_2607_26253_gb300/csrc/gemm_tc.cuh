@@ -388,6 +388,41 @@ gemm_tc_kernel(const __grid_constant__ CUtensorMap tmW, const __grid_constant__ 
         const int mrow = quarter * 32 + lane;
         const int etid = threadIdx.x - 64;  // 0..127
         const uint32_t lane_base = (uint32_t)(quarter * 32) << 16;
+        // Per-row values (1/rms, position, KV slot, sampler key) staged once per tile: in
+        // decode mode every tile has the same rows, so they are loaded once, while the
+        // mainloop streams weights.
+        int staged_rbase = -1;
+        auto stage_rows = [&](int r_base, int rin) {
+            if constexpr (EPI == EPI_QKV || EPI == EPI_SWIGLU || EPI == EPI_LMHEAD) {
+                if (etid < rin) {
+                    const int r = r_base + etid;
+                    float part[16];
+#pragma unroll
+                    for (int t = 0; t < 16; ++t)
+                        part[t] = (t < p.ssq_tiles) ? __ldcg(&p.ssq[(int64_t)t * p.rows_cap + r]) : 0.f;
+                    float s = 0.f;
+#pragma unroll
+                    for (int t = 0; t < 16; ++t) s += part[t];
+                    for (int t = 16; t < p.ssq_tiles; ++t) s += __ldcg(&p.ssq[(int64_t)t * p.rows_cap + r]);
+                    S.inv_rms[etid] = rsqrtf(s * p.inv_dim + p.eps);
+                    if constexpr (EPI == EPI_QKV) {
+                        S.row_pos[etid] = p.row_pos[r];
+                        S.row_slot[etid] = p.row_slot[r];
+                    }
+                    if constexpr (EPI == EPI_LMHEAD) S.row_seed[etid] = p.row_seed[r];
+                } else {
+                    S.inv_rms[etid] = 0.f;
+                    S.row_pos[etid] = 0;
+                    S.row_slot[etid] = 0;
+                    S.row_seed[etid] = 0ull;
+                }
+                named_bar_sync(1, 128);
+            }
+        };
+        if (p.decode && u0 < u1) {
+            stage_rows(0, min(kTileR, rows));
+            staged_rbase = 0;
+        }
         int seg = 0;
         for (int64_t u = u0; u < u1; ++seg) {
             const int tile = (int)(u / kch);
@@ -444,31 +479,9 @@ gemm_tc_kernel(const __grid_constant__ CUtensorMap tmW, const __grid_constant__ 
                 __threadfence();
             }
             if (do_epi) {
-                if constexpr (EPI == EPI_QKV || EPI == EPI_SWIGLU || EPI == EPI_LMHEAD) {
-                    // per-row values of this tile, staged once: 1/rms, position, slot, sampler key
-                    if (etid < rin) {
-                        const int r = r_base + etid;
-                        float part[16];
-#pragma unroll
-                        for (int t = 0; t < 16; ++t)
-                            part[t] = (t < p.ssq_tiles) ? __ldcg(&p.ssq[(int64_t)t * p.rows_cap + r]) : 0.f;
-                        float s = 0.f;
-#pragma unroll
-                        for (int t = 0; t < 16; ++t) s += part[t];
-                        for (int t = 16; t < p.ssq_tiles; ++t) s += __ldcg(&p.ssq[(int64_t)t * p.rows_cap + r]);
-                        S.inv_rms[etid] = rsqrtf(s * p.inv_dim + p.eps);
-                        if constexpr (EPI == EPI_QKV) {
-                            S.row_pos[etid] = p.row_pos[r];
-                            S.row_slot[etid] = p.row_slot[r];
-                        }
-                        if constexpr (EPI == EPI_LMHEAD) S.row_seed[etid] = p.row_seed[r];
-                    } else {
-                        S.inv_rms[etid] = 0.f;
-                        S.row_pos[etid] = 0;
-                        S.row_slot[etid] = 0;
-                        S.row_seed[etid] = 0ull;
-                    }
-                    named_bar_sync(1, 128);
+                if (staged_rbase != r_base) {
+                    stage_rows(r_base, rin);
+                    staged_rbase = r_base;
                 }
                 for (int c0 = 0; c0 < rin; c0 += 32) {
                     float v[32];
