@@ -175,9 +175,10 @@ SARA_API int sara_teacher_force(sara_handle *h, int32_t n_seq, int32_t prompt_le
 
 /*
  * Profiling hook (benchmarks): set `rows` live rollouts at context length `ctx` (synthetic
- * row state; the step's own state is overwritten) and launch `iters` times, after two
- * warm-up launches, either one decode kernel of layer 0 or the whole decode step, timing
- * them with CUDA events on the handle's stream.  *ms_per_launch = elapsed / iters.
+ * row state; the step's own state is overwritten) and launch, after two warm-up launches,
+ * `iters` copies of either one decode kernel of layer 0 or the whole decode step, captured
+ * in a CUDA graph (no host launch cost) and timed with CUDA events on the handle's stream.
+ * *ms_per_launch = elapsed / iters.
  *   kernel: 0 = whole decode step (eager launches), 1 = QKV projection + RoPE + KV append,
  *           2 = decode attention, 3 = O projection + residual, 4 = gate/up + SwiGLU,
  *           5 = down projection + residual, 6 = lm_head + fused sampling partials.

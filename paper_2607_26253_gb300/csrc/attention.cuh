@@ -39,7 +39,14 @@ struct AttnParams {
     float *part;              // [items][n_kv][G][hd + 2] fp32 partials (m, l, o[hd])
     int *cnt;                 // [rows][n_kv] arrival counters, zero between launches
     int *err;
+    uint64_t *stamps;         // optional [blocks][16] phase timestamps (profiling builds)
 };
+
+#ifdef SARA_STAMPS
+#define ATTN_STAMP(i) do { if (p.stamps && threadIdx.x == 0 && blockIdx.y == 0 && blockIdx.x < 152) p.stamps[(size_t)blockIdx.x * 16 + (i)] = globaltimer_ns(); } while (0)
+#else
+#define ATTN_STAMP(i) do { } while (0)
+#endif
 
 template <int DPL>
 __device__ __forceinline__ void attn_load_words(const uint16_t *p, uint32_t (&w)[DPL / 2]) {
@@ -67,10 +74,12 @@ attn_rows_kernel(AttnParams p) {
     __shared__ float s_w[G][kAttnMaxSplits];
     __shared__ int s_last;
 
+    ATTN_STAMP(0);
     pdl_wait_prior_grids();
     pdl_allow_dependents();
     const int n_items = p.n_items_dev ? *p.n_items_dev : p.n_items_fixed;
     const int kvh = blockIdx.y;
+    ATTN_STAMP(1);
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const int half = lane >> 4, dl = lane & 15;
     const int hw = warp * 2 + half;  // half-warp id 0..7
@@ -119,6 +128,7 @@ attn_rows_kernel(AttnParams p) {
                 attn_load_words<DPL>(Vb + (int64_t)pc * HD, V[j]);
             }
         };
+        ATTN_STAMP(2);
         if (wstart < p1) load_rows(wstart, kw, vw);
         for (int wbase = wstart; wbase < p1; wbase += kStride) {
             uint32_t nk[kAttnPPI][NW], nv[kAttnPPI][NW];
@@ -174,6 +184,7 @@ attn_rows_kernel(AttnParams p) {
                     for (int i = 0; i < NW; ++i) { kw[j][i] = nk[j][i]; vw[j][i] = nv[j][i]; }
             }
         }
+        ATTN_STAMP(3);
         // merge the 8 half-warp states
 #pragma unroll
         for (int g = 0; g < G; ++g) {
@@ -220,12 +231,14 @@ attn_rows_kernel(AttnParams p) {
             }
             __threadfence();
             __syncthreads();
+            ATTN_STAMP(4);
             if (threadIdx.x == 0) {
                 const int old = atomicAdd(&p.cnt[row * p.n_kv + kvh], 1);
                 s_last = (old == nsplit - 1);
                 if (s_last) p.cnt[row * p.n_kv + kvh] = 0;
             }
             __syncthreads();
+            ATTN_STAMP(5);
             if (s_last) {
                 __threadfence();
                 const int i0 = p.row_item0[row];
@@ -257,10 +270,12 @@ attn_rows_kernel(AttnParams p) {
                     for (int sp = 0; sp < nsplit; ++sp) acc += s_w[g][sp] * __ldcg(src + sp * sp_stride);
                     p.out[((int64_t)row * p.n_heads + kvh * G + g) * HD + d] = f32_to_bf16(acc / s_fin_l[g]);
                 }
+                ATTN_STAMP(6);
             }
         }
         __syncthreads();  // shared state reused by the next item
     }
+    ATTN_STAMP(7);
 }
 
 }  // namespace sara

@@ -143,6 +143,9 @@ void launch(cudaStream_t s, bool pdl, dim3 grid, dim3 block, size_t smem, Kern k
 // Grid of a decode GEMM: one whole tile per CTA when the tile count nearly fills the SMs
 // (no split reduction at all), else one CTA per SM with the stream-K split.
 int gemm_grid(int sms, int tiles, bool decode) {
+#ifdef SARA_STAMPS
+    if (const char *e = getenv("SARA_GEMM_GRID")) return std::max(1, std::min(sms, atoi(e)));  // profiling sweeps
+#endif
     if (decode && tiles <= sms && tiles * 20 >= sms * 17) return tiles;
     return sms;
 }
@@ -242,6 +245,7 @@ void enqueue_kernel(sara_handle &h, cudaStream_t s, bool decode, int which, int 
             a.part = h.attn_part;
             a.cnt = h.attn_cnt;
             a.err = &h.vars->err;
+            a.stamps = h.stamps;
             launch_attention(s, pdl, h.sms, hd, a);
             break;
         }
@@ -776,7 +780,7 @@ void profile_impl(sara_handle &h, int which, int rows, int ctx, int iters, doubl
     if (!h.has_model) throw SaraError(SARA_EINVAL, "profiling needs a model");
     if (which < 0 || which > K_LMHEAD) throw SaraError(SARA_EINVAL, "unknown kernel id");
     if (rows < 1 || rows > m.max_seqs || iters < 1 || !ms) throw SaraError(SARA_EINVAL, "rows / iters out of range");
-    const int steps = which == 0 ? iters + 2 : 0;  // the whole step advances positions
+    const int steps = which == 0 ? 2 * iters + 2 : 0;  // the whole step advances positions
     if (ctx < 2 || ctx + steps + 1 > h.cap_s || steps + 1 > m.max_gen_len) throw SaraError(SARA_EINVAL, "ctx out of range");
     cudaStream_t s = h.stream;
     StepConst K{};
@@ -817,16 +821,28 @@ void profile_impl(sara_handle &h, int which, int rows, int ctx, int iters, doubl
     CK(cudaMemsetAsync(h.stamps, 0, (size_t)h.sms * 16 * 8, s));
 #endif
     CK(cudaStreamSynchronize(s));
-    auto one = [&] {
-        if (which == 0) enqueue_forward(h, s, true, h.use_pdl, nullptr);
-        else enqueue_kernel(h, s, true, which, 0, false, nullptr);
+    auto one = [&](cudaStream_t st) {
+        if (which == 0) enqueue_forward(h, st, true, h.use_pdl, nullptr);
+        else enqueue_kernel(h, st, true, which, 0, h.use_pdl, nullptr);
     };
-    one();
-    one();
+    one(s);
+    one(s);
+    CK(cudaStreamSynchronize(s));
+    // time the launches from a captured graph, so host launch cost is not measured
+    cudaGraph_t g = nullptr;
+    cudaGraphExec_t ge = nullptr;
+    CK(cudaStreamBeginCapture(h.cap_stream, cudaStreamCaptureModeRelaxed));
+    for (int i = 0; i < iters; ++i) one(h.cap_stream);
+    CK(cudaStreamEndCapture(h.cap_stream, &g));
+    CK(cudaGraphInstantiate(&ge, g, 0));
+    CK(cudaGraphLaunch(ge, s));  // warm the graph
+    CK(cudaStreamSynchronize(s));
     CK(cudaEventRecord(h.ev0, s));
-    for (int i = 0; i < iters; ++i) one();
+    CK(cudaGraphLaunch(ge, s));
     CK(cudaEventRecord(h.ev1, s));
     CK(cudaStreamSynchronize(s));
+    cudaGraphExecDestroy(ge);
+    cudaGraphDestroy(g);
     float t = 0.f;
     CK(cudaEventElapsedTime(&t, h.ev0, h.ev1));
     CK(cudaMemcpy(&v, h.vars, sizeof(v), cudaMemcpyDeviceToHost));
