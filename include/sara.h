@@ -213,6 +213,23 @@ SARA_API int sara_gemm_bf16(const uint16_t *X, const uint16_t *W, float *Y, int3
                             void *stream);
 
 /*
+ * The same GEMM as sara_gemm_bf16 for callers that cannot allocate device memory -- for
+ * example code running inside a host framework whose memory pool has already reserved the
+ * GPU (a raw cudaMalloc there fails or fragments the pool), or a plugin whose interface only
+ * hands over inputs and outputs.  The paper has no counterpart; this is a library service.
+ * It allocates nothing: the stream-K scratch is a fixed array inside the library
+ * (8 MiB of tile sums for at most 64 CTAs + 8 KiB of tile counters), which every GPU that
+ * loads the library holds until the process exits.  The first call on a device looks up
+ * the array's device address (cudaGetSymbolAddress); make that first call before any
+ * stream capture.  Every call shares the array: each call clears what it needs before its
+ * kernel, and calls whose work overlaps on the GPU (several streams or threads) race and
+ * must be serialised by the caller.  Shapes as sara_gemm_bf16, plus Nout <= 262,144
+ * (SARA_EINVAL beyond).  X, W, Y device pointers; work is issued on `stream`.
+ */
+SARA_API int sara_gemm_bf16_static(const uint16_t *X, const uint16_t *W, float *Y, int32_t R,
+                                   int32_t Nout, int32_t K, void *stream);
+
+/*
  * Decode attention for b sequences, one new query each (softmax(q K^T / sqrt(hd)) V with
  * grouped-query heads): q [b][n_heads][hd] bf16; kv cache of sequence i at kv + i*kv_stride
  * elements, laid out [2 (K,V)][n_kv_heads][cap][hd] bf16, valid for positions < ctx[i];

@@ -5,7 +5,7 @@ RMSNorm/RoPE epilogues, Gumbel-max sampling, and the on-device Algorithm 1 contr
 lives in libsara.so, built from csrc/ by build.py.  This package only marshals arguments.
 """
 from .sara import (ABANDONED, COMMITTED, INCOMPLETE, UNDRAWN, Handle, ModelCfg, SaraError, attention_decode,
-                   gemm_bf16, load, model_cfg, sample, tau_fraction)
+                   gemm_bf16, gemm_bf16_static, load, model_cfg, sample, tau_fraction)
 
-__all__ = ["Handle", "ModelCfg", "SaraError", "attention_decode", "gemm_bf16", "load", "model_cfg", "sample",
+__all__ = ["Handle", "ModelCfg", "SaraError", "attention_decode", "gemm_bf16", "gemm_bf16_static", "load", "model_cfg", "sample",
            "tau_fraction", "UNDRAWN", "COMMITTED", "ABANDONED", "INCOMPLETE"]

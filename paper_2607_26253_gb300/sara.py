@@ -20,7 +20,7 @@ SARA_OK, SARA_EINVAL, SARA_ENOMEM, SARA_ETIMEOUT, SARA_EDEVICE = 0, -1, -2, -3, 
 UNDRAWN, COMMITTED, ABANDONED, INCOMPLETE = 0, 2, 3, 4
 EXPORTED = ("sara_create", "sara_collect_step", "sara_teacher_force", "sara_last_error", "sara_destroy",
             "sara_gemm_workspace_bytes", "sara_gemm_bf16", "sara_attention_workspace_bytes",
-            "sara_attention_decode", "sara_sample", "sara_profile")
+            "sara_attention_decode", "sara_sample", "sara_profile", "sara_gemm_bf16_static")
 
 c_p = ctypes.c_void_p
 
@@ -103,6 +103,8 @@ def load(path: str = LIB_PATH):
     lib.sara_profile.argtypes = [c_p, ctypes.c_int32, ctypes.c_int32, ctypes.c_int32, ctypes.c_int32,
                                  ctypes.POINTER(ctypes.c_double)]
     lib.sara_profile.restype = ctypes.c_int
+    lib.sara_gemm_bf16_static.argtypes = [c_p, c_p, c_p, ctypes.c_int32, ctypes.c_int32, ctypes.c_int32, c_p]
+    lib.sara_gemm_bf16_static.restype = ctypes.c_int
     if path == LIB_PATH:
         _lib = lib
     return lib
@@ -266,6 +268,19 @@ def gemm_bf16(X, W, workspace=None):
         workspace = torch.zeros(nbytes, dtype=torch.uint8, device=X.device)
     _check(load().sara_gemm_bf16(X.data_ptr(), W.data_ptr(), Y.data_ptr(), R, N, K, workspace.data_ptr(),
                                  workspace.numel(), torch.cuda.current_stream().cuda_stream))
+    return Y
+
+
+def gemm_bf16_static(X, W, out=None):
+    """Y = X @ W^T like gemm_bf16, through the entry point that allocates nothing (its scratch
+    is a fixed array inside the library).  X [R, K], W [N, K] torch bf16 CUDA; `out` [R, N]
+    fp32 CUDA may be passed so the call itself allocates nothing."""
+    import torch
+    R, K = X.shape
+    N = W.shape[0]
+    Y = out if out is not None else torch.empty((R, N), dtype=torch.float32, device=X.device)
+    _check(load().sara_gemm_bf16_static(X.data_ptr(), W.data_ptr(), Y.data_ptr(), R, N, K,
+                                        torch.cuda.current_stream().cuda_stream))
     return Y
 
 
