@@ -231,9 +231,9 @@ SARA_API int sara_gemm_bf16_static(const uint16_t *X, const uint16_t *W, float *
 
 /*
  * Decode attention for b sequences, one new query each (softmax(q K^T / sqrt(hd)) V with
- * grouped-query heads): q [b][n_heads][hd] bf16; kv cache of sequence i at kv + i*kv_stride
- * elements, laid out [2 (K,V)][n_kv_heads][cap][hd] bf16, valid for positions < ctx[i];
- * out [b][n_heads][hd] bf16.  Split over the context in chunks of 128 positions with an
+ * grouped-query heads): q [b][n_heads][hd] fp16; kv cache of sequence i at kv + i*kv_stride
+ * elements, laid out [2 (K,V)][n_kv_heads][cap][hd] fp16, valid for positions < ctx[i];
+ * out [b][n_heads][hd] bf16 (the high part of the step's bf16 hi/lo output pair).  Split over the context in chunks of 128 positions with an
  * fp32 log-sum-exp combine.  hd in {32, 64, 128}; n_heads / n_kv_heads in {1, 2, 4, 6, 8};
  * max_ctx <= 96 * 128.
  * workspace: >= sara_attention_workspace_bytes(b, n_heads, hd, max_ctx), counter area zero.

@@ -3,6 +3,8 @@
 // Used for decode (row = live rollout, KV = its slot) and for prefill (row = one prompt
 // token, KV = the prompt's slot, causal by construction).
 //
+// q and the KV cache are fp16; the output is a bf16 hi/lo pair (the next GEMM's operand).
+//
 // Work item = (row, split of `chunk` positions) for one KV head (blockIdx.y): the CTA loads
 // the G = n_heads / n_kv query heads that share the KV head once and streams the split's K
 // and V rows (256 contiguous bytes each at hd = 128) exactly once with 16-byte loads, the
@@ -23,9 +25,10 @@ constexpr int kAttnPPI = 4;         // positions per half-warp per iteration
 constexpr int kAttnMaxSplits = 96;  // largest split count the merge handles in shared memory
 
 struct AttnParams {
-    const uint16_t *q;        // [rows][n_heads][hd]
-    uint16_t *out;            // [rows][n_heads][hd]
-    const uint16_t *kv;       // slot s at kv + s * slot_stride: [2][n_kv][cap][hd]
+    const uint16_t *q;        // [rows][n_heads][hd] fp16
+    uint16_t *out;            // [rows][n_heads][hd] bf16 hi
+    uint16_t *out_lo;         // [rows][n_heads][hd] bf16 lo (may be null)
+    const uint16_t *kv;       // slot s at kv + s * slot_stride: [2][n_kv][cap][hd] fp16
     int64_t slot_stride;
     int cap;
     const int *row_slot;      // [rows]
@@ -47,6 +50,20 @@ struct AttnParams {
 #else
 #define ATTN_STAMP(i) do { } while (0)
 #endif
+
+__device__ __forceinline__ float2 half2_bits_to_float2(uint32_t w) {
+    __half2 h;
+    *reinterpret_cast<uint32_t *>(&h) = w;
+    return __half22float2(h);
+}
+
+// bf16 hi/lo store of one output element
+__device__ __forceinline__ void attn_store(const AttnParams &p, int64_t idx, float v) {
+    uint16_t hi, lo;
+    split_bf16(v, hi, lo);
+    p.out[idx] = hi;
+    if (p.out_lo) p.out_lo[idx] = lo;
+}
 
 template <int DPL>
 __device__ __forceinline__ void attn_load_words(const uint16_t *p, uint32_t (&w)[DPL / 2]) {
@@ -103,8 +120,9 @@ attn_rows_kernel(AttnParams p) {
             attn_load_words<DPL>(p.q + ((int64_t)row * p.n_heads + kvh * G + g) * HD + dl * DPL, w);
 #pragma unroll
             for (int i = 0; i < NW; ++i) {
-                q[g][2 * i] = __uint_as_float(w[i] << 16) * p.scale_log2;
-                q[g][2 * i + 1] = __uint_as_float(w[i] & 0xffff0000u) * p.scale_log2;
+                const float2 f = half2_bits_to_float2(w[i]);
+                q[g][2 * i] = f.x * p.scale_log2;
+                q[g][2 * i + 1] = f.y * p.scale_log2;
             }
         }
         float m[G], l[G], o[G][DPL];
@@ -140,10 +158,12 @@ attn_rows_kernel(AttnParams p) {
             for (int j = 0; j < kAttnPPI; ++j)
 #pragma unroll
                 for (int i = 0; i < NW; ++i) {
-                    kf[j][2 * i] = __uint_as_float(kw[j][i] << 16);
-                    kf[j][2 * i + 1] = __uint_as_float(kw[j][i] & 0xffff0000u);
-                    vf[j][2 * i] = __uint_as_float(vw[j][i] << 16);
-                    vf[j][2 * i + 1] = __uint_as_float(vw[j][i] & 0xffff0000u);
+                    const float2 k2 = half2_bits_to_float2(kw[j][i]);
+                    const float2 v2 = half2_bits_to_float2(vw[j][i]);
+                    kf[j][2 * i] = k2.x;
+                    kf[j][2 * i + 1] = k2.y;
+                    vf[j][2 * i] = v2.x;
+                    vf[j][2 * i + 1] = v2.y;
                 }
 #pragma unroll
             for (int g = 0; g < G; ++g) {
@@ -212,7 +232,7 @@ attn_rows_kernel(AttnParams p) {
 #pragma unroll
                 for (int h = 0; h < 8; ++h)
                     if (s_m[h][g] != -INFINITY) acc += s_o[h][g][d] * exp2f(s_m[h][g] - M);
-                p.out[((int64_t)row * p.n_heads + kvh * G + g) * HD + d] = f32_to_bf16(acc / s_fin_l[g]);
+                attn_store(p, ((int64_t)row * p.n_heads + kvh * G + g) * HD + d, acc / s_fin_l[g]);
             }
         } else {
             float *mine = p.part + ((int64_t)item * p.n_kv + kvh) * G * (HD + 2);
@@ -268,7 +288,7 @@ attn_rows_kernel(AttnParams p) {
                     const float *src = base + g * (HD + 2) + 2 + d;
 #pragma unroll 4
                     for (int sp = 0; sp < nsplit; ++sp) acc += s_w[g][sp] * __ldcg(src + sp * sp_stride);
-                    p.out[((int64_t)row * p.n_heads + kvh * G + g) * HD + d] = f32_to_bf16(acc / s_fin_l[g]);
+                    attn_store(p, ((int64_t)row * p.n_heads + kvh * G + g) * HD + d, acc / s_fin_l[g]);
                 }
                 ATTN_STAMP(6);
             }

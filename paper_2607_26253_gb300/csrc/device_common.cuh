@@ -5,6 +5,7 @@
 #pragma once
 #include <cuda.h>
 #include <cuda_bf16.h>
+#include <cuda_fp16.h>
 #include <cuda_runtime.h>
 #include <stdint.h>
 
@@ -55,6 +56,20 @@ __device__ __forceinline__ float gumbel_from_hash(uint64_t h) {
 __device__ __forceinline__ float bf16_to_f32(uint16_t b) { return __uint_as_float((uint32_t)b << 16); }
 __device__ __forceinline__ uint16_t f32_to_bf16(float f) {
     return __bfloat16_as_ushort(__float2bfloat16_rn(f));
+}
+
+// fp16 bit pattern of f, saturated to the finite range (the KV cache and q are fp16).
+__device__ __forceinline__ uint16_t f32_to_f16_sat(float f) {
+    f = fminf(fmaxf(f, -65504.0f), 65504.0f);
+    return __half_as_ushort(__float2half_rn(f));
+}
+__device__ __forceinline__ float f16_to_f32(uint16_t b) { return __half2float(__ushort_as_half(b)); }
+
+// An fp32 value as two bf16 values hi + lo (hi = bf16(v), lo = bf16(v - hi)), so that a
+// bf16 tensor-core product with a bf16 weight keeps ~16 mantissa bits of the activation.
+__device__ __forceinline__ void split_bf16(float v, uint16_t &hi, uint16_t &lo) {
+    hi = f32_to_bf16(v);
+    lo = f32_to_bf16(v - bf16_to_f32(hi));
 }
 
 __device__ __forceinline__ uint32_t smem_u32(const void *p) {

@@ -46,9 +46,11 @@ struct DeviceBuf {
 struct Acts {  // activation buffers of one row set (decode or prefill)
     int rows_cap = 0;
     float *x_f32 = nullptr;
-    uint16_t *xg = nullptr, *q = nullptr, *att = nullptr, *h = nullptr;
+    // GEMM operands as bf16 hi/lo pairs; q is fp16
+    uint16_t *xg = nullptr, *xg_lo = nullptr, *q = nullptr, *att = nullptr, *att_lo = nullptr, *h = nullptr,
+             *h_lo = nullptr;
     float *ssq_a = nullptr, *ssq_m = nullptr;
-    CUtensorMap tm_xg{}, tm_att{}, tm_h{};
+    CUtensorMap tm_xg{}, tm_xg_lo{}, tm_att{}, tm_att_lo{}, tm_h{}, tm_h_lo{};
 };
 
 }  // namespace
@@ -151,9 +153,11 @@ int gemm_grid(int sms, int tiles, bool decode) {
 }
 
 template <int EPI>
-void launch_gemm(cudaStream_t s, bool pdl, int grid, const CUtensorMap &tw, const CUtensorMap &tx, const GemmParams &p) {
+void launch_gemm(cudaStream_t s, bool pdl, int grid, const CUtensorMap &tw, const CUtensorMap &tx,
+                 const CUtensorMap &tx_lo, GemmParams p) {
     grid = gemm_grid(grid, p.m_tiles, p.decode != 0);
-    launch(s, pdl, dim3(grid), dim3(kGemmThreads), kGemmSmemBytes, gemm_tc_kernel<EPI>, tw, tx, p);
+    p.has_lo = 1;
+    launch(s, pdl, dim3(grid), dim3(kGemmThreads), kGemmSmemBytes, gemm_tc_kernel<EPI>, tw, tx, tx_lo, p);
 }
 
 template <int HD>
@@ -223,13 +227,14 @@ void enqueue_kernel(sara_handle &h, cudaStream_t s, bool decode, int which, int 
             p.kv = kv_l;
             p.kv_slot_stride = decode ? h.kv_seq_slot : h.kv_pr_slot;
             p.kv_cap = decode ? h.cap_s : h.cap_p;
-            launch_gemm<EPI_QKV>(s, pdl, G, h.tm_qkv[l], A.tm_xg, p);
+            launch_gemm<EPI_QKV>(s, pdl, G, h.tm_qkv[l], A.tm_xg, A.tm_xg_lo, p);
             break;
         }
         case K_ATTN: {
             AttnParams a{};
             a.q = A.q;
             a.out = A.att;
+            a.out_lo = A.att_lo;
             a.kv = kv_l;
             a.slot_stride = decode ? h.kv_seq_slot : h.kv_pr_slot;
             a.cap = decode ? h.cap_s : h.cap_p;
@@ -253,28 +258,31 @@ void enqueue_kernel(sara_handle &h, cudaStream_t s, bool decode, int which, int 
             GemmParams p = gemm_base(h, d / 128, H * hd / 64, A, rows_dev, decode);
             p.x_f32 = A.x_f32;
             p.xg_out = A.xg;
+            p.xg_lo = A.xg_lo;
             p.g_next = h.mlp_norm[l];
             p.ssq_out = A.ssq_m;
             p.ld = d;
-            launch_gemm<EPI_RESID>(s, pdl, G, h.tm_o[l], A.tm_att, p);
+            launch_gemm<EPI_RESID>(s, pdl, G, h.tm_o[l], A.tm_att, A.tm_att_lo, p);
             break;
         }
         case K_GATEUP: {
             GemmParams p = gemm_base(h, 2 * F / 128, d / 64, A, rows_dev, decode);
             p.ssq = A.ssq_m;
             p.h_out = A.h;
+            p.h_lo = A.h_lo;
             p.ld = F;
-            launch_gemm<EPI_SWIGLU>(s, pdl, G, h.tm_gu[l], A.tm_xg, p);
+            launch_gemm<EPI_SWIGLU>(s, pdl, G, h.tm_gu[l], A.tm_xg, A.tm_xg_lo, p);
             break;
         }
         case K_DOWN: {
             GemmParams p = gemm_base(h, d / 128, F / 64, A, rows_dev, decode);
             p.x_f32 = A.x_f32;
             p.xg_out = A.xg;
+            p.xg_lo = A.xg_lo;
             p.g_next = last ? h.final_norm : h.attn_norm[l + 1];
             p.ssq_out = A.ssq_a;
             p.ld = d;
-            launch_gemm<EPI_RESID>(s, pdl, G, h.tm_down[l], A.tm_h, p);
+            launch_gemm<EPI_RESID>(s, pdl, G, h.tm_down[l], A.tm_h, A.tm_h_lo, p);
             break;
         }
         case K_LMHEAD: {
@@ -285,7 +293,7 @@ void enqueue_kernel(sara_handle &h, cudaStream_t s, bool decode, int which, int 
             p.row_seed = c.row_seed;
             p.arg_val = h.lm_val;
             p.arg_idx = h.lm_idx;
-            launch_gemm<EPI_LMHEAD>(s, pdl, G, h.tm_lm, A.tm_xg, p);
+            launch_gemm<EPI_LMHEAD>(s, pdl, G, h.tm_lm, A.tm_xg, A.tm_xg_lo, p);
             break;
         }
         default: throw SaraError(SARA_EINVAL, "unknown kernel id");
@@ -302,7 +310,7 @@ void enqueue_forward(sara_handle &h, cudaStream_t s, bool decode, bool pdl, floa
     const int *rows_dev = decode ? &h.vars->live : &h.vars->pre_rows;
     launch(s, false, dim3(A.rows_cap), dim3(128), 0, embed_kernel, (const uint16_t *)h.embed,
            (const uint16_t *)h.attn_norm[0], rows_dev, decode ? (const int *)c.row_tok : (const int *)c.pre_tok,
-           m.d_model, A.rows_cap, m.vocab, A.x_f32, A.xg, A.ssq_a, &h.vars->err);
+           m.d_model, A.rows_cap, m.vocab, A.x_f32, A.xg, A.xg_lo, A.ssq_a, &h.vars->err);
     for (int l = 0; l < m.layers; ++l) {
         enqueue_kernel(h, s, decode, K_QKV, l, pdl, nullptr);
         if (!decode && l == m.layers - 1) break;  // the prompt's last hidden state is not needed
@@ -450,9 +458,12 @@ void alloc_acts(sara_handle &h, Acts &A, int rows) {
     const int d = m.d_model, Hhd = m.n_heads * m.head_dim;
     A.x_f32 = h.mem.alloc<float>((size_t)rows * d);
     A.xg = h.mem.alloc<uint16_t>((size_t)rows * d);
+    A.xg_lo = h.mem.alloc<uint16_t>((size_t)rows * d);
     A.q = h.mem.alloc<uint16_t>((size_t)rows * Hhd);
     A.att = h.mem.alloc<uint16_t>((size_t)rows * Hhd);
+    A.att_lo = h.mem.alloc<uint16_t>((size_t)rows * Hhd);
     A.h = h.mem.alloc<uint16_t>((size_t)rows * m.ffn);
+    A.h_lo = h.mem.alloc<uint16_t>((size_t)rows * m.ffn);
     A.ssq_a = h.mem.alloc<float>((size_t)(d / 128) * rows);
     A.ssq_m = h.mem.alloc<float>((size_t)(d / 128) * rows);
 }
@@ -469,8 +480,11 @@ void make_tensor_maps(sara_handle &h) {
     h.tm_lm = make_tmap_bf16(h.lm_head, d, m.vocab, kTileK, kTileM);
     for (Acts *A : {&h.dec, &h.pre}) {
         A->tm_xg = make_tmap_bf16(A->xg, d, A->rows_cap, kTileK, kXBoxRows);
+        A->tm_xg_lo = make_tmap_bf16(A->xg_lo, d, A->rows_cap, kTileK, kXBoxRows);
         A->tm_att = make_tmap_bf16(A->att, H * hd, A->rows_cap, kTileK, kXBoxRows);
+        A->tm_att_lo = make_tmap_bf16(A->att_lo, H * hd, A->rows_cap, kTileK, kXBoxRows);
         A->tm_h = make_tmap_bf16(A->h, F, A->rows_cap, kTileK, kXBoxRows);
+        A->tm_h_lo = make_tmap_bf16(A->h_lo, F, A->rows_cap, kTileK, kXBoxRows);
     }
 }
 

@@ -88,7 +88,7 @@ int sara_gemm_bf16_static(const uint16_t *X, const uint16_t *W, float *Y, int32_
         p.err = nullptr;
         p.y_f32 = Y;
         p.ld = Nout;
-        gemm_tc_kernel<EPI_F32><<<grid, kGemmThreads, kGemmSmemBytes, s>>>(tw, tx, p);
+        gemm_tc_kernel<EPI_F32><<<grid, kGemmThreads, kGemmSmemBytes, s>>>(tw, tx, tx, p);
         CK(cudaGetLastError());
         return SARA_OK;
     } catch (const SaraError &e) {

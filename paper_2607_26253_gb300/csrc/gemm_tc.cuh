@@ -2,7 +2,10 @@
 //     Y[r][n] = sum_c X[r][c] * W[n][c]        (X: activations, W: a linear layer's weight)
 // computed "swap-AB" on the 5th-generation tensor core: the weight tile is the MMA's A
 // operand (M = 128 output features), the activation rows are B (N = rows rounded up to
-// 16, <= 128), the fp32 accumulator lives in tensor memory.  Operands are staged in shared
+// 16, <= 128), the fp32 accumulator lives in tensor memory.  Activations arrive as a bf16
+// pair hi + lo (hi = bf16(x), lo = bf16(x - hi)); both are multiplied with the same weight
+// tile into the same accumulator, so the product keeps ~16 mantissa bits of x at the cost of
+// one extra MMA per weight tile (the GEMM is weight-bandwidth bound).  Operands are staged in shared
 // memory by TMA (128-byte swizzle) through a multi-stage mbarrier pipeline; one elected
 // thread issues tcgen05.mma; four epilogue warps read the accumulator with tcgen05.ld.
 //
@@ -26,14 +29,14 @@ namespace sara {
 
 enum EpiKind : int {
     EPI_F32 = 0,     // Y fp32 [rows][ld]
-    EPI_QKV = 1,     // RMSNorm scale, RoPE on q/k, q -> q_out, k/v -> KV cache
-    EPI_RESID = 2,   // x += Y; xg = bf16(x * g_next); per-tile sum of squares of x
-    EPI_SWIGLU = 3,  // RMSNorm scale; tile = 64 gate rows + 64 up rows -> h = silu(g) * u
+    EPI_QKV = 1,     // RMSNorm scale, RoPE on q/k, q -> q_out (fp16), k/v -> KV cache (fp16)
+    EPI_RESID = 2,   // x += Y; xg = x * g_next as a bf16 hi/lo pair; per-tile sum of squares of x
+    EPI_SWIGLU = 3,  // RMSNorm scale; tile = 64 gate rows + 64 up rows -> h = silu(g) * u (hi/lo)
     EPI_LMHEAD = 4,  // RMSNorm scale; optional fp32 logits; Gumbel-max partial argmax per tile
 };
 
 constexpr int kGemmThreads = 192;
-constexpr int kGemmStages = 5;
+constexpr int kGemmStages = 4;
 constexpr int kTileM = 128;       // weight rows per tile (MMA M)
 constexpr int kTileK = 64;        // reduction elements per pipeline stage (128 B of bf16)
 constexpr int kTileR = 128;       // activation rows per tile (max MMA N here)
@@ -48,6 +51,7 @@ struct GemmParams {
     const int *rows_dev;       // device count of valid rows (nullptr -> rows_fixed)
     int rows_fixed;
     int decode;                // 1: a single row tile, weights prefetched before the PDL wait
+    int has_lo;                // 1: the activation's lo part (second tensor map) is multiplied too
     unsigned long long *ws_acc;  // [gridDim.x][kTileR * kTileM] fixed-point tile sums, zero between launches
     int *ws_cnt;               // [tiles] arrival counters, zero between launches
     int *err;
@@ -55,7 +59,7 @@ struct GemmParams {
     float *y_f32; int ld;      // EPI_F32 output, EPI_LMHEAD logits (optional); row stride
     const float *ssq;          // [ssq_tiles][rows_cap] per-128-feature partial sums of x^2
     int ssq_tiles; float inv_dim; float eps;
-    uint16_t *q_out;           // EPI_QKV: [rows][n_heads * head_dim]
+    uint16_t *q_out;           // EPI_QKV: [rows][n_heads * head_dim] fp16
     int n_heads, n_kv, head_dim;
     const float2 *rope;        // [positions][head_dim / 2] (cos, sin)
     const int *row_pos;        // [rows] position of the row's token
@@ -64,10 +68,12 @@ struct GemmParams {
     int64_t kv_slot_stride;    //   laid out [2][n_kv][kv_cap][head_dim]
     int kv_cap;
     float *x_f32;              // EPI_RESID residual stream [rows][ld]
-    uint16_t *xg_out;          // EPI_RESID bf16(x * g_next) [rows][ld]
+    uint16_t *xg_out;          // EPI_RESID x * g_next, bf16 hi [rows][ld]
+    uint16_t *xg_lo;           //   and bf16 lo
     const uint16_t *g_next;    // EPI_RESID next RMSNorm weight [ld]
     float *ssq_out;            // EPI_RESID [m_tiles][rows_cap]
-    uint16_t *h_out;           // EPI_SWIGLU [rows][ld]
+    uint16_t *h_out;           // EPI_SWIGLU [rows][ld] bf16 hi
+    uint16_t *h_lo;            //   and bf16 lo
     const uint64_t *row_seed;  // EPI_LMHEAD sampler key of the row
     float *arg_val; int *arg_idx;  // EPI_LMHEAD [rows][m_tiles] partial max / argmax
     uint64_t *stamps;          // optional [gridDim.x][16] phase timestamps (profiling builds)
@@ -93,7 +99,7 @@ struct GemmSmem {
 };
 
 constexpr size_t kGemmSmemBytes =
-    1024 /* alignment slack */ + (size_t)kGemmStages * (kWStageBytes + kXStageBytes) + sizeof(GemmSmem);
+    1024 /* alignment slack */ + (size_t)kGemmStages * (kWStageBytes + 2 * kXStageBytes) + sizeof(GemmSmem);
 
 // Stream-K partition: CTA c owns units [unit_begin(c), unit_begin(c+1)).
 __device__ __forceinline__ int64_t unit_begin(int c, int64_t U, int G) { return (int64_t)c * U / G; }
@@ -138,7 +144,10 @@ __device__ __forceinline__ void gemm_epilogue_chunk(const GemmParams &p, GemmSme
                 const int64_t idx = (int64_t)(r_base + c0 + c) * p.ld + n;
                 const float x = xo[c] + v[c];
                 p.x_f32[idx] = x;
-                p.xg_out[idx] = f32_to_bf16(x * g);
+                uint16_t hi, lo;
+                split_bf16(x * g, hi, lo);
+                p.xg_out[idx] = hi;
+                p.xg_lo[idx] = lo;
                 v[c] = x * x;
             }
         }
@@ -178,13 +187,13 @@ __device__ __forceinline__ void gemm_epilogue_chunk(const GemmParams &p, GemmSme
                     y = (i < half) ? (y * cs[c].x - o * cs[c].y) : (y * cs[c].x + o * cs[c].y);
                 }
                 if (head < nq) {
-                    p.q_out[(int64_t)r * (nq * hd) + n] = f32_to_bf16(y);
+                    p.q_out[(int64_t)r * (nq * hd) + n] = f32_to_f16_sat(y);
                 } else {
                     const int isv = head >= nq + nkv;
                     const int kvh = head - nq - isv * nkv;
                     uint16_t *dst = p.kv + (int64_t)S.row_slot[c0 + c] * p.kv_slot_stride +
                                     ((int64_t)(isv * nkv + kvh) * p.kv_cap + S.row_pos[c0 + c]) * hd + i;
-                    *dst = f32_to_bf16(y);
+                    *dst = f32_to_f16_sat(y);
                 }
             }
         }
@@ -196,7 +205,10 @@ __device__ __forceinline__ void gemm_epilogue_chunk(const GemmParams &p, GemmSme
                 if (c < ncols) {
                     const float g = v[c], u = S.xch[(mrow + 64) * kEpiLd + c];
                     const float h = g / (1.0f + expf(-g)) * u;
-                    p.h_out[(int64_t)(r_base + c0 + c) * p.ld + f] = f32_to_bf16(h);
+                    uint16_t hi, lo;
+                    split_bf16(h, hi, lo);
+                    p.h_out[(int64_t)(r_base + c0 + c) * p.ld + f] = hi;
+                    p.h_lo[(int64_t)(r_base + c0 + c) * p.ld + f] = lo;
                 }
             }
         }
@@ -234,12 +246,14 @@ __device__ __forceinline__ void gemm_epilogue_chunk(const GemmParams &p, GemmSme
 
 template <int EPI>
 __global__ void __launch_bounds__(kGemmThreads, 1)
-gemm_tc_kernel(const __grid_constant__ CUtensorMap tmW, const __grid_constant__ CUtensorMap tmX, GemmParams p) {
+gemm_tc_kernel(const __grid_constant__ CUtensorMap tmW, const __grid_constant__ CUtensorMap tmX,
+               const __grid_constant__ CUtensorMap tmXlo, GemmParams p) {
     extern __shared__ uint8_t smem_raw[];
     uint8_t *base = reinterpret_cast<uint8_t *>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~(uintptr_t)1023);
     uint8_t *sW = base;
     uint8_t *sX = base + (size_t)kGemmStages * kWStageBytes;
-    GemmSmem &S = *reinterpret_cast<GemmSmem *>(sX + (size_t)kGemmStages * kXStageBytes);
+    uint8_t *sXlo = sX + (size_t)kGemmStages * kXStageBytes;
+    GemmSmem &S = *reinterpret_cast<GemmSmem *>(sXlo + (size_t)kGemmStages * kXStageBytes);
 
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const int G = gridDim.x, cta = blockIdx.x;
@@ -255,6 +269,7 @@ gemm_tc_kernel(const __grid_constant__ CUtensorMap tmW, const __grid_constant__ 
         fence_mbar_init();
         prefetch_tensormap(&tmW);
         prefetch_tensormap(&tmX);
+        if (p.has_lo) prefetch_tensormap(&tmXlo);
     }
     if (warp == 1) { tmem_alloc(&S.tmem_base, 256); tmem_relinquish(); }
     tc_fence_before();
@@ -309,16 +324,20 @@ gemm_tc_kernel(const __grid_constant__ CUtensorMap tmW, const __grid_constant__ 
                 const int m_tile = tile % m_tiles, r_tile = tile / m_tiles;
                 const int rin = min(kTileR, max(rows - r_tile * kTileR, 0));
                 const int nbox = max(1, (rin + kXBoxRows - 1) / kXBoxRows);
-                const uint32_t xbytes = (uint32_t)(nbox * kXBoxRows * kTileK * 2);
+                const uint32_t xbytes = (uint32_t)(nbox * kXBoxRows * kTileK * 2) * (p.has_lo ? 2u : 1u);
                 if (i >= n_pre) {
                     mbar_arrive_expect_tx(&S.full[s], (uint32_t)kWStageBytes + xbytes);
                     tma_load_2d(sW + (size_t)s * kWStageBytes, &tmW, &S.full[s], kc * kTileK, m_tile * kTileM, pol_w);
                 } else {
                     mbar_arrive_expect_tx(&S.full[s], xbytes);
                 }
-                for (int b = 0; b < nbox; ++b)
+                for (int b = 0; b < nbox; ++b) {
                     tma_load_2d(sX + (size_t)s * kXStageBytes + b * kXBoxRows * kTileK * 2, &tmX, &S.full[s],
                                 kc * kTileK, r_tile * kTileR + b * kXBoxRows, pol_x);
+                    if (p.has_lo)
+                        tma_load_2d(sXlo + (size_t)s * kXStageBytes + b * kXBoxRows * kTileK * 2, &tmXlo, &S.full[s],
+                                    kc * kTileK, r_tile * kTileR + b * kXBoxRows, pol_x);
+                }
             }
             // On abort, the last load issued on every stage lands before the CTA exits.
             if (*(volatile int *)&S.abort_flag) {
@@ -364,10 +383,12 @@ gemm_tc_kernel(const __grid_constant__ CUtensorMap tmW, const __grid_constant__ 
                     if (i == 0) GEMM_STAMP(2);
                     const uint32_t aw = smem_u32(sW + (size_t)s * kWStageBytes);
                     const uint32_t ax = smem_u32(sX + (size_t)s * kXStageBytes);
+                    const uint32_t axl = smem_u32(sXlo + (size_t)s * kXStageBytes);
 #pragma unroll
                     for (int kk = 0; kk < kTileK / 16; ++kk) {
-                        tc_mma_bf16(d, sdesc_kmajor_sw128(aw + kk * 32), sdesc_kmajor_sw128(ax + kk * 32), idesc,
-                                    (first && kk == 0) ? 0u : 1u);
+                        const uint64_t adesc = sdesc_kmajor_sw128(aw + kk * 32);
+                        tc_mma_bf16(d, adesc, sdesc_kmajor_sw128(ax + kk * 32), idesc, (first && kk == 0) ? 0u : 1u);
+                        if (p.has_lo) tc_mma_bf16(d, adesc, sdesc_kmajor_sw128(axl + kk * 32), idesc, 1u);
                     }
                     first = false;
                     tc_commit(&S.empty[s]);

@@ -102,7 +102,7 @@ int sara_gemm_bf16(const uint16_t *X, const uint16_t *W, float *Y, int32_t R, in
         p.err = nullptr;
         p.y_f32 = Y;
         p.ld = Nout;
-        gemm_tc_kernel<EPI_F32><<<sms, kGemmThreads, kGemmSmemBytes, static_cast<cudaStream_t>(stream)>>>(tw, tx, p);
+        gemm_tc_kernel<EPI_F32><<<sms, kGemmThreads, kGemmSmemBytes, static_cast<cudaStream_t>(stream)>>>(tw, tx, tx, p);
         CK(cudaGetLastError());
     });
 }

@@ -8,11 +8,12 @@
 
 namespace sara {
 
-// x_f32[r] = E[tok[r]]; xg[r] = bf16(x * g); ssq[t][r] = sum over features [128t, 128t+128)
-// of x^2.  One CTA (128 threads) per row; rows >= *rows_dev exit.
+// x_f32[r] = E[tok[r]]; xg[r] = x * g as a bf16 hi/lo pair; ssq[t][r] = sum over features
+// [128t, 128t+128) of x^2.  One CTA (128 threads) per row; rows >= *rows_dev exit.
 static __global__ void __launch_bounds__(128) embed_kernel(const uint16_t *E, const uint16_t *g, const int *rows_dev,
                                                            const int *row_tok, int d, int rows_cap, int vocab,
-                                                           float *x_f32, uint16_t *xg, float *ssq, int *err) {
+                                                           float *x_f32, uint16_t *xg, uint16_t *xg_lo, float *ssq,
+                                                           int *err) {
     pdl_wait_prior_grids();
     pdl_allow_dependents();
     const int rows = min(*rows_dev, rows_cap);
@@ -28,7 +29,10 @@ static __global__ void __launch_bounds__(128) embed_kernel(const uint16_t *E, co
             const int f = t * 128 + threadIdx.x;
             const float x = bf16_to_f32(er[f]);
             x_f32[(int64_t)r * d + f] = x;
-            xg[(int64_t)r * d + f] = f32_to_bf16(x * bf16_to_f32(g[f]));
+            uint16_t hi, lo;
+            split_bf16(x * bf16_to_f32(g[f]), hi, lo);
+            xg[(int64_t)r * d + f] = hi;
+            xg_lo[(int64_t)r * d + f] = lo;
             const float s = warp_sum(x * x);
             if ((threadIdx.x & 31) == 0) red[threadIdx.x >> 5] = s;
             __syncthreads();

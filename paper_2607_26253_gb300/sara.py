@@ -285,11 +285,12 @@ def gemm_bf16_static(X, W, out=None):
 
 
 def attention_decode(q, kv, ctx, n_kv_heads: int, cap: int, max_ctx: int | None = None):
-    """Decode attention: q [b, H, hd] bf16, kv [b, 2, KVH, cap, hd] bf16, ctx [b] int32 (CUDA)."""
+    """Decode attention: q [b, H, hd] fp16, kv [b, 2, KVH, cap, hd] fp16, ctx [b] int32 (CUDA);
+    returns bf16 [b, H, hd]."""
     import torch
     b, H, hd = q.shape
     max_ctx = int(ctx.max().item()) if max_ctx is None else max_ctx
-    out = torch.empty_like(q)
+    out = torch.empty(q.shape, dtype=torch.bfloat16, device=q.device)
     nbytes = load().sara_attention_workspace_bytes(b, H, hd, max_ctx)
     ws = torch.zeros(nbytes, dtype=torch.uint8, device=q.device)
     _check(load().sara_attention_decode(q.data_ptr(), kv.data_ptr(), kv.stride(0), ctx.data_ptr(), out.data_ptr(),

@@ -79,19 +79,19 @@ def _attention_ref(q, kv, ctx, n_kv):
 @pytest.mark.parametrize("hd,H,KVH,ctxs", [(128, 12, 2, [1, 17, 256, 257, 1000]),
                                           (128, 16, 2, [4096, 300, 2]),
                                           (32, 4, 2, [1, 31, 64, 513]),
-                                          (64, 8, 8, [100, 255])])
+                                          (64, 8, 8, [100, 255]),
+                                          (128, 8, 2, [8576, 129])])
 def test_attention_matches_float64(pkg, hd, H, KVH, ctxs):
     import torch
     rng = np.random.default_rng(hd + H + len(ctxs))
     b = len(ctxs)
     cap = max(ctxs) + 16
-    q = _bf16(rng, (b, H, hd))
-    kv = _bf16(rng, (b, 2, KVH, cap, hd))
+    q = rng.standard_normal((b, H, hd)).astype(np.float16)
+    kv = rng.standard_normal((b, 2, KVH, cap, hd)).astype(np.float16)
     ctx = np.array(ctxs, np.int32)
-    out = pkg.attention_decode(_dev_bf16(q), _dev_bf16(kv), _dev(ctx), KVH, cap)
+    out = pkg.attention_decode(torch.from_numpy(q).cuda(), torch.from_numpy(kv).cuda(), _dev(ctx), KVH, cap)
     got = synth.bf16_bits_to_f32(out.view(torch.int16).cpu().numpy().view(np.uint16)).astype(np.float64)
-    want = _attention_ref(synth.bf16_bits_to_f32(q).astype(np.float64),
-                          synth.bf16_bits_to_f32(kv).astype(np.float64), ctx, KVH)
+    want = _attention_ref(q.astype(np.float64), kv.astype(np.float64), ctx, KVH)
     # the bf16 rounding of the output (2^-9 relative) dominates
     assert np.all(np.abs(got - want) <= 2.0 ** -8 * np.abs(want) + 1e-3)
 
