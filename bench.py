@@ -133,6 +133,13 @@ def decode_algorithmic_bytes(m: synth.ModelShape, Lp: int, lens: np.ndarray) -> 
     return ctx_sum * kvtok + L.sum() * kvtok + L.sum() * m.d_model * 2
 
 
+def step_algorithmic_bytes(m: synth.ModelShape, rows: int, ctx: int) -> float:
+    """Bytes one decode step over `rows` rows at context `ctx` must move: the weights once,
+    the K/V of every context position read, the new K/V written, the embedding rows."""
+    kvtok = m.kv_bytes_per_token()
+    return weight_bytes_per_step(m) + rows * (ctx - 1) * kvtok + rows * kvtok + rows * m.d_model * 2
+
+
 def weight_bytes_per_step(m: synth.ModelShape) -> int:
     return m.layers * (m.layer_weight_bytes() + 4 * m.d_model) + 2 * m.vocab * m.d_model + 2 * m.d_model
 
@@ -268,11 +275,13 @@ def run_mine(args):
     e2e_ms = f0.elapsed_time(f1)
 
     # ------------------------------------------------------------------ dominant kernel roofline
+    # the decode-step kernel (one launch = one whole forward over the live rows) at the
+    # step's mean live rows and the median mid-rollout context
     mean_rows = max(1, int(round(tok / max(dsteps, 1))))
     mid_ctx = w.prompt_len + int(np.median(batches[0][1].lengths)) // 2
-    k_ms = h.profile(4, mean_rows, mid_ctx, iters=50)  # gate/up projection + SwiGLU of layer 0
-    gu_bytes = 2 * m.ffn * m.d_model * 2 + mean_rows * m.d_model * 2 + mean_rows * m.ffn * 2
-    step_ms = h.profile(0, mean_rows, mid_ctx, iters=10)  # whole eager decode step, same rows
+    k_ms = h.profile(1, mean_rows, mid_ctx, iters=20)
+    k_bytes = step_algorithmic_bytes(m, mean_rows, mid_ctx)
+    step_ms = h.profile(0, mean_rows, mid_ctx, iters=20)  # kernel + sampling / bookkeeping
     h.close()
 
     # ------------------------------------------------------------------ reduce over ranks
@@ -289,7 +298,7 @@ def run_mine(args):
         return
 
     peak, peak_kind = peaks()
-    achieved = gu_bytes / (k_ms * 1e-3) / 1e9
+    achieved = k_bytes / (k_ms * 1e-3) / 1e9
     traffic = read_traffic(args.workload)
     cpu = None
     if not args.no_cpu_baseline:
@@ -316,10 +325,12 @@ def run_mine(args):
         "rollouts_per_s": rollouts / (ms * 1e-3),
         "decode_hbm_gbs": dec_bytes / (ms * 1e-3) / 1e9,
         "decode_hbm_frac": dec_bytes / (ms * 1e-3) / 1e9 / peak,
-        "decode_step_ms_eager": step_ms,
+        "decode_step_ms": step_ms,
+        "decode_kernel_ms": k_ms,
         "roofline": {"bound": "hbm", "achieved": achieved, "peak": peak, "unit": "GB/s",
                      "frac": achieved / peak, "traffic": traffic,
-                     "kernel": f"gate/up projection + SwiGLU (layer 0), {mean_rows} live rows",
+                     "kernel": f"decode_step_kernel (whole forward), {mean_rows} live rows at context {mid_ctx}",
+                     "bytes_per_launch": k_bytes,
                      "peak_kind": f"{peak_kind} burst copy"},
         "e2e": {"value": e2e_tok / (e2e_ms * 1e-3), "unit": "tokens/s", "h2d_bytes_per_step": h2d / args.steps,
                 "d2h_bytes_per_step": d2h / args.steps},
@@ -327,10 +338,11 @@ def run_mine(args):
         "gpu_launches": None,
         "clocks": clocks,
     }
-    # kernels launched per step: controller + (round starts) + per decode step 2 + 5 per layer + 2
-    per_step = 2 + 5 * m.layers + 2
-    line["gpu_launches"] = int(dsteps * per_step + sum(o.counters["rounds"] for o in outs) *
-                               (1 + m.layers * 5) + dsteps + args.steps)
+    # kernels launched: per decode step the controller, the decode-step kernel and the
+    # sampling/bookkeeping kernel; per round start the prefill (embedding + 5 per layer
+    # but the last layer's 4) and the KV fan-out; per call the init kernel
+    rounds = sum(o.counters["rounds"] for o in outs)
+    line["gpu_launches"] = int(3 * dsteps + rounds * (1 + 5 * m.layers - 4 + 1) + args.steps)
     print(json.dumps(line))
     if world > 1:
         dist.destroy_process_group()
@@ -338,7 +350,7 @@ def run_mine(args):
 
 def read_traffic(workload: str):
     """DRAM bytes per launch of the dominant kernel from the committed ncu summary, if any."""
-    path = os.path.join(ROOT, "profiles", f"gemm_gateup_{workload.replace('.', 'p')}_ncu.md")
+    path = os.path.join(ROOT, "profiles", f"decode_step_{workload.replace('.', 'p')}_ncu.md")
     try:
         for line in open(path):
             if line.startswith("traffic_bytes_per_launch:"):
@@ -359,8 +371,8 @@ def run_kernel_profile(args):
     w = synth.WORKLOADS[args.workload]
     m = w.model
     weights = synth.model_weights(m, w.weight_seed)
-    cfg = pkg.model_cfg(m, max_prompts=w.n_prompts, max_active=16, max_seqs=32, max_prompt_len=w.prompt_len,
-                        max_gen_len=512, max_k=w.k)
+    cfg = pkg.model_cfg(m, max_prompts=w.n_prompts, max_active=max(16, args.rows), max_seqs=max(32, args.rows),
+                        max_prompt_len=w.prompt_len, max_gen_len=512, max_k=w.k)
     with pkg.Handle(cfg, weights, stream=torch.cuda.current_stream()) as h:
         ms = h.profile(args.kernel_profile, args.rows, w.prompt_len + 128, iters=args.iters)
     print(json.dumps({"kernel": args.kernel_profile, "rows": args.rows, "ms_per_launch": ms}))

@@ -176,12 +176,12 @@ SARA_API int sara_teacher_force(sara_handle *h, int32_t n_seq, int32_t prompt_le
 /*
  * Profiling hook (benchmarks): set `rows` live rollouts at context length `ctx` (synthetic
  * row state; the step's own state is overwritten) and launch, after two warm-up launches,
- * `iters` copies of either one decode kernel of layer 0 or the whole decode step, captured
- * in a CUDA graph (no host launch cost) and timed with CUDA events on the handle's stream.
- * *ms_per_launch = elapsed / iters.
- *   kernel: 0 = whole decode step (eager launches), 1 = QKV projection + RoPE + KV append,
- *           2 = decode attention, 3 = O projection + residual, 4 = gate/up + SwiGLU,
- *           5 = down projection + residual, 6 = lm_head + fused sampling partials.
+ * `iters` copies of the decode step, captured in a CUDA graph (no host launch cost) and
+ * timed with CUDA events on the handle's stream.  *ms_per_launch = elapsed / iters.
+ *   kernel: 0 = whole decode step (the persistent decode-step kernel, then sampling and
+ *               bookkeeping; positions advance by one per launch),
+ *           1 = the decode-step kernel alone (embedding, every layer, lm_head with the
+ *               Gumbel-max partials; positions fixed).
  * Requires 1 <= rows <= max_seqs, ctx >= 2 and room for the positions the launches use.
  */
 SARA_API int sara_profile(sara_handle *h, int32_t kernel, int32_t rows, int32_t ctx, int32_t iters,

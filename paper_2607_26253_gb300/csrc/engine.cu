@@ -1,6 +1,7 @@
-// Host engine behind include/sara.h: device memory layout, weight packing, TMA descriptors,
-// the step graph (a conditional WHILE loop whose body is controller -> [round start:
-// prefill + prompt-KV fan-out] -> decode step -> sampling/bookkeeping), and the C ABI.
+// Host engine behind include/sara.h: device memory layout, weight packing (pre-swizzled
+// 16 KB tiles), the step graph (a conditional WHILE loop whose body is controller ->
+// [round start: prefill + prompt-KV fan-out] -> persistent decode-step kernel ->
+// sampling/bookkeeping), and the C ABI.
 #include <cuda.h>
 #include <cuda_runtime.h>
 
@@ -16,6 +17,7 @@
 #include "../../include/sara.h"
 #include "attention.cuh"
 #include "controller.cuh"
+#include "decode_step.cuh"
 #include "gemm_tc.cuh"
 #include "host_util.h"
 #include "step_kernels.cuh"
@@ -43,7 +45,7 @@ struct DeviceBuf {
     }
 };
 
-struct Acts {  // activation buffers of one row set (decode or prefill)
+struct Acts {  // activation buffers of the prefill rows (row-major, TMA operands)
     int rows_cap = 0;
     float *x_f32 = nullptr;
     // GEMM operands as bf16 hi/lo pairs; q is fp16
@@ -63,17 +65,25 @@ struct sara_handle {
     bool use_graph = true, use_pdl = true;
     std::string err;
     DeviceBuf mem;
-    // weights
-    uint16_t *embed = nullptr, *lm_head = nullptr, *final_norm = nullptr;
-    std::vector<uint16_t *> attn_norm, mlp_norm, w_qkv, w_o, w_gu, w_down;
-    std::vector<CUtensorMap> tm_qkv, tm_o, tm_gu, tm_down;
-    CUtensorMap tm_lm{};
-    // KV caches
-    uint16_t *kv_seq = nullptr, *kv_pr = nullptr;
-    int cap_s = 0, cap_p = 0;
+    // weights: embedding row-major, projections as pre-swizzled 16 KB tiles (all layers
+    // of one kind contiguous), norms [layers][d]
+    uint16_t *embed = nullptr, *final_norm = nullptr, *norm_attn = nullptr, *norm_mlp = nullptr;
+    uint8_t *wb_qkv = nullptr, *wb_o = nullptr, *wb_gu = nullptr, *wb_down = nullptr, *wb_lm = nullptr;
+    int64_t ls_qkv = 0, ls_o = 0, ls_gu = 0, ls_down = 0;
+    // KV caches: rollout slots in the blocked decode layout, prompt slots row-major
+    uint8_t *kv_seq = nullptr;
+    uint16_t *kv_pr = nullptr;
+    int cap_s = 0, cap_p = 0, kv_nblk = 0;
     int64_t kv_seq_layer = 0, kv_seq_slot = 0, kv_pr_layer = 0, kv_pr_slot = 0;
     float2 *rope = nullptr;
-    Acts dec, pre;
+    Acts pre;
+    // decode-step activations (blocked operands) and phase counters
+    int rows_cap16 = 0;
+    float *dx = nullptr, *ssqA = nullptr, *ssqM = nullptr;
+    uint8_t *xg_hi = nullptr, *xg_lo = nullptr, *att_hi = nullptr, *att_lo = nullptr, *h_hi = nullptr, *h_lo = nullptr;
+    unsigned long long *accQ = nullptr, *accO = nullptr, *accGU = nullptr, *accD = nullptr;
+    unsigned long long *phase_cnt = nullptr;  // [1 + 8 layers + 1] then the epoch
+    int n_phase_cnt = 0;
     int pre_cap = 0, att_cap = 0;
     // workspaces
     unsigned long long *gemm_acc = nullptr;
@@ -124,22 +134,36 @@ void set_kernel_attrs() {
     CK(cudaFuncSetAttribute(gemm_tc_kernel<EPI_RESID>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)kGemmSmemBytes));
     CK(cudaFuncSetAttribute(gemm_tc_kernel<EPI_SWIGLU>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)kGemmSmemBytes));
     CK(cudaFuncSetAttribute(gemm_tc_kernel<EPI_LMHEAD>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)kGemmSmemBytes));
+    CK(cudaFuncSetAttribute(decode_step_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)kMegaSmemBytes));
     done = true;
 }
 
 template <typename Kern, typename... Args>
-void launch(cudaStream_t s, bool pdl, dim3 grid, dim3 block, size_t smem, Kern kern, Args... args) {
+void launch_ex(cudaStream_t s, bool pdl, bool coop, dim3 grid, dim3 block, size_t smem, Kern kern, Args... args) {
     cudaLaunchConfig_t cfg{};
     cfg.gridDim = grid;
     cfg.blockDim = block;
     cfg.dynamicSmemBytes = smem;
     cfg.stream = s;
-    cudaLaunchAttribute attr[1];
-    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
-    attr[0].val.programmaticStreamSerializationAllowed = 1;
+    cudaLaunchAttribute attr[2];
+    unsigned n = 0;
+    if (pdl) {
+        attr[n].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+        attr[n].val.programmaticStreamSerializationAllowed = 1;
+        ++n;
+    }
+    if (coop) {  // every CTA resident at once (the decode step's CTAs wait on one another)
+        attr[n].id = cudaLaunchAttributeCooperative;
+        attr[n].val.cooperative = 1;
+        ++n;
+    }
     cfg.attrs = attr;
-    cfg.numAttrs = pdl ? 1 : 0;
+    cfg.numAttrs = n;
     CK(cudaLaunchKernelEx(&cfg, kern, args...));
+}
+template <typename Kern, typename... Args>
+void launch(cudaStream_t s, bool pdl, dim3 grid, dim3 block, size_t smem, Kern kern, Args... args) {
+    launch_ex(s, pdl, false, grid, block, smem, kern, args...);
 }
 
 // Grid of a decode GEMM: one whole tile per CTA when the tile count nearly fills the SMs
@@ -183,13 +207,13 @@ void launch_attention(cudaStream_t s, bool pdl, int sms, int hd, const AttnParam
     }
 }
 
-GemmParams gemm_base(const sara_handle &h, int m_tiles, int k_chunks, const Acts &A, const int *rows_dev, bool decode) {
+GemmParams gemm_base(const sara_handle &h, int m_tiles, int k_chunks, const Acts &A, const int *rows_dev) {
     GemmParams p{};
     p.m_tiles = m_tiles;
     p.k_chunks = k_chunks;
     p.rows_cap = A.rows_cap;
     p.rows_dev = rows_dev;
-    p.decode = decode ? 1 : 0;
+    p.decode = 0;
     p.ws_acc = h.gemm_acc;
     p.ws_cnt = h.gemm_cnt;
     p.err = &h.vars->err;
@@ -200,34 +224,35 @@ GemmParams gemm_base(const sara_handle &h, int m_tiles, int k_chunks, const Acts
     return p;
 }
 
-enum Kern { K_QKV = 1, K_ATTN = 2, K_OPROJ = 3, K_GATEUP = 4, K_DOWN = 5, K_LMHEAD = 6 };
+enum Kern { K_QKV = 1, K_ATTN = 2, K_OPROJ = 3, K_GATEUP = 4, K_DOWN = 5 };
 
-// Launch one projection / attention kernel of layer l for a row set (decode: live rollouts,
-// KV = rollout slots; prefill: fresh prompt tokens, KV = prompt slots).
-void enqueue_kernel(sara_handle &h, cudaStream_t s, bool decode, int which, int l, bool pdl, float *logits_stage) {
+// Launch one projection / attention kernel of layer l over the prefill rows (one row per
+// fresh prompt token, KV = the prompt slots).  Weights are read from the blocked tiles.
+void enqueue_prefill_kernel(sara_handle &h, cudaStream_t s, int which, int l, bool pdl) {
     const sara_model_cfg &m = h.cfg;
     const StepPtrs &c = h.ptrs;
-    Acts &A = decode ? h.dec : h.pre;
-    const int *rows_dev = decode ? &h.vars->live : &h.vars->pre_rows;
+    Acts &A = h.pre;
+    const int *rows_dev = &h.vars->pre_rows;
     const int d = m.d_model, H = m.n_heads, KVH = m.n_kv_heads, hd = m.head_dim, F = m.ffn;
     const int G = h.sms;
     const bool last = l == m.layers - 1;
-    uint16_t *kv_l = decode ? h.kv_seq + l * h.kv_seq_layer : h.kv_pr + l * h.kv_pr_layer;
+    uint16_t *kv_l = h.kv_pr + l * h.kv_pr_layer;
     switch (which) {
         case K_QKV: {
-            GemmParams p = gemm_base(h, (H + 2 * KVH) * hd / 128, d / 64, A, rows_dev, decode);
+            GemmParams p = gemm_base(h, (H + 2 * KVH) * hd / 128, d / 64, A, rows_dev);
+            p.w_blk = h.wb_qkv + l * h.ls_qkv;
             p.ssq = A.ssq_a;
             p.q_out = A.q;
             p.n_heads = H;
             p.n_kv = KVH;
             p.head_dim = hd;
             p.rope = h.rope;
-            p.row_pos = decode ? c.row_pos : c.pre_pos;
-            p.row_slot = decode ? c.row_slot : c.pre_slot;
+            p.row_pos = c.pre_pos;
+            p.row_slot = c.pre_slot;
             p.kv = kv_l;
-            p.kv_slot_stride = decode ? h.kv_seq_slot : h.kv_pr_slot;
-            p.kv_cap = decode ? h.cap_s : h.cap_p;
-            launch_gemm<EPI_QKV>(s, pdl, G, h.tm_qkv[l], A.tm_xg, A.tm_xg_lo, p);
+            p.kv_slot_stride = h.kv_pr_slot;
+            p.kv_cap = h.cap_p;
+            launch_gemm<EPI_QKV>(s, pdl, G, A.tm_xg, A.tm_xg, A.tm_xg_lo, p);
             break;
         }
         case K_ATTN: {
@@ -236,16 +261,16 @@ void enqueue_kernel(sara_handle &h, cudaStream_t s, bool decode, int which, int 
             a.out = A.att;
             a.out_lo = A.att_lo;
             a.kv = kv_l;
-            a.slot_stride = decode ? h.kv_seq_slot : h.kv_pr_slot;
-            a.cap = decode ? h.cap_s : h.cap_p;
-            a.row_slot = decode ? c.row_slot : c.pre_slot;
-            a.row_pos = decode ? c.row_pos : c.pre_pos;
-            a.items = decode ? c.att_items : c.pre_items;
-            a.n_items_dev = decode ? &h.vars->att_items : &h.vars->pre_rows;
-            a.row_item0 = decode ? c.row_item0 : c.pre_item0;
+            a.slot_stride = h.kv_pr_slot;
+            a.cap = h.cap_p;
+            a.row_slot = c.pre_slot;
+            a.row_pos = c.pre_pos;
+            a.items = c.pre_items;
+            a.n_items_dev = &h.vars->pre_rows;
+            a.row_item0 = c.pre_item0;
             a.n_heads = H;
             a.n_kv = KVH;
-            a.chunk = decode ? kDecodeChunk : h.cap_p;  // prefill: one split per row
+            a.chunk = h.cap_p;  // one split per row
             a.scale_log2 = (float)(1.4426950408889634 / std::sqrt((double)hd));
             a.part = h.attn_part;
             a.cnt = h.attn_cnt;
@@ -255,83 +280,138 @@ void enqueue_kernel(sara_handle &h, cudaStream_t s, bool decode, int which, int 
             break;
         }
         case K_OPROJ: {
-            GemmParams p = gemm_base(h, d / 128, H * hd / 64, A, rows_dev, decode);
+            GemmParams p = gemm_base(h, d / 128, H * hd / 64, A, rows_dev);
+            p.w_blk = h.wb_o + l * h.ls_o;
             p.x_f32 = A.x_f32;
             p.xg_out = A.xg;
             p.xg_lo = A.xg_lo;
-            p.g_next = h.mlp_norm[l];
+            p.g_next = h.norm_mlp + (size_t)l * d;
             p.ssq_out = A.ssq_m;
             p.ld = d;
-            launch_gemm<EPI_RESID>(s, pdl, G, h.tm_o[l], A.tm_att, A.tm_att_lo, p);
+            launch_gemm<EPI_RESID>(s, pdl, G, A.tm_att, A.tm_att, A.tm_att_lo, p);
             break;
         }
         case K_GATEUP: {
-            GemmParams p = gemm_base(h, 2 * F / 128, d / 64, A, rows_dev, decode);
+            GemmParams p = gemm_base(h, 2 * F / 128, d / 64, A, rows_dev);
+            p.w_blk = h.wb_gu + l * h.ls_gu;
             p.ssq = A.ssq_m;
             p.h_out = A.h;
             p.h_lo = A.h_lo;
             p.ld = F;
-            launch_gemm<EPI_SWIGLU>(s, pdl, G, h.tm_gu[l], A.tm_xg, A.tm_xg_lo, p);
+            launch_gemm<EPI_SWIGLU>(s, pdl, G, A.tm_xg, A.tm_xg, A.tm_xg_lo, p);
             break;
         }
         case K_DOWN: {
-            GemmParams p = gemm_base(h, d / 128, F / 64, A, rows_dev, decode);
+            GemmParams p = gemm_base(h, d / 128, F / 64, A, rows_dev);
+            p.w_blk = h.wb_down + l * h.ls_down;
             p.x_f32 = A.x_f32;
             p.xg_out = A.xg;
             p.xg_lo = A.xg_lo;
-            p.g_next = last ? h.final_norm : h.attn_norm[l + 1];
+            p.g_next = last ? h.final_norm : h.norm_attn + (size_t)(l + 1) * d;
             p.ssq_out = A.ssq_a;
             p.ld = d;
-            launch_gemm<EPI_RESID>(s, pdl, G, h.tm_down[l], A.tm_h, A.tm_h_lo, p);
-            break;
-        }
-        case K_LMHEAD: {
-            GemmParams p = gemm_base(h, m.vocab / 128, d / 64, A, rows_dev, true);
-            p.ssq = A.ssq_a;
-            p.y_f32 = logits_stage;
-            p.ld = m.vocab;
-            p.row_seed = c.row_seed;
-            p.arg_val = h.lm_val;
-            p.arg_idx = h.lm_idx;
-            launch_gemm<EPI_LMHEAD>(s, pdl, G, h.tm_lm, A.tm_xg, A.tm_xg_lo, p);
+            launch_gemm<EPI_RESID>(s, pdl, G, A.tm_h, A.tm_h, A.tm_h_lo, p);
             break;
         }
         default: throw SaraError(SARA_EINVAL, "unknown kernel id");
     }
 }
 
-// One forward pass over a row set: embedding, every layer, and (decode) lm_head with fused
-// sampling followed by the step bookkeeping.  Prefill stops after the last layer's K/V.
-// The first kernel of the sequence is launched without PDL.
-void enqueue_forward(sara_handle &h, cudaStream_t s, bool decode, bool pdl, float *logits_stage) {
+MegaParams mega_params(const sara_handle &h, float *logits) {
+    const sara_model_cfg &m = h.cfg;
+    MegaParams p{};
+    p.layers = m.layers;
+    p.d = m.d_model;
+    p.H = m.n_heads;
+    p.KVH = m.n_kv_heads;
+    p.hd = m.head_dim;
+    p.F = m.ffn;
+    p.V = m.vocab;
+    p.Gq = m.n_heads / m.n_kv_heads;
+    p.nqkv = (m.n_heads + 2 * m.n_kv_heads) * m.head_dim;
+    p.eps = m.rms_eps;
+    p.scale_log2 = (float)(1.4426950408889634 / std::sqrt((double)m.head_dim));
+    p.w_qkv = h.wb_qkv;
+    p.w_o = h.wb_o;
+    p.w_gu = h.wb_gu;
+    p.w_down = h.wb_down;
+    p.w_lm = h.wb_lm;
+    p.ls_qkv = h.ls_qkv;
+    p.ls_o = h.ls_o;
+    p.ls_gu = h.ls_gu;
+    p.ls_down = h.ls_down;
+    p.embed = h.embed;
+    p.attn_norm = h.norm_attn;
+    p.mlp_norm = h.norm_mlp;
+    p.final_norm = h.final_norm;
+    p.rope = h.rope;
+    p.kv = h.kv_seq;
+    p.kv_layer = h.kv_seq_layer;
+    p.kv_slot = h.kv_seq_slot;
+    p.kv_nblk = h.kv_nblk;
+    p.c = h.ptrs;
+    p.rows_cap = m.max_seqs;
+    p.rows_cap16 = h.rows_cap16;
+    p.x = h.dx;
+    p.xg_hi = h.xg_hi;
+    p.xg_lo = h.xg_lo;
+    p.att_hi = h.att_hi;
+    p.att_lo = h.att_lo;
+    p.h_hi = h.h_hi;
+    p.h_lo = h.h_lo;
+    p.ssqA = h.ssqA;
+    p.ssqM = h.ssqM;
+    p.accQ = h.accQ;
+    p.accO = h.accO;
+    p.accGU = h.accGU;
+    p.accD = h.accD;
+    p.part = h.attn_part;
+    p.att_cnt = h.attn_cnt;
+    p.logits = logits;
+    p.arg_val = h.lm_val;
+    p.arg_idx = h.lm_idx;
+    p.cnt = h.phase_cnt;
+    p.epoch = h.phase_cnt + h.n_phase_cnt;
+    return p;
+}
+
+// One decode step over the live rows: the persistent decode-step kernel (embedding, every
+// layer, lm_head with the Gumbel-max partials) followed by the sampling reduction and
+// bookkeeping kernel.
+void enqueue_decode_step(sara_handle &h, cudaStream_t s, float *logits_stage) {
+    launch_ex(s, false, true, dim3(h.sms), dim3(kMegaThreads), kMegaSmemBytes, decode_step_kernel,
+              mega_params(h, logits_stage));
+    launch(s, false, dim3(h.cfg.max_seqs), dim3(256), 0, sample_finish_kernel, h.ptrs);
+}
+
+// Prefill of the fresh prompts of a round: embedding, every layer up to the last layer's
+// K/V (the prompt's last hidden state is not needed: its last token is the rollouts' first
+// decode row).
+void enqueue_prefill(sara_handle &h, cudaStream_t s, bool pdl) {
     const sara_model_cfg &m = h.cfg;
     const StepPtrs &c = h.ptrs;
-    Acts &A = decode ? h.dec : h.pre;
-    const int *rows_dev = decode ? &h.vars->live : &h.vars->pre_rows;
+    Acts &A = h.pre;
     launch(s, false, dim3(A.rows_cap), dim3(128), 0, embed_kernel, (const uint16_t *)h.embed,
-           (const uint16_t *)h.attn_norm[0], rows_dev, decode ? (const int *)c.row_tok : (const int *)c.pre_tok,
-           m.d_model, A.rows_cap, m.vocab, A.x_f32, A.xg, A.xg_lo, A.ssq_a, &h.vars->err);
+           (const uint16_t *)h.norm_attn, (const int *)&h.vars->pre_rows, (const int *)c.pre_tok, m.d_model,
+           A.rows_cap, m.vocab, A.x_f32, A.xg, A.xg_lo, A.ssq_a, &h.vars->err);
     for (int l = 0; l < m.layers; ++l) {
-        enqueue_kernel(h, s, decode, K_QKV, l, pdl, nullptr);
-        if (!decode && l == m.layers - 1) break;  // the prompt's last hidden state is not needed
-        enqueue_kernel(h, s, decode, K_ATTN, l, pdl, nullptr);
-        enqueue_kernel(h, s, decode, K_OPROJ, l, pdl, nullptr);
-        enqueue_kernel(h, s, decode, K_GATEUP, l, pdl, nullptr);
-        enqueue_kernel(h, s, decode, K_DOWN, l, pdl, nullptr);
+        enqueue_prefill_kernel(h, s, K_QKV, l, pdl);
+        if (l == m.layers - 1) break;
+        enqueue_prefill_kernel(h, s, K_ATTN, l, pdl);
+        enqueue_prefill_kernel(h, s, K_OPROJ, l, pdl);
+        enqueue_prefill_kernel(h, s, K_GATEUP, l, pdl);
+        enqueue_prefill_kernel(h, s, K_DOWN, l, pdl);
     }
-    if (!decode) return;
-    enqueue_kernel(h, s, true, K_LMHEAD, m.layers - 1, pdl, logits_stage);
-    launch(s, pdl, dim3(A.rows_cap), dim3(256), 0, sample_finish_kernel, c);
 }
 
 void enqueue_kv_fanout(sara_handle &h, cudaStream_t s, bool pdl, const StepPtrs &c) {
     const sara_model_cfg &m = h.cfg;
     launch(s, pdl, dim3(h.sms * 8), dim3(256), 0, kv_fanout_kernel, (const uint16_t *)h.kv_pr, h.kv_seq, c, m.layers,
-           m.n_kv_heads, m.head_dim, h.cap_p, h.cap_s, m.max_active, m.max_seqs);
+           m.n_kv_heads, m.head_dim, h.cap_p, h.kv_seq_layer, h.kv_seq_slot, h.kv_nblk, m.max_active);
 }
 
 void enqueue_round_start(sara_handle &h, cudaStream_t s, bool pdl) {
-    enqueue_forward(h, s, false, pdl, nullptr);
+    enqueue_prefill(h, s, pdl);
     enqueue_kv_fanout(h, s, pdl, h.ptrs);
 }
 
@@ -375,7 +455,7 @@ void build_graph(sara_handle &h) {
         enqueue_round_start(h, h.cap_stream2, pdl);
         cudaGraph_t ib2;
         CK(cudaStreamEndCapture(h.cap_stream2, &ib2));
-        enqueue_forward(h, cs, true, pdl, nullptr);
+        enqueue_decode_step(h, cs, nullptr);
     }
     cudaGraph_t b2;
     CK(cudaStreamEndCapture(cs, &b2));
@@ -395,61 +475,80 @@ void run_host_loop(sara_handle &h) {
         if (v.done || v.err) break;
         if (!h.has_model) continue;
         if (v.round_steps == 0 && v.live > 0) enqueue_round_start(h, s, h.use_pdl);
-        enqueue_forward(h, s, true, h.use_pdl, nullptr);
+        enqueue_decode_step(h, s, nullptr);
     }
 }
 
 // ------------------------------------------------------------------------ weights
-void upload(const void *src, void *dst, size_t bytes, bool on_device, cudaStream_t s) {
-    CK(cudaMemcpyAsync(dst, src, bytes, on_device ? cudaMemcpyDeviceToDevice : cudaMemcpyHostToDevice, s));
+
+// Copy a row-major bf16 matrix [N][K] (host or device) into blocked 16 KB tiles at dst,
+// through the device staging buffer tmp.
+void block_matrix(cudaStream_t s, const void *src, bool on_device, uint16_t *tmp, uint8_t *dst, int N, int K) {
+    CK(cudaMemcpyAsync(tmp, src, (size_t)N * K * 2, on_device ? cudaMemcpyDeviceToDevice : cudaMemcpyHostToDevice, s));
+    launch(s, false, dim3(1024), dim3(256), 0, block_weights_kernel, (const uint16_t *)tmp, dst, N, K);
 }
 
 void load_weights(sara_handle &h, const sara_weights *w) {
     const sara_model_cfg &m = h.cfg;
-    const int d = m.d_model, H = m.n_heads, KVH = m.n_kv_heads, hd = m.head_dim, F = m.ffn, V = m.vocab;
+    const int d = m.d_model, H = m.n_heads, KVH = m.n_kv_heads, hd = m.head_dim, F = m.ffn, V = m.vocab, L = m.layers;
     const bool dev = w->on_device != 0;
     cudaStream_t s = h.stream;
     if (!w->embed || !w->lm_head || !w->final_norm || !w->attn_norm || !w->wq || !w->wk || !w->wv || !w->wo ||
         !w->mlp_norm || !w->wgate || !w->wup || !w->wdown)
         throw SaraError(SARA_EINVAL, "a weight pointer is NULL");
-    h.embed = h.mem.alloc<uint16_t>((size_t)V * d, false);
-    h.lm_head = h.mem.alloc<uint16_t>((size_t)V * d, false);
-    h.final_norm = h.mem.alloc<uint16_t>(d, false);
-    upload(w->embed, h.embed, (size_t)V * d * 2, dev, s);
-    upload(w->lm_head, h.lm_head, (size_t)V * d * 2, dev, s);
-    upload(w->final_norm, h.final_norm, (size_t)d * 2, dev, s);
-    const size_t qkv = (size_t)(H + 2 * KVH) * hd * d;
-    const cudaMemcpyKind kind = dev ? cudaMemcpyDeviceToDevice : cudaMemcpyHostToDevice;
-    for (int l = 0; l < m.layers; ++l) {
+    for (int l = 0; l < L; ++l)
         if (!w->attn_norm[l] || !w->wq[l] || !w->wk[l] || !w->wv[l] || !w->wo[l] || !w->mlp_norm[l] || !w->wgate[l] ||
             !w->wup[l] || !w->wdown[l])
             throw SaraError(SARA_EINVAL, "a per-layer weight pointer is NULL");
-        uint16_t *an = h.mem.alloc<uint16_t>(d, false), *mn = h.mem.alloc<uint16_t>(d, false);
-        upload(w->attn_norm[l], an, (size_t)d * 2, dev, s);
-        upload(w->mlp_norm[l], mn, (size_t)d * 2, dev, s);
-        // fused q|k|v rows
-        uint16_t *wqkv = h.mem.alloc<uint16_t>(qkv, false);
-        upload(w->wq[l], wqkv, (size_t)H * hd * d * 2, dev, s);
-        upload(w->wk[l], wqkv + (size_t)H * hd * d, (size_t)KVH * hd * d * 2, dev, s);
-        upload(w->wv[l], wqkv + (size_t)(H + KVH) * hd * d, (size_t)KVH * hd * d * 2, dev, s);
-        uint16_t *wo = h.mem.alloc<uint16_t>((size_t)d * H * hd, false);
-        upload(w->wo[l], wo, (size_t)d * H * hd * 2, dev, s);
-        // gate/up interleaved in blocks of 64 rows: [g 0..63, u 0..63, g 64..127, u 64..127, ...]
-        uint16_t *wgu = h.mem.alloc<uint16_t>((size_t)2 * F * d, false);
-        CK(cudaMemcpy2DAsync(wgu, (size_t)128 * d * 2, w->wgate[l], (size_t)64 * d * 2, (size_t)64 * d * 2, F / 64,
-                             kind, s));
-        CK(cudaMemcpy2DAsync(wgu + (size_t)64 * d, (size_t)128 * d * 2, w->wup[l], (size_t)64 * d * 2,
-                             (size_t)64 * d * 2, F / 64, kind, s));
-        uint16_t *wd = h.mem.alloc<uint16_t>((size_t)d * F, false);
-        upload(w->wdown[l], wd, (size_t)d * F * 2, dev, s);
-        h.attn_norm.push_back(an);
-        h.mlp_norm.push_back(mn);
-        h.w_qkv.push_back(wqkv);
-        h.w_o.push_back(wo);
-        h.w_gu.push_back(wgu);
-        h.w_down.push_back(wd);
+    const cudaMemcpyKind kind = dev ? cudaMemcpyDeviceToDevice : cudaMemcpyHostToDevice;
+    const int nqkv = (H + 2 * KVH) * hd;
+    h.ls_qkv = (int64_t)nqkv * d * 2;
+    h.ls_o = (int64_t)d * H * hd * 2;
+    h.ls_gu = (int64_t)2 * F * d * 2;
+    h.ls_down = (int64_t)d * F * 2;
+    h.embed = h.mem.alloc<uint16_t>((size_t)V * d, false);
+    h.final_norm = h.mem.alloc<uint16_t>(d, false);
+    h.norm_attn = h.mem.alloc<uint16_t>((size_t)L * d, false);
+    h.norm_mlp = h.mem.alloc<uint16_t>((size_t)L * d, false);
+    h.wb_qkv = h.mem.alloc<uint8_t>((size_t)L * h.ls_qkv, false);
+    h.wb_o = h.mem.alloc<uint8_t>((size_t)L * h.ls_o, false);
+    h.wb_gu = h.mem.alloc<uint8_t>((size_t)L * h.ls_gu, false);
+    h.wb_down = h.mem.alloc<uint8_t>((size_t)L * h.ls_down, false);
+    h.wb_lm = h.mem.alloc<uint8_t>((size_t)V * d * 2, false);
+    CK(cudaMemcpyAsync(h.embed, w->embed, (size_t)V * d * 2, kind, s));
+    CK(cudaMemcpyAsync(h.final_norm, w->final_norm, (size_t)d * 2, kind, s));
+    // staging buffer for one row-major matrix, freed when loading is done
+    const size_t stage = std::max({(size_t)V * d, (size_t)nqkv * d, (size_t)2 * F * d, (size_t)d * H * hd});
+    uint16_t *tmp = nullptr;
+    if (cudaMalloc(&tmp, stage * 2) != cudaSuccess) throw SaraError(SARA_ENOMEM, "cudaMalloc of the weight staging buffer failed");
+    try {
+        block_matrix(s, w->lm_head, dev, tmp, h.wb_lm, V, d);
+        for (int l = 0; l < L; ++l) {
+            CK(cudaMemcpyAsync(h.norm_attn + (size_t)l * d, w->attn_norm[l], (size_t)d * 2, kind, s));
+            CK(cudaMemcpyAsync(h.norm_mlp + (size_t)l * d, w->mlp_norm[l], (size_t)d * 2, kind, s));
+            // fused q|k|v rows
+            CK(cudaMemcpyAsync(tmp, w->wq[l], (size_t)H * hd * d * 2, kind, s));
+            CK(cudaMemcpyAsync(tmp + (size_t)H * hd * d, w->wk[l], (size_t)KVH * hd * d * 2, kind, s));
+            CK(cudaMemcpyAsync(tmp + (size_t)(H + KVH) * hd * d, w->wv[l], (size_t)KVH * hd * d * 2, kind, s));
+            launch(s, false, dim3(1024), dim3(256), 0, block_weights_kernel, (const uint16_t *)tmp,
+                   h.wb_qkv + l * h.ls_qkv, nqkv, d);
+            block_matrix(s, w->wo[l], dev, tmp, h.wb_o + l * h.ls_o, d, H * hd);
+            // gate/up interleaved in blocks of 64 rows: [g 0..63, u 0..63, g 64..127, u 64..127, ...]
+            CK(cudaMemcpy2DAsync(tmp, (size_t)128 * d * 2, w->wgate[l], (size_t)64 * d * 2, (size_t)64 * d * 2, F / 64,
+                                 kind, s));
+            CK(cudaMemcpy2DAsync(tmp + (size_t)64 * d, (size_t)128 * d * 2, w->wup[l], (size_t)64 * d * 2,
+                                 (size_t)64 * d * 2, F / 64, kind, s));
+            launch(s, false, dim3(1024), dim3(256), 0, block_weights_kernel, (const uint16_t *)tmp,
+                   h.wb_gu + l * h.ls_gu, 2 * F, d);
+            block_matrix(s, w->wdown[l], dev, tmp, h.wb_down + l * h.ls_down, d, F);
+        }
+        CK(cudaStreamSynchronize(s));
+    } catch (...) {
+        cudaStreamSynchronize(s);
+        cudaFree(tmp);
+        throw;
     }
-    CK(cudaStreamSynchronize(s));
+    CK(cudaFree(tmp));
 }
 
 void alloc_acts(sara_handle &h, Acts &A, int rows) {
@@ -468,24 +567,55 @@ void alloc_acts(sara_handle &h, Acts &A, int rows) {
     A.ssq_m = h.mem.alloc<float>((size_t)(d / 128) * rows);
 }
 
+// Decode-step buffers: residual stream, blocked hi/lo operands (rows padded to 16), the
+// fixed-point projection sums (zero between uses) and the phase counters.
+void alloc_decode(sara_handle &h) {
+    const sara_model_cfg &m = h.cfg;
+    const int S = m.max_seqs, d = m.d_model, Hhd = m.n_heads * m.head_dim, F = m.ffn;
+    const int nqkv = (m.n_heads + 2 * m.n_kv_heads) * m.head_dim;
+    h.rows_cap16 = (S + 15) & ~15;
+    const size_t R16 = h.rows_cap16;
+    h.dx = h.mem.alloc<float>((size_t)S * d);
+    h.xg_hi = h.mem.alloc<uint8_t>(R16 * d * 2);
+    h.xg_lo = h.mem.alloc<uint8_t>(R16 * d * 2);
+    h.att_hi = h.mem.alloc<uint8_t>(R16 * Hhd * 2);
+    h.att_lo = h.mem.alloc<uint8_t>(R16 * Hhd * 2);
+    h.h_hi = h.mem.alloc<uint8_t>(R16 * F * 2);
+    h.h_lo = h.mem.alloc<uint8_t>(R16 * F * 2);
+    h.ssqA = h.mem.alloc<float>((size_t)(d / 128) * S);
+    h.ssqM = h.mem.alloc<float>((size_t)(d / 128) * S);
+    h.accQ = h.mem.alloc<unsigned long long>((size_t)S * nqkv);
+    h.accO = h.mem.alloc<unsigned long long>((size_t)S * d);
+    h.accGU = h.mem.alloc<unsigned long long>((size_t)S * 2 * F);
+    h.accD = h.mem.alloc<unsigned long long>((size_t)S * d);
+    h.n_phase_cnt = 1 + kPhasesPerLayer * m.layers + 1;
+    h.phase_cnt = h.mem.alloc<unsigned long long>((size_t)h.n_phase_cnt + 1);
+}
+
+// Phase counters and the fixed-point sums back to zero (start of every call: a step that
+// failed part-way may have left them anywhere).
+void reset_decode_state(sara_handle &h, cudaStream_t s) {
+    const sara_model_cfg &m = h.cfg;
+    const size_t S = m.max_seqs, d = m.d_model;
+    const size_t nqkv = (size_t)(m.n_heads + 2 * m.n_kv_heads) * m.head_dim;
+    CK(cudaMemsetAsync(h.phase_cnt, 0, ((size_t)h.n_phase_cnt + 1) * 8, s));
+    CK(cudaMemsetAsync(h.accQ, 0, S * nqkv * 8, s));
+    CK(cudaMemsetAsync(h.accO, 0, S * d * 8, s));
+    CK(cudaMemsetAsync(h.accGU, 0, S * 2 * m.ffn * 8, s));
+    CK(cudaMemsetAsync(h.accD, 0, S * d * 8, s));
+    CK(cudaMemsetAsync(h.attn_cnt, 0, S * m.n_kv_heads * 4, s));
+}
+
 void make_tensor_maps(sara_handle &h) {
     const sara_model_cfg &m = h.cfg;
-    const int d = m.d_model, H = m.n_heads, KVH = m.n_kv_heads, hd = m.head_dim, F = m.ffn;
-    for (int l = 0; l < m.layers; ++l) {
-        h.tm_qkv.push_back(make_tmap_bf16(h.w_qkv[l], d, (H + 2 * KVH) * hd, kTileK, kTileM));
-        h.tm_o.push_back(make_tmap_bf16(h.w_o[l], H * hd, d, kTileK, kTileM));
-        h.tm_gu.push_back(make_tmap_bf16(h.w_gu[l], d, 2 * F, kTileK, kTileM));
-        h.tm_down.push_back(make_tmap_bf16(h.w_down[l], F, d, kTileK, kTileM));
-    }
-    h.tm_lm = make_tmap_bf16(h.lm_head, d, m.vocab, kTileK, kTileM);
-    for (Acts *A : {&h.dec, &h.pre}) {
-        A->tm_xg = make_tmap_bf16(A->xg, d, A->rows_cap, kTileK, kXBoxRows);
-        A->tm_xg_lo = make_tmap_bf16(A->xg_lo, d, A->rows_cap, kTileK, kXBoxRows);
-        A->tm_att = make_tmap_bf16(A->att, H * hd, A->rows_cap, kTileK, kXBoxRows);
-        A->tm_att_lo = make_tmap_bf16(A->att_lo, H * hd, A->rows_cap, kTileK, kXBoxRows);
-        A->tm_h = make_tmap_bf16(A->h, F, A->rows_cap, kTileK, kXBoxRows);
-        A->tm_h_lo = make_tmap_bf16(A->h_lo, F, A->rows_cap, kTileK, kXBoxRows);
-    }
+    const int d = m.d_model, H = m.n_heads, hd = m.head_dim, F = m.ffn;
+    Acts *A = &h.pre;
+    A->tm_xg = make_tmap_bf16(A->xg, d, A->rows_cap, kTileK, kXBoxRows);
+    A->tm_xg_lo = make_tmap_bf16(A->xg_lo, d, A->rows_cap, kTileK, kXBoxRows);
+    A->tm_att = make_tmap_bf16(A->att, H * hd, A->rows_cap, kTileK, kXBoxRows);
+    A->tm_att_lo = make_tmap_bf16(A->att_lo, H * hd, A->rows_cap, kTileK, kXBoxRows);
+    A->tm_h = make_tmap_bf16(A->h, F, A->rows_cap, kTileK, kXBoxRows);
+    A->tm_h_lo = make_tmap_bf16(A->h_lo, F, A->rows_cap, kTileK, kXBoxRows);
 }
 
 void validate_cfg(const sara_model_cfg &m) {
@@ -586,12 +716,15 @@ void create_impl(sara_handle &h, const sara_model_cfg *cfgp, const sara_weights 
         c.max_seqs = S;
         h.gen_tok = h.mem.alloc<int32_t>((size_t)P * K * m.max_gen_len, false);
         c.gen_tok = h.gen_tok;
-        // KV caches: rollout slots [layer][slot][2][kv][cap_s][hd], prompt slots [layer][pslot][2][kv][cap_p][hd]
-        h.kv_seq_slot = 2LL * KVH * h.cap_s * hd;
+        // KV caches: rollout slots [layer][slot][kv][128-position block] in the blocked decode
+        // layout (64 KB per block, zero-filled so padded head dims read as 0); prompt slots
+        // row-major [layer][pslot][2][kv][cap_p][hd]
+        h.kv_nblk = (h.cap_s + kKVPos - 1) / kKVPos;
+        h.kv_seq_slot = (int64_t)KVH * h.kv_nblk * kKVBlockBytes;
         h.kv_seq_layer = h.kv_seq_slot * S;
         h.kv_pr_slot = 2LL * KVH * h.cap_p * hd;
         h.kv_pr_layer = h.kv_pr_slot * Bc;
-        h.kv_seq = h.mem.alloc<uint16_t>((size_t)h.kv_seq_layer * m.layers);
+        h.kv_seq = h.mem.alloc<uint8_t>((size_t)h.kv_seq_layer * m.layers);
         h.kv_pr = h.mem.alloc<uint16_t>((size_t)h.kv_pr_layer * m.layers);
         // rotary table: angle = pos * theta^(-2i/hd), computed in double
         std::vector<float2> rope((size_t)h.cap_s * (hd / 2));
@@ -602,8 +735,8 @@ void create_impl(sara_handle &h, const sara_model_cfg *cfgp, const sara_weights 
             }
         h.rope = h.mem.alloc<float2>(rope.size(), false);
         CK(cudaMemcpy(h.rope, rope.data(), rope.size() * sizeof(float2), cudaMemcpyHostToDevice));
-        alloc_acts(h, h.dec, S);
         alloc_acts(h, h.pre, h.pre_cap);
+        alloc_decode(h);
         // GEMM stream-K workspace: one fixed-point tile sum per CTA + per-tile counters (zeroed)
         h.gemm_acc = h.mem.alloc<unsigned long long>((size_t)h.sms * kTileR * kTileM);
         const int max_m = std::max({(m.n_heads + 2 * KVH) * hd, d, 2 * m.ffn, m.vocab}) / 128;
@@ -686,6 +819,7 @@ void collect_impl(sara_handle &h, const sara_prompts *pr, int64_t N, int32_t k, 
         CK(cudaMemcpyAsync(h.p_len, pr->lengths, (size_t)P * k * 4, kin, s));
         if (h.has_model) CK(cudaMemcpyAsync(h.p_tok, pr->tokens, (size_t)P * Lp * 4, kin, s));
     }
+    if (h.has_model) reset_decode_state(h, s);
     launch(s, false, dim3(1), dim3(kCtlThreads), 0, ctl_init_kernel, h.ptrs);
     if (h.use_graph) CK(cudaGraphLaunch(h.exec, s));
     else run_host_loop(h);
@@ -764,11 +898,12 @@ void teacher_impl(sara_handle &h, int n, int Lp, const int32_t *prompts, int T, 
     const StepPtrs saved = h.ptrs;
     h.ptrs = c;
     try {
+        reset_decode_state(h, s);
         launch(s, false, dim3(1), dim3(kCtlThreads), 0, teacher_setup_kernel, c, n, (const int64_t *)h.uid_dev);
-        enqueue_forward(h, s, false, false, nullptr);
+        enqueue_prefill(h, s, false);
         enqueue_kv_fanout(h, s, false, c);
         for (int step = 0; step < T; ++step) {
-            enqueue_forward(h, s, true, false, h.logit_stage);
+            enqueue_decode_step(h, s, h.logit_stage);
             // rows stay in rollout order for all T steps (every rollout has length T)
             CK(cudaMemcpy2DAsync(logits + (size_t)step * m.vocab, (size_t)T * m.vocab * 4, h.logit_stage,
                                  (size_t)m.vocab * 4, (size_t)m.vocab * 4, n, kout, s));
@@ -786,13 +921,14 @@ void teacher_impl(sara_handle &h, int n, int Lp, const int32_t *prompts, int T, 
     if (v.live != 0 || v.exec_steps != T) throw SaraError(SARA_EDEVICE, "teacher forcing ran an unexpected number of steps");
 }
 
-// Profiling hook: `rows` live rollouts at context `ctx` (synthetic row state), `iters` launches
-// of one kernel of layer 0 (or of the whole eager decode step, kernel 0) timed with CUDA
-// events on the handle's stream after two warm-up launches.
+// Profiling hook: `rows` live rollouts at context `ctx` (synthetic row state), `iters`
+// launches of the whole decode step (kernel 0: decode-step kernel + sampling/bookkeeping,
+// positions advance) or of the decode-step kernel alone (kernel 1, positions fixed), timed
+// with CUDA events on the handle's stream around a captured graph after two warm-up launches.
 void profile_impl(sara_handle &h, int which, int rows, int ctx, int iters, double *ms) {
     const sara_model_cfg &m = h.cfg;
     if (!h.has_model) throw SaraError(SARA_EINVAL, "profiling needs a model");
-    if (which < 0 || which > K_LMHEAD) throw SaraError(SARA_EINVAL, "unknown kernel id");
+    if (which < 0 || which > 1) throw SaraError(SARA_EINVAL, "unknown kernel id (0 = decode step, 1 = decode-step kernel)");
     if (rows < 1 || rows > m.max_seqs || iters < 1 || !ms) throw SaraError(SARA_EINVAL, "rows / iters out of range");
     const int steps = which == 0 ? 2 * iters + 2 : 0;  // the whole step advances positions
     if (ctx < 2 || ctx + steps + 1 > h.cap_s || steps + 1 > m.max_gen_len) throw SaraError(SARA_EINVAL, "ctx out of range");
@@ -817,6 +953,7 @@ void profile_impl(sara_handle &h, int which, int rows, int ctx, int iters, doubl
     v.att_items = rows * nsplit;
     v.round_maxL = 1 << 30;
     const StepPtrs &c = h.ptrs;
+    reset_decode_state(h, s);
     CK(cudaMemcpyAsync(h.kc, &K, sizeof(K), cudaMemcpyHostToDevice, s));
     CK(cudaMemcpyAsync(h.vars, &v, sizeof(v), cudaMemcpyHostToDevice, s));
     CK(cudaMemcpyAsync(c.row_slot, slot.data(), rows * 4, cudaMemcpyHostToDevice, s));
@@ -830,14 +967,14 @@ void profile_impl(sara_handle &h, int which, int rows, int ctx, int iters, doubl
     CK(cudaMemcpyAsync(c.seq_gen, zero.data(), rows * 4, cudaMemcpyHostToDevice, s));
     CK(cudaMemcpyAsync(c.seq_len, len.data(), rows * 4, cudaMemcpyHostToDevice, s));
     CK(cudaMemcpyAsync(c.seq_uid, uid.data(), rows * 8, cudaMemcpyHostToDevice, s));
-#ifdef SARA_STAMPS
-    if (!h.stamps) h.stamps = h.mem.alloc<uint64_t>((size_t)h.sms * 16);
-    CK(cudaMemsetAsync(h.stamps, 0, (size_t)h.sms * 16 * 8, s));
-#endif
     CK(cudaStreamSynchronize(s));
     auto one = [&](cudaStream_t st) {
-        if (which == 0) enqueue_forward(h, st, true, h.use_pdl, nullptr);
-        else enqueue_kernel(h, st, true, which, 0, h.use_pdl, nullptr);
+        if (which == 0) {
+            enqueue_decode_step(h, st, nullptr);
+        } else {
+            launch_ex(st, false, true, dim3(h.sms), dim3(kMegaThreads), kMegaSmemBytes, decode_step_kernel,
+                      mega_params(h, nullptr));
+        }
     };
     one(s);
     one(s);
@@ -862,23 +999,6 @@ void profile_impl(sara_handle &h, int which, int rows, int ctx, int iters, doubl
     CK(cudaMemcpy(&v, h.vars, sizeof(v), cudaMemcpyDeviceToHost));
     check_step_error(v);
     *ms = (double)t / iters;
-#ifdef SARA_STAMPS
-    if (h.stamps && which != 0) {  // phase breakdown of the last launch, relative to the earliest entry
-        std::vector<uint64_t> st((size_t)h.sms * 16);
-        CK(cudaMemcpy(st.data(), h.stamps, st.size() * 8, cudaMemcpyDeviceToHost));
-        uint64_t t0 = ~0ull;
-        for (int c = 0; c < h.sms; ++c) t0 = std::min(t0, st[(size_t)c * 16]);
-        for (int i = 0; i < 16; ++i) {
-            std::vector<double> d;
-            for (int c = 0; c < h.sms; ++c)
-                if (st[(size_t)c * 16 + i]) d.push_back((double)(st[(size_t)c * 16 + i] - t0) * 1e-3);
-            std::sort(d.begin(), d.end());
-            if (!d.empty())
-                fprintf(stderr, "stamp %d: n=%zu min %.2f med %.2f max %.2f us\n", i, d.size(), d.front(), d[d.size() / 2],
-                        d.back());
-        }
-    }
-#endif
 }
 
 int guard(sara_handle *h, const std::function<void()> &fn) {

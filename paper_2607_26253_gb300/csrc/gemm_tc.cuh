@@ -51,6 +51,7 @@ struct GemmParams {
     const int *rows_dev;       // device count of valid rows (nullptr -> rows_fixed)
     int rows_fixed;
     int decode;                // 1: a single row tile, weights prefetched before the PDL wait
+    const uint8_t *w_blk;      // non-null: W stored as pre-swizzled 16 KB tiles [Nout/128][K/64] (bulk copies)
     int has_lo;                // 1: the activation's lo part (second tensor map) is multiplied too
     unsigned long long *ws_acc;  // [gridDim.x][kTileR * kTileM] fixed-point tile sums, zero between launches
     int *ws_cnt;               // [tiles] arrival counters, zero between launches
@@ -267,7 +268,7 @@ gemm_tc_kernel(const __grid_constant__ CUtensorMap tmW, const __grid_constant__ 
         S.epi_abort = 0;
         S.skip = (p.err != nullptr) && (*(volatile int *)p.err != 0);
         fence_mbar_init();
-        prefetch_tensormap(&tmW);
+        if (!p.w_blk) prefetch_tensormap(&tmW);
         prefetch_tensormap(&tmX);
         if (p.has_lo) prefetch_tensormap(&tmXlo);
     }
@@ -304,8 +305,12 @@ gemm_tc_kernel(const __grid_constant__ CUtensorMap tmW, const __grid_constant__ 
                     const int tile = (int)(u / kch), kc = (int)(u % kch);
                     const int m_tile = tile % m_tiles;
                     mbar_expect_tx(&S.full[i], (uint32_t)kWStageBytes);
-                    tma_load_2d(sW + i * kWStageBytes, &tmW, &S.full[i], kc * kTileK, m_tile * kTileM,
-                                l2_policy_evict_first());
+                    if (p.w_blk)
+                        bulk_load(sW + i * kWStageBytes, p.w_blk + ((int64_t)m_tile * kch + kc) * kWStageBytes,
+                                  kWStageBytes, &S.full[i], l2_policy_evict_first());
+                    else
+                        tma_load_2d(sW + i * kWStageBytes, &tmW, &S.full[i], kc * kTileK, m_tile * kTileM,
+                                    l2_policy_evict_first());
                 }
             }
             pdl_wait_prior_grids();
@@ -327,7 +332,12 @@ gemm_tc_kernel(const __grid_constant__ CUtensorMap tmW, const __grid_constant__ 
                 const uint32_t xbytes = (uint32_t)(nbox * kXBoxRows * kTileK * 2) * (p.has_lo ? 2u : 1u);
                 if (i >= n_pre) {
                     mbar_arrive_expect_tx(&S.full[s], (uint32_t)kWStageBytes + xbytes);
-                    tma_load_2d(sW + (size_t)s * kWStageBytes, &tmW, &S.full[s], kc * kTileK, m_tile * kTileM, pol_w);
+                    if (p.w_blk)
+                        bulk_load(sW + (size_t)s * kWStageBytes, p.w_blk + ((int64_t)m_tile * kch + kc) * kWStageBytes,
+                                  kWStageBytes, &S.full[s], pol_w);
+                    else
+                        tma_load_2d(sW + (size_t)s * kWStageBytes, &tmW, &S.full[s], kc * kTileK, m_tile * kTileM,
+                                    pol_w);
                 } else {
                     mbar_arrive_expect_tx(&S.full[s], xbytes);
                 }

@@ -1,6 +1,6 @@
-// Small kernels of the step graph: embedding gather (with the first RMSNorm's inputs),
-// prompt-KV fan-out into rollout slots, sampling reduction + per-step bookkeeping, and the
-// teacher-forcing round setup.
+// Small kernels of the step graph: embedding gather for the prefill rows (with the first
+// RMSNorm's inputs), sampling reduction + per-step bookkeeping, and the teacher-forcing
+// round setup.
 #pragma once
 #include "controller.cuh"
 #include "device_common.cuh"
@@ -39,34 +39,6 @@ static __global__ void __launch_bounds__(128) embed_kernel(const uint16_t *E, co
             if (threadIdx.x == 0) ssq[(int64_t)t * rows_cap + r] = red[0] + red[1] + red[2] + red[3];
             __syncthreads();
         }
-    }
-}
-
-// Copy every layer's prompt KV (positions < Lp - 1) from prompt slot seq_pslot[s] into
-// rollout slot s, for s < live (run once at a round start).
-static __global__ void kv_fanout_kernel(const uint16_t *pkv, uint16_t *kv, const StepPtrs c, int layers, int n_kv,
-                                        int hd, int cap_p, int cap_s, int max_active, int max_seqs) {
-    pdl_wait_prior_grids();
-    pdl_allow_dependents();
-    const int live = c.v->live;
-    const int Lpre = c.kc->Lp - 1;
-    const int vec_per_row = hd / 8;  // 16-byte vectors per position
-    const int64_t per_plane = (int64_t)Lpre * vec_per_row;
-    const int64_t per_slot = 2LL * n_kv * per_plane;
-    const int64_t total = (int64_t)layers * live * per_slot;
-    for (int64_t e = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; e < total; e += (int64_t)gridDim.x * blockDim.x) {
-        const int64_t l = e / ((int64_t)live * per_slot);
-        int64_t rem = e - l * live * per_slot;
-        const int s = (int)(rem / per_slot);
-        rem -= (int64_t)s * per_slot;
-        const int plane = (int)(rem / per_plane);  // 0 .. 2*n_kv-1
-        rem -= (int64_t)plane * per_plane;
-        const int pos = (int)(rem / vec_per_row), v = (int)(rem % vec_per_row);
-        const int ps = c.seq_pslot[s];
-        const uint4 *src =
-            reinterpret_cast<const uint4 *>(pkv + (((l * max_active + ps) * 2LL * n_kv + plane) * cap_p + pos) * hd) + v;
-        uint4 *dst = reinterpret_cast<uint4 *>(kv + (((l * max_seqs + s) * 2LL * n_kv + plane) * cap_s + pos) * hd) + v;
-        *dst = *src;
     }
 }
 

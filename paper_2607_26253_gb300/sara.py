@@ -238,7 +238,8 @@ class Handle:
         return StepOutput(status, n, s, rnd, toks, counters, float(res.device_ms))
 
     def profile(self, kernel: int, rows: int, ctx: int, iters: int = 20) -> float:
-        """Milliseconds per launch of one decode kernel (see sara_profile in include/sara.h)."""
+        """Milliseconds per launch of the decode step (kernel 0) or of the decode-step kernel
+        alone (kernel 1); see sara_profile in include/sara.h."""
         ms = ctypes.c_double()
         _check(load().sara_profile(self._h, kernel, rows, ctx, iters, ctypes.byref(ms)), self._h)
         return ms.value
