@@ -1,37 +1,49 @@
-// One decode step of the policy (embedding -> every layer -> lm_head with fused Gumbel-max
-// partials) as a single persistent, cooperative kernel: one CTA per SM, phases separated
+// One decode step of the policy (embedding -> every layer -> lm_head logits) as a single
+// persistent, cooperative kernel: one CTA per SM, phases separated
 // by release/acquire arrival counters in global memory instead of kernel boundaries.
 //
 // Why: at decode batch sizes the per-layer work is a few MB of weights per projection, so
 // a kernel per projection spends most of its time starting, filling its pipeline and
 // draining.  Here the weight stream never stops: the producer warp walks the whole step's
 // weight tiles (and the attention phase's KV blocks, which do not depend on this step's
-// activations) ahead of the consumers through an 8-slot shared-memory ring, across phase
-// boundaries.  Only the small activation operands wait for the previous phase.
+// activations) ahead of the consumers through a ring of 32 KB shared-memory slots, across
+// phase boundaries.  Only the small activation operands wait for the previous phase.
+//
+// GEMM orientation: the activation rows are the MMA's M (128, rows beyond the live count
+// are don't-care) and 256 weight rows its N, so one tcgen05.mma (K = 16) consumes 8 KB of
+// weights.  The instruction's cost hardly depends on N, so this keeps the tensor pipe off
+// the critical path at the HBM rate even with the activation split into a bf16 hi/lo pair
+// (two MMAs per k-step, ~16 mantissa bits of the activation).
+//
+// Split-K: a phase's (tile, k-chunk) units are cut into equal contiguous ranges over its
+// CTAs; each CTA stores its fp32 partial tile with plain stores and the consuming phase
+// sums a tile's partials in CTA order (deterministic, no atomics).
 //
 // Warp roles (352 threads, 11 warps):
-//   warp 0   W producer: 16 KB bulk copies of pre-swizzled weight tiles and KV blocks
+//   warp 0   W producer: bulk copies of pre-swizzled weight tiles and KV blocks
 //   warp 1   tcgen05 issuer and tensor-memory owner
 //   warp 2   X producer: activation chunks, after the phase they come from has completed
-//   warps 3..10  compute: GEMM epilogues (fixed-point folds), attention softmax / merge,
-//                residual + RMSNorm + SwiGLU finalisation, embedding, sampling partials
+//   warps 3..10  compute: GEMM epilogues, attention softmax / merge, residual + RMSNorm +
+//                SwiGLU finalisation, embedding, logits
 //
 // Phases of layer l (counter index 1 + 8l + k):
-//   0 QKV   x_g W_qkv^T          -> accQ (64-bit fixed point, atomic fold over k-splits)
-//   1 ATT   q, k, v = RMSNorm scale + RoPE of accQ; new k, v appended to the KV cache;
-//           softmax(q K^T) V on the tensor cores per 128-position split; split merge
-//   2 O     att W_o^T            -> accO
-//   3 FIN_O x += accO; x_g = x * g_mlp (bf16 hi/lo, blocked); per-row sum of squares
-//   4 GU    x_g W_gu^T           -> accGU (gate / up interleaved in 64-row blocks)
+//   0 QKV   x_g W_qkv^T -> partials        (a subset of the CTAs: few tiles)
+//   1 ATT   q, k, v = RMSNorm scale + RoPE of the summed partials; new k, v appended to
+//           the KV cache; softmax(q K^T) V on the tensor cores per 128-position split;
+//           the last split of a row to finish merges them
+//   2 O     att W_o^T -> partials           (a subset of the CTAs)
+//   3 FIN_O x += sum; x_g = x * g_mlp (bf16 hi/lo, blocked); per-row sum of squares
+//   4 GU    x_g W_gu^T -> partials          (gate / up interleaved in 64-row blocks)
 //   5 FIN_GU h = silu(r g) * (r u), r = 1/rms(x)  (bf16 hi/lo, blocked)
-//   6 DOWN  h W_down^T           -> accD
-//   7 FIN_D x += accD; x_g = x * g_next; sum of squares
-// then lm_head over whole 128-token tiles with the Gumbel-max partial argmax per tile.
+//   6 DOWN  h W_down^T -> partials
+//   7 FIN_D x += sum; x_g = x * g_next; sum of squares
+// then lm_head over whole 256-token tiles, writing the logits of the live rows.
 //
-// Layouts (all chosen so that one bulk copy lands an MMA operand in shared memory in the
+// Layouts (all chosen so that bulk copies land MMA operands in shared memory in the
 // 128-byte-swizzled K-major form the tensor core reads):
-//   weights       [N/128][K/64] blocks of 128 rows x 64 elements (16 KB), swizzled
-//   activations   [K/64][rows16][64] bf16 (hi and lo planes), swizzled per 8-row atom
+//   weights       tiles of 256 rows (the last may have 128): [N/256][K/64][rows][64],
+//                 16-byte granule j of row r at granule j ^ (r % 8)
+//   activations   [K/64][rows16][64] bf16 (hi and lo planes), same swizzle
 //   KV cache      per (layer, slot, kv head, 128-position block): K as [d/64][128 pos][64 d]
 //                 and V transposed as [pos/64][128 d][64 pos], fp16, head dim padded to 128
 #pragma once
@@ -42,19 +54,19 @@ namespace sara {
 
 constexpr int kMegaThreads = 352;
 constexpr int kMegaCThreads = 256;  // compute warps 3..10
-constexpr int kWSlots = 8;
-constexpr int kSlotBytes = 16384;
+constexpr int kWSlots = 4;
+constexpr int kSlotBytes = 32768;
 constexpr int kXRingBytes = 65536;
 constexpr int kMaxXStages = 8;
+constexpr int kTileN = 256;           // weight rows (output features) per GEMM tile
 constexpr int kKVPos = 128;           // positions per KV block and per attention split
 constexpr int kKVBlockBytes = 65536;  // K 2 x 16 KB + V^T 2 x 16 KB
 constexpr int kMegaMaxSplits = 96;
 constexpr int kPhasesPerLayer = 8;
+constexpr int kSmallPhaseUnits = 4;   // QKV / O: units per participating CTA (the ring's depth)
 constexpr uint32_t kTmemCols = 512;
 constexpr uint32_t kTmemS = 256;  // attention scores, 2 buffers x 16 columns
 constexpr uint32_t kTmemO = 288;  // attention output, 2 buffers x 16 columns
-constexpr float kFix = 4294967296.0f;                 // 2^32
-constexpr float kUnfix = 2.3283064365386963e-10f;     // 2^-32
 
 struct MegaParams {
     int layers, d, H, KVH, hd, F, V, Gq, nqkv;
@@ -70,20 +82,46 @@ struct MegaParams {
     int kv_nblk;                                    // 128-position blocks per (slot, kv head)
     StepPtrs c;
     int rows_cap, rows_cap16;
+    int gp_qkv, gp_o;                               // CTAs taking part in the QKV / O projections
     float *x;                                       // [rows_cap][d] residual stream
     uint8_t *xg_hi, *xg_lo;                         // blocked [d/64][rows_cap16][64]
     uint8_t *att_hi, *att_lo;                       // blocked [H*hd/64][rows_cap16][64]
     uint8_t *h_hi, *h_lo;                           // blocked [F/64][rows_cap16][64]
     float *ssqA, *ssqM;                             // [d/128][rows_cap] partial sums of x^2
-    unsigned long long *accQ, *accO, *accGU, *accD; // [rows_cap][N] fixed point, zero between uses
-    float *part;                                    // [items][KVH][Gq][hd + 2] split partials
+    float *gpart;                                   // [segments][rows_cap][256] GEMM partial tiles
+    float *part;                                    // [items][KVH][Gq][hd + 2] attention split partials
     int *att_cnt;                                   // [rows_cap][KVH] split arrival counters
-    float *logits;                                  // optional [rows][V] fp32
-    float *arg_val;                                 // [rows][V/128] partial max
-    int *arg_idx;                                   //   and its token
+    float *logits;                                  // [rows_cap][V] fp32 (read by the sampling kernel)
     unsigned long long *cnt;                        // phase arrival counters (monotonic)
     unsigned long long *epoch;                      // launches completed since the reset
+    uint64_t *stamps;                               // profiling builds: [cta][phase + 1][4] timestamps
+    int n_stamp_ph;
 };
+
+// Profiling builds (-DSARA_STAMPS): per CTA and phase, when the compute warps arrived (0),
+// when the phase's input dependency was observed (1), when the W producer finished issuing
+// the phase's copies (2) and when the MMA issuer committed the phase's last MMA (3).
+#ifdef SARA_STAMPS
+#define MEGA_STAMP(ph, kind)                                                                              \
+    do {                                                                                                  \
+        if (p.stamps) p.stamps[((size_t)blockIdx.x * p.n_stamp_ph + (ph)) * 4 + (kind)] = globaltimer_ns(); \
+    } while (0)
+// Detail stamps of the attention and first finalize phases of one layer (layer 2), first
+// unit of each CTA: the last four phase slots of the same array (the fifth-last holds the
+// kernel start).
+#define MEGA_DETAIL(i)                                                                                          \
+    do {                                                                                                        \
+        if (p.stamps) p.stamps[((size_t)blockIdx.x * p.n_stamp_ph + p.n_stamp_ph - 4 + ((i) >> 2)) * 4 + ((i) & 3)] = \
+                          globaltimer_ns();                                                                       \
+    } while (0)
+#else
+#define MEGA_STAMP(ph, kind) \
+    do {                     \
+    } while (0)
+#define MEGA_DETAIL(i) \
+    do {               \
+    } while (0)
+#endif
 
 struct MegaSmem {
     uint64_t wfull[kWSlots], wempty[kWSlots];
@@ -97,13 +135,10 @@ struct MegaSmem {
     int last_flag;
     int rows, rows16, nx, n_items;
     float rstd[128];
-    unsigned long long seed[128];
     float att_m[2][8], att_l[2][8];
-    float red[4][8];
+    float red[4][8], red2[4][8];
     float mw[8][kMegaMaxSplits];
     float ml[8];
-    float lm_v[2][4][32];
-    int lm_i[2][4][32];
 };
 
 constexpr size_t kMegaSmemBytes =
@@ -122,6 +157,11 @@ __host__ __device__ __forceinline__ int kv_k_off(int pp, int d) {
 __host__ __device__ __forceinline__ int kv_v_off(int pp, int d) {
     const int c = pp & 63;
     return 32768 + (pp >> 6) * 16384 + d * 128 + ((((c >> 3) ^ (d & 7)) << 4) | ((c & 7) << 1));
+}
+// Byte offset of the (tile t, k-chunk kc) block of a blocked weight matrix [N][K].
+__host__ __device__ __forceinline__ int64_t wblk_off(int N, int K, int t, int kc) {
+    const int rows = (N - t * kTileN) < kTileN ? (N - t * kTileN) : kTileN;
+    return (int64_t)t * kTileN * K * 2 + (int64_t)kc * rows * 128;
 }
 
 // ------------------------------------------------------------------------------ waits
@@ -169,53 +209,67 @@ __device__ __forceinline__ bool spin_counter(const unsigned long long *cnt, unsi
 // ------------------------------------------------------------------------------ phases
 struct GemmPh {
     const uint8_t *w;
-    int m_tiles, kch;
+    int N, K, kch, T, Gp;
     const uint8_t *xhi, *xlo;
-    unsigned long long *acc;
-    int ld;
+    bool whole;  // whole tiles per CTA (lm_head: the argmax of a tile is finished in one CTA)
 };
 
 // GEMM phase k (0 QKV, 2 O, 4 GU, 6 DOWN) of layer l; l == layers: lm_head.
 __device__ __forceinline__ GemmPh gemm_phase(const MegaParams &p, int l, int k) {
     GemmPh g;
+    g.whole = false;
+    g.Gp = gridDim.x;
     if (l == p.layers) {
-        g.w = p.w_lm; g.m_tiles = p.V / 128; g.kch = p.d / 64; g.xhi = p.xg_hi; g.xlo = p.xg_lo; g.acc = nullptr;
-        g.ld = p.V;
-        return g;
+        g.w = p.w_lm; g.N = p.V; g.K = p.d; g.xhi = p.xg_hi; g.xlo = p.xg_lo; g.whole = true;
+    } else if (k == 0) {
+        g.w = p.w_qkv + l * p.ls_qkv; g.N = p.nqkv; g.K = p.d; g.xhi = p.xg_hi; g.xlo = p.xg_lo; g.Gp = p.gp_qkv;
+    } else if (k == 2) {
+        g.w = p.w_o + l * p.ls_o; g.N = p.d; g.K = p.H * p.hd; g.xhi = p.att_hi; g.xlo = p.att_lo; g.Gp = p.gp_o;
+    } else if (k == 4) {
+        g.w = p.w_gu + l * p.ls_gu; g.N = 2 * p.F; g.K = p.d; g.xhi = p.xg_hi; g.xlo = p.xg_lo;
+    } else {
+        g.w = p.w_down + l * p.ls_down; g.N = p.d; g.K = p.F; g.xhi = p.h_hi; g.xlo = p.h_lo;
     }
-    switch (k) {
-        case 0:
-            g.w = p.w_qkv + l * p.ls_qkv; g.m_tiles = p.nqkv / 128; g.kch = p.d / 64;
-            g.xhi = p.xg_hi; g.xlo = p.xg_lo; g.acc = p.accQ; g.ld = p.nqkv;
-            break;
-        case 2:
-            g.w = p.w_o + l * p.ls_o; g.m_tiles = p.d / 128; g.kch = p.H * p.hd / 64;
-            g.xhi = p.att_hi; g.xlo = p.att_lo; g.acc = p.accO; g.ld = p.d;
-            break;
-        case 4:
-            g.w = p.w_gu + l * p.ls_gu; g.m_tiles = 2 * p.F / 128; g.kch = p.d / 64;
-            g.xhi = p.xg_hi; g.xlo = p.xg_lo; g.acc = p.accGU; g.ld = 2 * p.F;
-            break;
-        default:
-            g.w = p.w_down + l * p.ls_down; g.m_tiles = p.d / 128; g.kch = p.F / 64;
-            g.xhi = p.h_hi; g.xlo = p.h_lo; g.acc = p.accD; g.ld = p.d;
-            break;
-    }
+    g.kch = g.K / 64;
+    g.T = (g.N + kTileN - 1) / kTileN;
+    // at most one CTA per unit (tile for lm_head), so every participating CTA holds a
+    // non-empty range and the CTAs between a tile's first and last owner all contributed
+    g.Gp = min(g.Gp, g.whole ? g.T : g.T * g.kch);
     return g;
 }
+__device__ __forceinline__ int tile_rows(const GemmPh &g, int t) { return min(kTileN, g.N - kTileN * t); }
 
-// This CTA's (tile, k-chunk) units: an equal share of the whole GEMM, or (lm_head) of
-// whole tiles so that every tile's argmax is finished by one CTA.
-__device__ __forceinline__ void gemm_range(const GemmPh &g, bool whole, int64_t &u0, int64_t &u1) {
-    const int G = gridDim.x, c = blockIdx.x;
-    if (whole) {
-        u0 = (int64_t)c * g.m_tiles / G * g.kch;
-        u1 = (int64_t)(c + 1) * g.m_tiles / G * g.kch;
-    } else {
-        const int64_t U = (int64_t)g.m_tiles * g.kch;
-        u0 = (int64_t)c * U / G;
-        u1 = (int64_t)(c + 1) * U / G;
+// This CTA's (tile, k-chunk) units: an equal contiguous share over the phase's CTAs, or
+// (lm_head) a share of whole tiles.
+// (Unit counts stay below 2^31 / SMs for every supported shape: 32-bit products suffice.)
+__device__ __forceinline__ void gemm_range(const GemmPh &g, int64_t &u0, int64_t &u1) {
+    const int c = blockIdx.x;
+    if (c >= g.Gp) {
+        u0 = u1 = 0;
+        return;
     }
+    if (g.whole) {
+        u0 = (int64_t)(c * g.T / g.Gp) * g.kch;
+        u1 = (int64_t)((c + 1) * g.T / g.Gp) * g.kch;
+    } else {
+        const int U = g.T * g.kch;
+        u0 = c * U / g.Gp;
+        u1 = (c + 1) * U / g.Gp;
+    }
+}
+// CTA owning unit u when U units are cut into Gp equal contiguous ranges.
+__device__ __forceinline__ int unit_owner(int u, int U, int Gp) {
+    int c = u * Gp / U;
+    while (c + 1 < Gp && (c + 1) * U / Gp <= u) ++c;
+    while (c > 0 && c * U / Gp > u) --c;
+    return c;
+}
+// First and last CTA holding a partial of tile t.  CTA c's partial of tile t is segment
+// c + t of the partial buffer (distinct for every (c, t) of a phase: ranges are ordered).
+__device__ __forceinline__ void tile_ctas(const GemmPh &g, int t, int &ca, int &cb) {
+    const int U = g.T * g.kch;
+    ca = unit_owner(t * g.kch, U, g.Gp);
+    cb = unit_owner((t + 1) * g.kch - 1, U, g.Gp);
 }
 
 struct AttUnit {
@@ -238,18 +292,12 @@ __device__ __forceinline__ AttUnit att_unit(const MegaParams &p, int64_t a) {
     return u;
 }
 __device__ __forceinline__ void att_range(const MegaParams &p, int n_items, int64_t &a0, int64_t &a1) {
-    const int64_t NU = (int64_t)n_items * p.KVH;
-    a0 = (int64_t)blockIdx.x * NU / gridDim.x;
-    a1 = (int64_t)(blockIdx.x + 1) * NU / gridDim.x;
+    const int NU = n_items * p.KVH;
+    a0 = (int)blockIdx.x * NU / (int)gridDim.x;
+    a1 = ((int)blockIdx.x + 1) * NU / (int)gridDim.x;
 }
 __device__ __forceinline__ uint8_t *kv_block(const MegaParams &p, int l, const AttUnit &u) {
     return p.kv + l * p.kv_layer + (int64_t)u.slot * p.kv_slot + ((int64_t)u.kvh * p.kv_nblk + u.sp) * kKVBlockBytes;
-}
-// Bytes of the four ring slots of one attention unit: K (d < 64), K (d >= 64), V^T (positions
-// < 64), V^T (positions >= 64).  Zero = slot not needed (arrive without data).
-__device__ __forceinline__ uint32_t att_slot_bytes(const MegaParams &p, const AttUnit &u, int q) {
-    if (q < 2) return (q * 64 < p.hd) ? (uint32_t)(((u.n + 7) & ~7) * 128) : 0u;
-    return (q == 2 || u.n > 64) ? (uint32_t)(p.hd * 128) : 0u;
 }
 
 // ------------------------------------------------------------------------------ W producer
@@ -259,44 +307,47 @@ __device__ __forceinline__ void mega_w_producer(const MegaParams &p, MegaSmem &S
     const uint64_t pol = l2_policy_evict_first();
     uint32_t wi = 0;
     bool ok = true;
-    auto slot = [&](uint32_t i) -> int { return (int)(i % kWSlots); };
     auto acquire = [&](uint32_t i) -> bool {
-        return i < kWSlots || mwait(&S.wempty[slot(i)], ((i / kWSlots) & 1) ^ 1, err, ab);
-    };
-    auto gemm = [&](const GemmPh &g, int64_t u0, int64_t u1) {
-        for (int64_t u = u0; u < u1 && ok; ++u, ++wi) {
-            if (!acquire(wi)) { ok = false; break; }
-            const int s = slot(wi);
-            mbar_arrive_expect_tx(&S.wfull[s], kSlotBytes);
-            bulk_load(sW + (size_t)s * kSlotBytes, g.w + u * kSlotBytes, kSlotBytes, &S.wfull[s], pol);
-        }
+        return i < kWSlots || mwait(&S.wempty[i % kWSlots], ((i / kWSlots) & 1) ^ 1, err, ab);
     };
     for (int l = 0; l <= p.layers && ok; ++l) {
         for (int k = 0; k < kPhasesPerLayer && ok; k += 2) {
             if (l == p.layers && k > 0) break;
             const GemmPh g = gemm_phase(p, l, k);
             int64_t u0, u1;
-            gemm_range(g, l == p.layers, u0, u1);
-            gemm(g, u0, u1);
-            if (k == 0 && l < p.layers) {
-                // the attention phase's KV blocks follow the QKV weights in ring order
+            gemm_range(g, u0, u1);
+            for (int64_t u = u0; u < u1; ++u, ++wi) {
+                if (!acquire(wi)) { ok = false; break; }
+                const int s = (int)(wi % kWSlots);
+                const int t = (int)(u / g.kch), kc = (int)(u - (int64_t)t * g.kch);
+                const uint32_t bytes = (uint32_t)tile_rows(g, t) * 128;
+                mbar_arrive_expect_tx(&S.wfull[s], bytes);
+                bulk_load(sW + (size_t)s * kSlotBytes, g.w + wblk_off(g.N, g.K, t, kc), bytes, &S.wfull[s], pol);
+            }
+            MEGA_STAMP(1 + kPhasesPerLayer * l + k, 2);
+            if (k == 0 && l < p.layers && ok) {
+                // the attention phase's KV blocks follow the QKV weights in ring order:
+                // slot 1 = K (d < 64 | d >= 64), slot 2 = V^T (positions < 64 | >= 64)
                 int64_t a0, a1;
                 att_range(p, S.n_items, a0, a1);
                 for (int64_t a = a0; a < a1 && ok; ++a) {
                     const AttUnit u = att_unit(p, a);
                     const uint8_t *blk = kv_block(p, l, u);
-                    for (int q = 0; q < 4; ++q, ++wi) {
-                        if (!acquire(wi)) { ok = false; break; }
-                        const int s = slot(wi);
-                        const uint32_t bytes = att_slot_bytes(p, u, q);
-                        if (bytes) {
-                            mbar_arrive_expect_tx(&S.wfull[s], bytes);
-                            bulk_load(sW + (size_t)s * kSlotBytes, blk + q * 16384, bytes, &S.wfull[s], pol);
-                        } else {
-                            mbar_arrive(&S.wfull[s]);
-                        }
-                    }
+                    const uint32_t kb = (uint32_t)(((u.n + 7) & ~7) * 128), vb = (uint32_t)(p.hd * 128);
+                    if (!acquire(wi)) { ok = false; break; }
+                    int s = (int)(wi % kWSlots);
+                    mbar_arrive_expect_tx(&S.wfull[s], p.hd > 64 ? 2 * kb : kb);
+                    bulk_load(sW + (size_t)s * kSlotBytes, blk, kb, &S.wfull[s], pol);
+                    if (p.hd > 64) bulk_load(sW + (size_t)s * kSlotBytes + 16384, blk + 16384, kb, &S.wfull[s], pol);
+                    ++wi;
+                    if (!acquire(wi)) { ok = false; break; }
+                    s = (int)(wi % kWSlots);
+                    mbar_arrive_expect_tx(&S.wfull[s], u.n > 64 ? 2 * vb : vb);
+                    bulk_load(sW + (size_t)s * kSlotBytes, blk + 32768, vb, &S.wfull[s], pol);
+                    if (u.n > 64) bulk_load(sW + (size_t)s * kSlotBytes + 16384, blk + 49152, vb, &S.wfull[s], pol);
+                    ++wi;
                 }
+                MEGA_STAMP(2 + kPhasesPerLayer * l, 2);
             }
         }
     }
@@ -323,11 +374,12 @@ __device__ __forceinline__ void mega_x_producer(const MegaParams &p, MegaSmem &S
             if (l == p.layers && k > 0) break;
             const GemmPh g = gemm_phase(p, l, k);
             int64_t u0, u1;
-            gemm_range(g, l == p.layers, u0, u1);
+            gemm_range(g, u0, u1);
             if (u0 >= u1) continue;
             // the phase this operand comes from: FIN_D of l-1 / embedding, ATT, FIN_O, FIN_GU
-            const int dep = (l == p.layers) ? kPhasesPerLayer * l : (k == 0 ? kPhasesPerLayer * l : 1 + 8 * l + k - 1);
+            const int dep = (l == p.layers || k == 0) ? kPhasesPerLayer * l : 1 + kPhasesPerLayer * l + k - 1;
             if (!spin_counter(&p.cnt[dep], S.target, err, ab)) { ok = false; break; }
+            MEGA_STAMP(1 + kPhasesPerLayer * l + k, 1);
             fence_proxy_async_global();
             for (int64_t u = u0; u < u1; ++u, ++xi) {
                 const int s = (int)(xi % NX);
@@ -355,21 +407,22 @@ __device__ __forceinline__ void mega_mma(const MegaParams &p, MegaSmem &S, uint8
     int *err = &p.c.v->err;
     const int NX = S.nx, R16 = S.rows16;
     const uint32_t plane = (uint32_t)R16 * 128, stage = 2 * plane;
-    const uint32_t idg = idesc_bf16_f32(128, (uint32_t)R16);
     const uint32_t ida = idesc_f16_f32(128, 16);
     uint32_t wi = 0, xi = 0;
-    int seg = 0, gi = 0;
+    int gi = 0, use0 = 0, use1 = 0, lmseg = 0;  // accumulator buffer uses
     bool ok = true;
     auto wslot = [&](uint32_t i) -> uint32_t { return smem_u32(sW + (size_t)(i % kWSlots) * kSlotBytes); };
     auto wwait = [&](uint32_t i) -> bool { return mwait(&S.wfull[i % kWSlots], (i / kWSlots) & 1, err, ab); };
     auto gemm = [&](const GemmPh &g, int64_t u0, int64_t u1) {
         for (int64_t u = u0; u < u1 && ok;) {
-            const int tile = (int)(u / g.kch);
-            const int64_t e = min(u1, (int64_t)(tile + 1) * g.kch);
-            const int a = seg & 1;
-            if (seg >= 2 && !mwait(&S.acc_empty[a], ((seg >> 1) - 1) & 1, err, ab)) { ok = false; break; }
+            const int t = (int)(u / g.kch);
+            const int64_t e = min(u1, (int64_t)(t + 1) * g.kch);
+            const int a = g.whole ? (lmseg & 1) : 0;  // lm_head alternates two accumulators
+            const int use_a = a ? use1 : use0;
+            if (use_a >= 1 && !mwait(&S.acc_empty[a], (use_a - 1) & 1, err, ab)) { ok = false; break; }
             tc_fence_after();
-            const uint32_t d = tmem + (uint32_t)(a * 128);
+            const uint32_t d = tmem + (uint32_t)(a * kTileN);
+            const uint32_t idg = idesc_bf16_f32(128, (uint32_t)tile_rows(g, t));
             bool first = true;
             for (; u < e; ++u, ++wi, ++xi) {
                 const int xs = (int)(xi % NX);
@@ -378,9 +431,9 @@ __device__ __forceinline__ void mega_mma(const MegaParams &p, MegaSmem &S, uint8
                 const uint32_t aw = wslot(wi), ax = smem_u32(sX + (size_t)xs * stage);
 #pragma unroll
                 for (int kk = 0; kk < 4; ++kk) {
-                    const uint64_t ad = sdesc_kmajor_sw128(aw + kk * 32);
-                    tc_mma_bf16(d, ad, sdesc_kmajor_sw128(ax + kk * 32), idg, (first && kk == 0) ? 0u : 1u);
-                    tc_mma_bf16(d, ad, sdesc_kmajor_sw128(ax + plane + kk * 32), idg, 1u);
+                    const uint64_t bd = sdesc_kmajor_sw128(aw + kk * 32);
+                    tc_mma_bf16(d, sdesc_kmajor_sw128(ax + kk * 32), bd, idg, (first && kk == 0) ? 0u : 1u);
+                    tc_mma_bf16(d, sdesc_kmajor_sw128(ax + plane + kk * 32), bd, idg, 1u);
                 }
                 first = false;
                 tc_commit(&S.wempty[wi % kWSlots]);
@@ -388,7 +441,8 @@ __device__ __forceinline__ void mega_mma(const MegaParams &p, MegaSmem &S, uint8
             }
             if (!ok) break;
             tc_commit(&S.acc_full[a]);
-            ++seg;
+            if (a) ++use1; else ++use0;
+            if (g.whole) ++lmseg;
         }
     };
     auto att = [&](int64_t a0, int64_t a1) {
@@ -397,34 +451,32 @@ __device__ __forceinline__ void mega_mma(const MegaParams &p, MegaSmem &S, uint8
         for (int i = 0; i <= n && ok; ++i) {
             if (i < n) {  // scores S = K q^T of unit i
                 const int g = gi + i, b = g & 1;
-                const uint32_t w0 = wb + 4 * i;
-                if (!mwait(&S.q_ready[b], (g >> 1) & 1, err, ab) || !wwait(w0) || !wwait(w0 + 1)) { ok = false; break; }
+                const uint32_t w0 = wb + 2 * i;
+                if (!mwait(&S.q_ready[b], (g >> 1) & 1, err, ab) || !wwait(w0)) { ok = false; break; }
                 tc_fence_after();
-                const uint32_t dS = tmem + kTmemS + 16 * b, qb = smem_u32(sQ + 4096 * b);
+                const uint32_t dS = tmem + kTmemS + 16 * b, qb = smem_u32(sQ + 4096 * b), kb = wslot(w0);
                 for (int ks = 0; ks < p.hd / 16; ++ks)
-                    tc_mma_bf16(dS, sdesc_kmajor_sw128(wslot(w0 + (ks >> 2)) + (ks & 3) * 32),
+                    tc_mma_bf16(dS, sdesc_kmajor_sw128(kb + (ks >> 2) * 16384 + (ks & 3) * 32),
                                 sdesc_kmajor_sw128(qb + (ks >> 2) * 2048 + (ks & 3) * 32), ida, ks > 0 ? 1u : 0u);
                 tc_commit(&S.s_full[b]);
                 tc_commit(&S.wempty[w0 % kWSlots]);
-                tc_commit(&S.wempty[(w0 + 1) % kWSlots]);
             }
             if (i >= 1) {  // output O^T = V^T P^T of unit i - 1
                 const int g = gi + i - 1, b = g & 1;
-                const uint32_t w0 = wb + 4 * (i - 1);
+                const uint32_t w1 = wb + 2 * (i - 1) + 1;
                 const AttUnit u = att_unit(p, a0 + i - 1);
-                if (!mwait(&S.p_ready[b], (g >> 1) & 1, err, ab) || !wwait(w0 + 2) || !wwait(w0 + 3)) { ok = false; break; }
+                if (!mwait(&S.p_ready[b], (g >> 1) & 1, err, ab) || !wwait(w1)) { ok = false; break; }
                 tc_fence_after();
-                const uint32_t dO = tmem + kTmemO + 16 * b, pb = smem_u32(sP + 4096 * b);
+                const uint32_t dO = tmem + kTmemO + 16 * b, pb = smem_u32(sP + 4096 * b), vb = wslot(w1);
                 const int ksteps = (u.n + 15) >> 4;
                 for (int ks = 0; ks < ksteps; ++ks)
-                    tc_mma_bf16(dO, sdesc_kmajor_sw128(wslot(w0 + 2 + (ks >> 2)) + (ks & 3) * 32),
+                    tc_mma_bf16(dO, sdesc_kmajor_sw128(vb + (ks >> 2) * 16384 + (ks & 3) * 32),
                                 sdesc_kmajor_sw128(pb + (ks >> 2) * 2048 + (ks & 3) * 32), ida, ks > 0 ? 1u : 0u);
                 tc_commit(&S.o_full[b]);
-                tc_commit(&S.wempty[(w0 + 2) % kWSlots]);
-                tc_commit(&S.wempty[(w0 + 3) % kWSlots]);
+                tc_commit(&S.wempty[w1 % kWSlots]);
             }
         }
-        wi = wb + 4 * n;
+        wi = wb + 2 * n;
         gi += n;
     };
     for (int l = 0; l <= p.layers && ok; ++l) {
@@ -432,12 +484,14 @@ __device__ __forceinline__ void mega_mma(const MegaParams &p, MegaSmem &S, uint8
             if (l == p.layers && k > 0) break;
             const GemmPh g = gemm_phase(p, l, k);
             int64_t u0, u1;
-            gemm_range(g, l == p.layers, u0, u1);
+            gemm_range(g, u0, u1);
             gemm(g, u0, u1);
+            MEGA_STAMP(1 + kPhasesPerLayer * l + k, 3);
             if (k == 0 && l < p.layers && ok) {
                 int64_t a0, a1;
                 att_range(p, S.n_items, a0, a1);
                 att(a0, a1);
+                MEGA_STAMP(2 + kPhasesPerLayer * l, 3);
             }
         }
     }
@@ -454,41 +508,44 @@ __device__ __forceinline__ void store_hilo(uint8_t *hi, uint8_t *lo, int64_t off
     *reinterpret_cast<uint16_t *>(lo + off) = l;
 }
 
-__device__ __forceinline__ float unfix(unsigned long long v) { return (float)(long long)v * kUnfix; }
-
-// 8 consecutive head dims (granule j) of one head of accQ, RMSNorm-scaled by `scale`, with
-// the rotary embedding (pairs i, i + hd/2) when `rot`.
-__device__ __forceinline__ void head_granule(const unsigned long long *src, int j, int hd, const float2 *cs, bool rot,
-                                             float scale, float (&y)[8]) {
+// 8 consecutive head dims (granule j) of one head of the QKV output (sum of the tile's
+// partials in CTA order), RMSNorm-scaled by `scale`, with the rotary embedding (pairs
+// i, i + hd/2) when `rot`.  A head lies inside one 256-feature tile, so the granule and its
+// rotation partner are read in the same pass over the contributors.
+__device__ __forceinline__ void head_granule(const MegaParams &p, const GemmPh &g, int r, int head, int j, int hd,
+                                             const float2 *cs, bool rot, float scale, float (&y)[8]) {
     const int d0 = j * 8, half = hd >> 1;
-    const ulonglong2 *a = reinterpret_cast<const ulonglong2 *>(src + d0);
-    float x[8];
+    const bool low = d0 < half;
+    const int pd0 = low ? d0 + half : d0 - half;
+    const int f0 = head * hd + d0, t = f0 / kTileN;
+    const int col = f0 - t * kTileN, pcol = head * hd + pd0 - t * kTileN;
+    int ca, cb;
+    tile_ctas(g, t, ca, cb);
+    float x[8], xp[8];
 #pragma unroll
-    for (int e = 0; e < 4; ++e) {
-        const ulonglong2 t = __ldcg(a + e);
-        x[2 * e] = unfix(t.x);
-        x[2 * e + 1] = unfix(t.y);
+    for (int e = 0; e < 8; ++e) x[e] = xp[e] = 0.f;
+#pragma unroll 4
+    for (int c = ca; c <= cb; ++c) {
+        const float *base = p.gpart + ((int64_t)(c + t) * p.rows_cap + r) * kTileN;
+        const float4 a = __ldcg(reinterpret_cast<const float4 *>(base + col));
+        const float4 b = __ldcg(reinterpret_cast<const float4 *>(base + col + 4));
+        const float4 pa = rot ? __ldcg(reinterpret_cast<const float4 *>(base + pcol)) : make_float4(0.f, 0.f, 0.f, 0.f);
+        const float4 pb = rot ? __ldcg(reinterpret_cast<const float4 *>(base + pcol + 4)) : make_float4(0.f, 0.f, 0.f, 0.f);
+        x[0] += a.x; x[1] += a.y; x[2] += a.z; x[3] += a.w;
+        x[4] += b.x; x[5] += b.y; x[6] += b.z; x[7] += b.w;
+        xp[0] += pa.x; xp[1] += pa.y; xp[2] += pa.z; xp[3] += pa.w;
+        xp[4] += pb.x; xp[5] += pb.y; xp[6] += pb.z; xp[7] += pb.w;
     }
     if (!rot) {
 #pragma unroll
         for (int e = 0; e < 8; ++e) y[e] = x[e] * scale;
         return;
     }
-    const bool low = d0 < half;
-    const int pd0 = low ? d0 + half : d0 - half;
-    const ulonglong2 *b = reinterpret_cast<const ulonglong2 *>(src + pd0);
-    float xp[8];
-#pragma unroll
-    for (int e = 0; e < 4; ++e) {
-        const ulonglong2 t = __ldcg(b + e);
-        xp[2 * e] = unfix(t.x);
-        xp[2 * e + 1] = unfix(t.y);
-    }
-    const int f0 = low ? d0 : pd0;
+    const int fr = low ? d0 : pd0;
 #pragma unroll
     for (int e = 0; e < 8; ++e) {
-        const float2 r = __ldg(&cs[f0 + e]);
-        y[e] = (low ? (x[e] * r.x - xp[e] * r.y) : (x[e] * r.x + xp[e] * r.y)) * scale;
+        const float2 c = __ldg(&cs[fr + e]);
+        y[e] = (low ? (x[e] * c.x - xp[e] * c.y) : (x[e] * c.x + xp[e] * c.y)) * scale;
     }
 }
 
@@ -498,10 +555,6 @@ __device__ __forceinline__ uint4 pack_f16x8(const float (&y)[8]) {
     for (int e = 0; e < 4; ++e)
         w[e] = (uint32_t)f32_to_f16_sat(y[2 * e]) | ((uint32_t)f32_to_f16_sat(y[2 * e + 1]) << 16);
     return make_uint4(w[0], w[1], w[2], w[3]);
-}
-
-__device__ __forceinline__ void argmax_combine(float &v, int &i, float ov, int oi) {
-    if (ov > v || (ov == v && oi < i)) { v = ov; i = oi; }
 }
 
 __device__ __forceinline__ void mega_compute(const MegaParams &p, MegaSmem &S, uint8_t *sW, uint8_t *sQ, uint8_t *sP,
@@ -517,66 +570,83 @@ __device__ __forceinline__ void mega_compute(const MegaParams &p, MegaSmem &S, u
     const int d = p.d, dt = d / 128, hd = p.hd, Gq = p.Gq;
     const int gw = cta * 8 + cw, nw = G * 8;
     const uint32_t lane_base = (uint32_t)(quarter * 32) << 16;
+    const int my_row = quarter * 32 + lane;  // GEMM accumulator lane = activation row
     uint32_t wi = 0;
-    int seg = 0, gi = 0;
+    int gi = 0, cuse0 = 0, cuse1 = 0, lmseg = 0;  // accumulator buffer uses
 
+    // phase arrival: the CTA's writes of this phase (made visible to thread 0 by the barrier)
+    // are released to the other CTAs with the counter increment
     auto arrive = [&](int idx) {
         fence_proxy_async_global();
-        __threadfence();
         named_bar_sync(1, kMegaCThreads);
         if (ctid == 0) {
-            __threadfence();
+            fence_acq_rel_gpu();
+            MEGA_STAMP(idx, 0);
             atomicAdd(&p.cnt[idx], 1ull);
         }
     };
     auto wait_phase = [&](int idx) {
-        if (ctid == 0) spin_counter(&p.cnt[idx], S.target, err, ab);
+        if (ctid == 0) {
+            spin_counter(&p.cnt[idx], S.target, err, ab);
+            MEGA_STAMP(idx + 1, 1);
+        }
         named_bar_sync(1, kMegaCThreads);
     };
     auto load_rstd = [&](const float *ssq) {
         if (ctid < R) {
             float s = 0.f;
+#pragma unroll 16
             for (int t = 0; t < dt; ++t) s += __ldcg(&ssq[(int64_t)t * p.rows_cap + ctid]);
             S.rstd[ctid] = rsqrtf(s / (float)d + p.eps);
         }
         named_bar_sync(1, kMegaCThreads);
     };
-    // fixed-point fold of this CTA's partial tile sums (every k-split adds into acc)
+    // this CTA's partial tiles: row my_row, columns [128 half, +128) of the tile
     auto gemm_epi = [&](const GemmPh &g, int64_t u0, int64_t u1) {
         for (int64_t u = u0; u < u1;) {
-            const int tile = (int)(u / g.kch);
-            u = min(u1, (int64_t)(tile + 1) * g.kch);
-            const int a = seg & 1;
-            mwait(&S.acc_full[a], (seg >> 1) & 1, err, ab);
+            const int t = (int)(u / g.kch);
+            u = min(u1, (int64_t)(t + 1) * g.kch);
+            mwait(&S.acc_full[0], cuse0 & 1, err, ab);
             tc_fence_after();
-            const int n = tile * 128 + quarter * 32 + lane;
-            for (int cc = half; cc * 32 < R; cc += 2) {
-                float v[32];
-                tmem_ld_32x32b_x32(tmem + lane_base + (uint32_t)(a * 128 + cc * 32), v);
+            const int rows_t = tile_rows(g, t);
+            if (quarter * 32 < R && half * 128 < rows_t) {
+                float *dst = p.gpart + ((int64_t)(cta + t) * p.rows_cap + my_row) * kTileN + half * 128;
+#pragma unroll 1
+                for (int cc = 0; cc < 4; ++cc) {
+                    float v[32];
+                    tmem_ld_32x32b_x32(tmem + lane_base + (uint32_t)(half * 128 + cc * 32), v);
+                    if (my_row < R) {
+                        float4 *q = reinterpret_cast<float4 *>(dst + cc * 32);
 #pragma unroll
-                for (int j = 0; j < 32; ++j) {
-                    const int r = cc * 32 + j;
-                    if (r < R) atomicAdd(&g.acc[(int64_t)r * g.ld + n], (unsigned long long)__float2ll_rn(v[j] * kFix));
+                        for (int e = 0; e < 8; ++e) q[e] = make_float4(v[4 * e], v[4 * e + 1], v[4 * e + 2], v[4 * e + 3]);
+                    }
                 }
             }
             tc_fence_before();
             __syncwarp();
-            if (lane == 0) mbar_arrive(&S.acc_empty[a]);
-            ++seg;
+            if (lane == 0) mbar_arrive(&S.acc_empty[0]);
+            ++cuse0;
         }
     };
-    // x += acc; x_g = x * gw (blocked hi/lo); per (row, 128-feature block) sum of squares
-    auto fin_resid = [&](unsigned long long *acc, const uint16_t *gn, float *ssq) {
+    // x += (sum of g's partials); x_g = x * gn (blocked hi/lo); per (row, 128-feature
+    // block) sum of squares of x.  g == nullptr: x as it is (embedding).
+    auto fin_resid = [&](const GemmPh *g, const uint16_t *gn, float *ssq) {
         for (int u = gw; u < R * dt; u += nw) {
             const int r = u / dt, t = u - r * dt;
             const int f = t * 128 + lane * 4;
             float4 x = __ldcg(reinterpret_cast<const float4 *>(p.x + (int64_t)r * d + f));
-            if (acc) {
-                ulonglong2 *ap = reinterpret_cast<ulonglong2 *>(acc + (int64_t)r * d + f);
-                const ulonglong2 a0 = __ldcg(ap), a1 = __ldcg(ap + 1);
-                x.x += unfix(a0.x); x.y += unfix(a0.y); x.z += unfix(a1.x); x.w += unfix(a1.y);
-                ap[0] = make_ulonglong2(0ull, 0ull);
-                ap[1] = make_ulonglong2(0ull, 0ull);
+            if (g) {
+                const int gt = f / kTileN, col = f - gt * kTileN;
+                int ca, cb;
+                tile_ctas(*g, gt, ca, cb);
+                float4 s = make_float4(0.f, 0.f, 0.f, 0.f);
+#pragma unroll 8
+                for (int c = ca; c <= cb; ++c) {
+                    const float4 v = __ldcg(reinterpret_cast<const float4 *>(
+                        p.gpart + ((int64_t)(c + gt) * p.rows_cap + r) * kTileN + col));
+                    s.x += v.x; s.y += v.y; s.z += v.z; s.w += v.w;
+                }
+                x.x += s.x; x.y += s.y; x.z += s.z; x.w += s.w;
                 *reinterpret_cast<float4 *>(p.x + (int64_t)r * d + f) = x;
             }
             const uint2 gb = *reinterpret_cast<const uint2 *>(gn + f);
@@ -618,14 +688,13 @@ __device__ __forceinline__ void mega_compute(const MegaParams &p, MegaSmem &S, u
     for (int l = 0; l < p.layers; ++l) {
         const int base = 1 + kPhasesPerLayer * l;
         int64_t u0, u1;
+        const GemmPh gq = gemm_phase(p, l, 0), go = gemm_phase(p, l, 2), gu = gemm_phase(p, l, 4),
+                     gdn = gemm_phase(p, l, 6);
         // ------------------------------------------------------------ QKV
-        {
-            const GemmPh g = gemm_phase(p, l, 0);
-            gemm_range(g, false, u0, u1);
-            gemm_epi(g, u0, u1);
-            wi += (uint32_t)(u1 - u0);
-            arrive(base + 0);
-        }
+        gemm_range(gq, u0, u1);
+        gemm_epi(gq, u0, u1);
+        wi += (uint32_t)(u1 - u0);
+        arrive(base + 0);
         // ------------------------------------------------------------ attention
         {
             wait_phase(base + 0);
@@ -634,68 +703,77 @@ __device__ __forceinline__ void mega_compute(const MegaParams &p, MegaSmem &S, u
             att_range(p, S.n_items, a0, a1);
             const int n = (int)(a1 - a0);
             const uint32_t wb = wi;
-            const float2 *rope = p.rope;
-            // warps 3..6 run the attention units; warps 7..10 wait at the phase arrival
-            for (int i = 0; half == 0 && i < n + 2; ++i) {
-                if (i < n) {  // q tile of unit i (+ the new position's k, v on the last split)
+            const bool det_layer = l == min(2, p.layers - 1);
+#define DETAIL(i)                                       \
+    do {                                                \
+        if (det_layer && ctid == 0 && i_unit == 0) MEGA_DETAIL(i); \
+    } while (0)
+            int i_unit = 0;
+            DETAIL(0);
+            // per unit i: all compute warps build the q tile (warps 3..6) and, on a row's last
+            // split, the new position's k and v (warps 7..10); warps 3..6 then run the softmax
+            // of unit i - 1 and the output / split merge of unit i - 2
+            for (int i = 0; i < n + 2; ++i) {
+                if (i < n) {
                     const AttUnit u = att_unit(p, a0 + i);
                     const int b = (gi + i) & 1;
                     const float rs = S.rstd[u.row];
-                    const float2 *cs = rope + (int64_t)(u.ctx - 1) * (hd / 2);
-                    const int g = ctid >> 4, j = ctid & 15;  // rows 0..7 (score columns 8..15 unused)
-                    uint4 pk = make_uint4(0, 0, 0, 0);
-                    if (g < Gq && j * 8 < hd) {
-                        float y[8];
-                        head_granule(p.accQ + (int64_t)u.row * p.nqkv + (u.kvh * Gq + g) * hd, j, hd, cs, true,
-                                     rs * p.scale_log2, y);
-                        pk = pack_f16x8(y);
-                    }
-                    *reinterpret_cast<uint4 *>(sQ + 4096 * b + (j >> 3) * 2048 + g * 128 + (((j & 7) ^ (g & 7)) << 4)) = pk;
-                    if (u.last && ctid < 32) {
+                    const float2 *cs = p.rope + (int64_t)(u.ctx - 1) * (hd / 2);
+                    if (half == 0) {  // q tile rows 0..7 (score columns 8..15 are unused)
+                        const int g = ctid >> 4, j = ctid & 15;
+                        uint4 pk = make_uint4(0, 0, 0, 0);
+                        if (g < Gq && j * 8 < hd) {
+                            float y[8];
+                            head_granule(p, gq, u.row, u.kvh * Gq + g, j, hd, cs, true, rs * p.scale_log2, y);
+                            pk = pack_f16x8(y);
+                        }
+                        *reinterpret_cast<uint4 *>(sQ + 4096 * b + (j >> 3) * 2048 + g * 128 + (((j & 7) ^ (g & 7)) << 4)) =
+                            pk;
+                    } else if (u.last && ctid < 160) {  // k, v of the new position (cache + ring slot)
                         const int jj = ctid & 15;
-                        const bool isv = ctid >= 16;
+                        const bool isv = ctid >= 144;
                         if (jj * 8 < hd) {
-                            const uint32_t w0 = wb + 4 * i;
                             const int pp = u.ctx - 1 - u.p0;
                             const int head = p.H + (isv ? p.KVH : 0) + u.kvh;
                             float y[8];
-                            head_granule(p.accQ + (int64_t)u.row * p.nqkv + head * hd, jj, hd, cs, !isv, rs, y);
+                            head_granule(p, gq, u.row, head, jj, hd, cs, !isv, rs, y);
                             uint8_t *gblk = kv_block(p, l, u);
+                            const uint32_t ws = wb + 2 * i + (isv ? 1 : 0);
+                            mwait(&S.wfull[ws % kWSlots], (ws / kWSlots) & 1, err, ab);
+                            uint8_t *slot = sW + (size_t)(ws % kWSlots) * kSlotBytes;
                             if (!isv) {
                                 const uint4 kp = pack_f16x8(y);
                                 const int off = kv_k_off(pp, jj * 8);
                                 *reinterpret_cast<uint4 *>(gblk + off) = kp;
-                                const uint32_t ws = w0 + (jj >> 3);
-                                mwait(&S.wfull[ws % kWSlots], (ws / kWSlots) & 1, err, ab);
-                                *reinterpret_cast<uint4 *>(sW + (size_t)(ws % kWSlots) * kSlotBytes + (off & 16383)) = kp;
+                                *reinterpret_cast<uint4 *>(slot + off) = kp;
                             } else {
-                                const uint32_t ws = w0 + 2 + (pp >> 6);
-                                mwait(&S.wfull[ws % kWSlots], (ws / kWSlots) & 1, err, ab);
-                                uint8_t *sv = sW + (size_t)(ws % kWSlots) * kSlotBytes;
 #pragma unroll
                                 for (int e = 0; e < 8; ++e) {
                                     const uint16_t hv = f32_to_f16_sat(y[e]);
                                     const int off = kv_v_off(pp, jj * 8 + e);
                                     *reinterpret_cast<uint16_t *>(gblk + off) = hv;
-                                    *reinterpret_cast<uint16_t *>(sv + (off & 16383)) = hv;
+                                    *reinterpret_cast<uint16_t *>(slot + off - 32768) = hv;
                                 }
                             }
                         }
                     }
                     fence_proxy_async_smem();
-                    named_bar_sync(2, 128);
+                    named_bar_sync(1, kMegaCThreads);
+                    i_unit = i;
+                    DETAIL(1);
                     if (ctid == 0) mbar_arrive(&S.q_ready[b]);
                 }
-                if (i >= 1 && i <= n) {  // softmax of unit i - 1 -> P
+                if (half == 0 && i >= 1 && i <= n) {  // softmax of unit i - 1 -> P
                     const AttUnit u = att_unit(p, a0 + i - 1);
                     const int g1 = gi + i - 1, b = g1 & 1;
                     mwait(&S.s_full[b], (g1 >> 1) & 1, err, ab);
+                    i_unit = i - 1;
+                    DETAIL(2);
                     tc_fence_after();
                     float sv[8];
                     tmem_ld_32x32b_x8(tmem + lane_base + kTmemS + 16 * b, sv);
                     const int pos = quarter * 32 + lane;
                     const bool valid = pos < u.n;
-                    float M[8];
 #pragma unroll
                     for (int g = 0; g < 8; ++g) {
                         sv[g] = valid ? sv[g] : -INFINITY;
@@ -704,42 +782,43 @@ __device__ __forceinline__ void mega_compute(const MegaParams &p, MegaSmem &S, u
                         for (int o = 16; o > 0; o >>= 1) m = fmaxf(m, __shfl_xor_sync(0xffffffffu, m, o));
                         if (lane == 0) S.red[quarter][g] = m;
                     }
+                    tc_fence_before();
                     named_bar_sync(2, 128);
-#pragma unroll
-                    for (int g = 0; g < 8; ++g)
-                        M[g] = fmaxf(fmaxf(S.red[0][g], S.red[1][g]), fmaxf(S.red[2][g], S.red[3][g]));
-                    named_bar_sync(2, 128);
+                    float M[8];
                     uint8_t *pb = sP + 4096 * b + (pos >> 6) * 2048;
                     const int pc = pos & 63;
 #pragma unroll
                     for (int g = 0; g < 8; ++g) {
+                        M[g] = fmaxf(fmaxf(S.red[0][g], S.red[1][g]), fmaxf(S.red[2][g], S.red[3][g]));
                         const float e = valid ? exp2f(sv[g] - M[g]) : 0.f;
                         *reinterpret_cast<uint16_t *>(pb + g * 128 + ((((pc >> 3) ^ (g & 7)) << 4) | ((pc & 7) << 1))) =
                             f32_to_f16_sat(e);
-                        const float s = warp_sum(e);
-                        if (lane == 0) S.red[quarter][g] = s;
+                        const float se = warp_sum(e);
+                        if (lane == 0) S.red2[quarter][g] = se;
                     }
                     fence_proxy_async_smem();
-                    tc_fence_before();
                     named_bar_sync(2, 128);
-                    if (ctid < 8) {
+                    DETAIL(3);
+                    if (ctid == 0) mbar_arrive(&S.p_ready[b]);
+                    if (ctid < 8) {  // read by the output step of this unit, after more barriers
                         float mc = M[0];
 #pragma unroll
                         for (int g = 1; g < 8; ++g) mc = (ctid == g) ? M[g] : mc;
                         S.att_m[b][ctid] = mc;
-                        S.att_l[b][ctid] = S.red[0][ctid] + S.red[1][ctid] + S.red[2][ctid] + S.red[3][ctid];
+                        S.att_l[b][ctid] = S.red2[0][ctid] + S.red2[1][ctid] + S.red2[2][ctid] + S.red2[3][ctid];
                     }
-                    named_bar_sync(2, 128);
-                    if (ctid == 0) mbar_arrive(&S.p_ready[b]);
                 }
-                if (i >= 2) {  // output of unit i - 2
+                if (half == 0 && i >= 2) {  // output of unit i - 2
                     const AttUnit u = att_unit(p, a0 + i - 2);
                     const int g2 = gi + i - 2, b = g2 & 1;
                     mwait(&S.o_full[b], (g2 >> 1) & 1, err, ab);
+                    i_unit = i - 2;
+                    DETAIL(4);
                     tc_fence_after();
                     float ov[8];
                     tmem_ld_32x32b_x8(tmem + lane_base + kTmemO + 16 * b, ov);
                     tc_fence_before();
+                    named_bar_sync(2, 128);  // att_m / att_l of this buffer are complete
                     const int dd = quarter * 32 + lane;
                     if (u.nsplit == 1) {
                         if (dd < hd) {
@@ -760,193 +839,180 @@ __device__ __forceinline__ void mega_compute(const MegaParams &p, MegaSmem &S, u
                             mine[ctid * (hd + 2)] = S.att_m[b][ctid];
                             mine[ctid * (hd + 2) + 1] = S.att_l[b][ctid];
                         }
-                        __threadfence();
                         named_bar_sync(2, 128);
+                        DETAIL(5);
                         if (ctid == 0) {
+                            fence_acq_rel_gpu();
                             const int old = atomicAdd(&p.att_cnt[u.row * p.KVH + u.kvh], 1);
                             S.last_flag = old == u.nsplit - 1;
                             if (S.last_flag) p.att_cnt[u.row * p.KVH + u.kvh] = 0;
+                            fence_acq_rel_gpu();
                         }
                         named_bar_sync(2, 128);
+                        DETAIL(6);
                         if (S.last_flag) {  // merge the row's splits in split order
-                            __threadfence();
                             const int ns = min(u.nsplit, kMegaMaxSplits);
                             const int64_t sp_stride = (int64_t)p.KVH * Gq * (hd + 2);
                             const float *pbase = p.part + ((int64_t)p.c.row_item0[u.row] * p.KVH + u.kvh) * Gq * (hd + 2);
+                            // split weights 2^(m_s - M) and the total weight L per head (warp cw: heads cw, cw + 4)
                             for (int g = cw; g < Gq; g += 4) {
+                                float ms[3], ls[3];
                                 float Mx = -INFINITY;
-                                for (int s = lane; s < ns; s += 32) Mx = fmaxf(Mx, __ldcg(pbase + s * sp_stride + g * (hd + 2)));
+#pragma unroll
+                                for (int q = 0; q < 3; ++q) {
+                                    const int sp = lane + 32 * q;
+                                    ms[q] = sp < ns ? __ldcg(pbase + sp * sp_stride + g * (hd + 2)) : -INFINITY;
+                                    ls[q] = sp < ns ? __ldcg(pbase + sp * sp_stride + g * (hd + 2) + 1) : 0.f;
+                                    Mx = fmaxf(Mx, ms[q]);
+                                }
 #pragma unroll
                                 for (int o = 16; o > 0; o >>= 1) Mx = fmaxf(Mx, __shfl_xor_sync(0xffffffffu, Mx, o));
                                 float L = 0.f;
-                                for (int s = lane; s < ns; s += 32) {
-                                    const float ms = __ldcg(pbase + s * sp_stride + g * (hd + 2));
-                                    const float w = exp2f(ms - Mx);
-                                    S.mw[g][s] = w;
-                                    L += w * __ldcg(pbase + s * sp_stride + g * (hd + 2) + 1);
+#pragma unroll
+                                for (int q = 0; q < 3; ++q) {
+                                    const int sp = lane + 32 * q;
+                                    const float w = sp < ns ? exp2f(ms[q] - Mx) : 0.f;
+                                    if (sp < ns) S.mw[g][sp] = w;
+                                    L += w * ls[q];
                                 }
                                 L = warp_sum(L);
                                 if (lane == 0) S.ml[g] = L;
                             }
                             named_bar_sync(2, 128);
-                            for (int e = ctid; e < Gq * hd; e += 128) {
-                                const int g = e / hd, de = e - g * hd;
-                                const float *src = pbase + g * (hd + 2) + 2 + de;
-                                float acc = 0.f;
-#pragma unroll 4
-                                for (int s = 0; s < ns; ++s) acc += S.mw[g][s] * __ldcg(src + s * sp_stride);
-                                store_hilo(p.att_hi, p.att_lo, xblk_off(u.row, (u.kvh * Gq + g) * hd + de, R16c),
-                                           acc / S.ml[g]);
+                            if (dd < hd) {  // thread dd: output dim dd of every head
+                                float acc[8];
+#pragma unroll
+                                for (int g = 0; g < 8; ++g) acc[g] = 0.f;
+                                const float *src = pbase + 2 + dd;
+#pragma unroll 2
+                                for (int sp = 0; sp < ns; ++sp) {
+                                    float v[8];
+#pragma unroll
+                                    for (int g = 0; g < 8; ++g) v[g] = g < Gq ? __ldcg(src + sp * sp_stride + g * (hd + 2)) : 0.f;
+#pragma unroll
+                                    for (int g = 0; g < 8; ++g) acc[g] += (g < Gq ? S.mw[g][sp] : 0.f) * v[g];
+                                }
+#pragma unroll
+                                for (int g = 0; g < 8; ++g)
+                                    if (g < Gq)
+                                        store_hilo(p.att_hi, p.att_lo, xblk_off(u.row, (u.kvh * Gq + g) * hd + dd, R16c),
+                                                   acc[g] / S.ml[g]);
                             }
                         }
                         named_bar_sync(2, 128);
+                        DETAIL(7);
                     }
                 }
             }
-            wi = wb + 4 * n;
+            wi = wb + 2 * n;
             gi += n;
+            i_unit = 0;
+            DETAIL(8);
             arrive(base + 1);
+            DETAIL(9);
+#undef DETAIL
         }
         // ------------------------------------------------------------ O projection
-        {
-            const GemmPh g = gemm_phase(p, l, 2);
-            gemm_range(g, false, u0, u1);
-            gemm_epi(g, u0, u1);
-            wi += (uint32_t)(u1 - u0);
-            arrive(base + 2);
-        }
+        gemm_range(go, u0, u1);
+        gemm_epi(go, u0, u1);
+        wi += (uint32_t)(u1 - u0);
+        arrive(base + 2);
         // ------------------------------------------------------------ residual, MLP norm input
-        {
-            wait_phase(base + 2);
-            fin_resid(p.accO, p.mlp_norm + (int64_t)l * d, p.ssqM);
-            // accQ is no longer read by anyone: clear the live rows for the next layer
-            const int64_t nz = (int64_t)R * p.nqkv / 2;
-            ulonglong2 *q2 = reinterpret_cast<ulonglong2 *>(p.accQ);
-            for (int64_t e = (int64_t)cta * kMegaCThreads + ctid; e < nz; e += (int64_t)G * kMegaCThreads)
-                q2[e] = make_ulonglong2(0ull, 0ull);
-            arrive(base + 3);
-        }
+        wait_phase(base + 2);
+        if (l == min(2, p.layers - 1) && ctid == 0) MEGA_DETAIL(10);
+        fin_resid(&go, p.mlp_norm + (int64_t)l * d, p.ssqM);
+        if (l == min(2, p.layers - 1) && ctid == 0) MEGA_DETAIL(11);
+        arrive(base + 3);
+        if (l == min(2, p.layers - 1) && ctid == 0) MEGA_DETAIL(12);
         // ------------------------------------------------------------ gate / up
-        {
-            const GemmPh g = gemm_phase(p, l, 4);
-            gemm_range(g, false, u0, u1);
-            gemm_epi(g, u0, u1);
-            wi += (uint32_t)(u1 - u0);
-            arrive(base + 4);
-        }
+        gemm_range(gu, u0, u1);
+        gemm_epi(gu, u0, u1);
+        wi += (uint32_t)(u1 - u0);
+        arrive(base + 4);
         // ------------------------------------------------------------ SwiGLU
         {
             wait_phase(base + 4);
             load_rstd(p.ssqM);
-            const int fb = p.F / 64;
+            const int fb = p.F / 128;
             for (int u = gw; u < R * fb; u += nw) {
-                const int r = u / fb, jb = u - r * fb;
+                const int r = u / fb, t = u - r * fb;
                 const float rs = S.rstd[r];
-                unsigned long long *gp = p.accGU + (int64_t)r * 2 * p.F + jb * 128 + 2 * lane;
-                ulonglong2 *g2 = reinterpret_cast<ulonglong2 *>(gp);
-                ulonglong2 *u2 = reinterpret_cast<ulonglong2 *>(gp + 64);
-                const ulonglong2 ga = __ldcg(g2), ua = __ldcg(u2);
-                *g2 = make_ulonglong2(0ull, 0ull);
-                *u2 = make_ulonglong2(0ull, 0ull);
-                const float gv0 = unfix(ga.x) * rs, gv1 = unfix(ga.y) * rs;
-                const float uv0 = unfix(ua.x) * rs, uv1 = unfix(ua.y) * rs;
-                const float h0 = gv0 / (1.0f + expf(-gv0)) * uv0, h1 = gv1 / (1.0f + expf(-gv1)) * uv1;
-                uint16_t a0h, a0l, a1h, a1l;
-                split_bf16(h0, a0h, a0l);
-                split_bf16(h1, a1h, a1l);
-                const int64_t off = xblk_off(r, jb * 64 + 2 * lane, R16c);
-                *reinterpret_cast<uint32_t *>(p.h_hi + off) = (uint32_t)a0h | ((uint32_t)a1h << 16);
-                *reinterpret_cast<uint32_t *>(p.h_lo + off) = (uint32_t)a0l | ((uint32_t)a1l << 16);
+                // h features 128 t + 4 lane .. +3: gate at tile column c, up at c + 64, with
+                // c = 4 lane (features < 64 of the tile) or 128 + 4 lane - 64 (the rest)
+                const int c0 = (lane < 16) ? 4 * lane : 128 + 4 * lane - 64;
+                int ca, cb;
+                tile_ctas(gu, t, ca, cb);
+                float4 gs = make_float4(0.f, 0.f, 0.f, 0.f), us = gs;
+#pragma unroll 4
+                for (int c = ca; c <= cb; ++c) {
+                    const float *src = p.gpart + ((int64_t)(c + t) * p.rows_cap + r) * kTileN + c0;
+                    const float4 a = __ldcg(reinterpret_cast<const float4 *>(src));
+                    const float4 bq = __ldcg(reinterpret_cast<const float4 *>(src + 64));
+                    gs.x += a.x; gs.y += a.y; gs.z += a.z; gs.w += a.w;
+                    us.x += bq.x; us.y += bq.y; us.z += bq.z; us.w += bq.w;
+                }
+                const float gv[4] = {gs.x * rs, gs.y * rs, gs.z * rs, gs.w * rs};
+                const float uv[4] = {us.x * rs, us.y * rs, us.z * rs, us.w * rs};
+                uint16_t hh[4], hl[4];
+#pragma unroll
+                for (int e = 0; e < 4; ++e) split_bf16(gv[e] / (1.0f + expf(-gv[e])) * uv[e], hh[e], hl[e]);
+                const int64_t off = xblk_off(r, t * 128 + 4 * lane, R16c);
+                *reinterpret_cast<uint2 *>(p.h_hi + off) =
+                    make_uint2((uint32_t)hh[0] | ((uint32_t)hh[1] << 16), (uint32_t)hh[2] | ((uint32_t)hh[3] << 16));
+                *reinterpret_cast<uint2 *>(p.h_lo + off) =
+                    make_uint2((uint32_t)hl[0] | ((uint32_t)hl[1] << 16), (uint32_t)hl[2] | ((uint32_t)hl[3] << 16));
             }
             arrive(base + 5);
         }
         // ------------------------------------------------------------ down
-        {
-            const GemmPh g = gemm_phase(p, l, 6);
-            gemm_range(g, false, u0, u1);
-            gemm_epi(g, u0, u1);
-            wi += (uint32_t)(u1 - u0);
-            arrive(base + 6);
-        }
+        gemm_range(gdn, u0, u1);
+        gemm_epi(gdn, u0, u1);
+        wi += (uint32_t)(u1 - u0);
+        arrive(base + 6);
         // ------------------------------------------------------------ residual, next norm input
-        {
-            wait_phase(base + 6);
-            const uint16_t *gn = (l + 1 < p.layers) ? p.attn_norm + (int64_t)(l + 1) * d : p.final_norm;
-            fin_resid(p.accD, gn, p.ssqA);
-            arrive(base + 7);
-        }
+        wait_phase(base + 6);
+        fin_resid(&gdn, (l + 1 < p.layers) ? p.attn_norm + (int64_t)(l + 1) * d : p.final_norm, p.ssqA);
+        arrive(base + 7);
     }
 
-    // ---------------------------------------------------------------- lm_head + Gumbel-max
+    // ---------------------------------------------------------------- lm_head
+    // logits = (x_g W_lm^T) / rms(x) for the live rows; the sampling kernel that follows
+    // spreads the Gumbel-max over the whole GPU
     {
         wait_phase(kPhasesPerLayer * p.layers);
         load_rstd(p.ssqA);
-        if (ctid < R) S.seed[ctid] = p.c.row_seed[ctid];
-        named_bar_sync(1, kMegaCThreads);
         const GemmPh g = gemm_phase(p, p.layers, 0);
         int64_t u0, u1;
-        gemm_range(g, true, u0, u1);
-        const int ntiles = p.V / 128;
+        gemm_range(g, u0, u1);
+        const bool act = my_row < R;
+        const float rs = act ? S.rstd[my_row] : 0.f;
         for (int64_t u = u0; u < u1; u += g.kch) {
-            const int tile = (int)(u / g.kch);
-            const int a = seg & 1;
-            mwait(&S.acc_full[a], (seg >> 1) & 1, err, ab);
+            const int t = (int)(u / g.kch);
+            const int a = lmseg & 1;
+            mwait(&S.acc_full[a], (a ? cuse1 : cuse0) & 1, err, ab);
             tc_fence_after();
-            const int n = tile * 128 + quarter * 32 + lane;
-            for (int cc = half; cc * 32 < R; cc += 2) {
-                float v[32];
-                int id[32];
-                tmem_ld_32x32b_x32(tmem + lane_base + (uint32_t)(a * 128 + cc * 32), v);
+            if (quarter * 32 < R && half * 128 < tile_rows(g, t)) {
+                float *dst = p.logits + (int64_t)my_row * p.V + t * kTileN + half * 128;
+#pragma unroll 1
+                for (int cc = 0; cc < 4; ++cc) {
+                    float v[32];
+                    tmem_ld_32x32b_x32(tmem + lane_base + (uint32_t)(a * kTileN + half * 128 + cc * 32), v);
+                    if (act) {
+                        float4 *q = reinterpret_cast<float4 *>(dst + cc * 32);
 #pragma unroll
-                for (int j = 0; j < 32; ++j) {
-                    const int r = cc * 32 + j;
-                    float z = -INFINITY;
-                    if (r < R) {
-                        z = v[j] * S.rstd[r];
-                        if (p.logits) p.logits[(int64_t)r * p.V + n] = z;
-                        z += gumbel_from_hash(splitmix_at(S.seed[r], (uint64_t)n + 1));
-                    }
-                    v[j] = z;
-                    id[j] = n;
-                }
-                // transpose-reduce: after the five steps lane l holds the argmax of column l
-#pragma unroll
-                for (int s = 16; s >= 1; s >>= 1) {
-                    const bool up = (lane & s) != 0;
-#pragma unroll
-                    for (int k = 0; k < s; ++k) {
-                        const float sendv = up ? v[k] : v[k + s];
-                        const int sendi = up ? id[k] : id[k + s];
-                        const float rv = __shfl_xor_sync(0xffffffffu, sendv, s);
-                        const int ri = __shfl_xor_sync(0xffffffffu, sendi, s);
-                        float kv = up ? v[k + s] : v[k];
-                        int ki = up ? id[k + s] : id[k];
-                        argmax_combine(kv, ki, rv, ri);
-                        v[k] = kv;
-                        id[k] = ki;
+                        for (int e = 0; e < 8; ++e)
+                            q[e] = make_float4(v[4 * e] * rs, v[4 * e + 1] * rs, v[4 * e + 2] * rs, v[4 * e + 3] * rs);
                     }
                 }
-                S.lm_v[half][quarter][lane] = v[0];
-                S.lm_i[half][quarter][lane] = id[0];
-                named_bar_sync(2 + half, 128);
-                if ((ctid & 127) < 32) {
-                    const int j = ctid & 31;
-                    float bv = S.lm_v[half][0][j];
-                    int bi = S.lm_i[half][0][j];
-                    for (int q = 1; q < 4; ++q) argmax_combine(bv, bi, S.lm_v[half][q][j], S.lm_i[half][q][j]);
-                    const int r = cc * 32 + j;
-                    if (r < R) {
-                        p.arg_val[(int64_t)r * ntiles + tile] = bv;
-                        p.arg_idx[(int64_t)r * ntiles + tile] = bi;
-                    }
-                }
-                named_bar_sync(2 + half, 128);
             }
             tc_fence_before();
             __syncwarp();
             if (lane == 0) mbar_arrive(&S.acc_empty[a]);
-            ++seg;
+            if (a) ++cuse1; else ++cuse0;
+            ++lmseg;
         }
+        named_bar_sync(1, kMegaCThreads);
+        if (ctid == 0) MEGA_STAMP(1 + kPhasesPerLayer * p.layers, 0);
     }
 }
 
@@ -985,6 +1051,7 @@ __global__ void __launch_bounds__(kMegaThreads, 1) decode_step_kernel(const __gr
         S.last_flag = 0;
         fence_mbar_init();
     }
+    if (threadIdx.x == 0) MEGA_STAMP(p.n_stamp_ph - 5, 0);  // kernel start
     if (warp == 1) {
         tmem_alloc(&S.tmem_base, kTmemCols);
         tmem_relinquish();
@@ -1015,17 +1082,17 @@ __global__ void __launch_bounds__(kMegaThreads, 1) decode_step_kernel(const __gr
 }
 
 // ------------------------------------------------------------------------------ layout kernels
-// Row-major W [N][K] (bf16) -> blocked tiles: tile (n/128, k/64) is 128 rows of 128 bytes,
-// 16-byte granule j of row r stored at granule j ^ (r % 8).
+// Row-major W [N][K] (bf16) -> blocked tiles of 256 rows (the last may have fewer): block
+// (t, kc) holds rows [256 t, ..) x columns [64 kc, +64), 16-byte granule j of row r stored at
+// granule j ^ (r % 8).  N must be a multiple of 128 and K of 64.
 static __global__ void block_weights_kernel(const uint16_t *src, uint8_t *dst, int N, int K) {
-    const int gpr = K / 8, kch = K / 64;
+    const int gpr = K / 8;
     const int64_t total = (int64_t)N * gpr;
     for (int64_t e = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; e < total; e += (int64_t)gridDim.x * blockDim.x) {
         const int n = (int)(e / gpr), j = (int)(e - (int64_t)n * gpr);
-        const int r = n & 127;
+        const int t = n / kTileN, r = n - t * kTileN;
         const uint4 v = *reinterpret_cast<const uint4 *>(src + (int64_t)n * K + (int64_t)j * 8);
-        *reinterpret_cast<uint4 *>(dst + (((int64_t)(n >> 7) * kch + (j >> 3)) * 128 + r) * 128 + (((j & 7) ^ (r & 7)) << 4)) =
-            v;
+        *reinterpret_cast<uint4 *>(dst + wblk_off(N, K, t, j >> 3) + (int64_t)r * 128 + (((j & 7) ^ (r & 7)) << 4)) = v;
     }
 }
 

@@ -218,6 +218,11 @@ __device__ __forceinline__ void bulk_load(void *smem_dst, const void *src, uint3
 __device__ __forceinline__ void fence_proxy_async_smem() { asm volatile("fence.proxy.async.shared::cta;" ::: "memory"); }
 __device__ __forceinline__ void fence_proxy_async_global() { asm volatile("fence.proxy.async.global;" ::: "memory"); }
 
+// Release / acquire fence at GPU scope (lighter than the sequentially consistent
+// __threadfence): orders this thread's prior accesses, and those of its CTA made visible to
+// it by a barrier, before its later ones.
+__device__ __forceinline__ void fence_acq_rel_gpu() { asm volatile("fence.acq_rel.gpu;" ::: "memory"); }
+
 __device__ __forceinline__ unsigned long long ld_acquire_u64(const unsigned long long *p) {
     unsigned long long v;
     asm volatile("ld.acquire.gpu.global.u64 %0, [%1];" : "=l"(v) : "l"(p) : "memory");

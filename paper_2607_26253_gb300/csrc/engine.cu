@@ -81,7 +81,8 @@ struct sara_handle {
     int rows_cap16 = 0;
     float *dx = nullptr, *ssqA = nullptr, *ssqM = nullptr;
     uint8_t *xg_hi = nullptr, *xg_lo = nullptr, *att_hi = nullptr, *att_lo = nullptr, *h_hi = nullptr, *h_lo = nullptr;
-    unsigned long long *accQ = nullptr, *accO = nullptr, *accGU = nullptr, *accD = nullptr;
+    float *gpart = nullptr;  // GEMM partial tiles of the decode step
+    int gp_qkv = 0, gp_o = 0;
     unsigned long long *phase_cnt = nullptr;  // [1 + 8 layers + 1] then the epoch
     int n_phase_cnt = 0;
     int pre_cap = 0, att_cap = 0;
@@ -99,8 +100,8 @@ struct sara_handle {
     int32_t *p_tok = nullptr, *p_len = nullptr;
     uint64_t *p_thr = nullptr;
     int32_t *gen_tok = nullptr;
+    float *logit_buf = nullptr;  // [max_seqs][vocab] logits of the decode step's live rows
     // teacher forcing staging (allocated on first use)
-    float *logit_stage = nullptr;
     int32_t *forced = nullptr, *sampled_out = nullptr;
     int64_t *uid_dev = nullptr;
     size_t forced_cap = 0;
@@ -317,7 +318,7 @@ void enqueue_prefill_kernel(sara_handle &h, cudaStream_t s, int which, int l, bo
     }
 }
 
-MegaParams mega_params(const sara_handle &h, float *logits) {
+MegaParams mega_params(const sara_handle &h) {
     const sara_model_cfg &m = h.cfg;
     MegaParams p{};
     p.layers = m.layers;
@@ -361,27 +362,25 @@ MegaParams mega_params(const sara_handle &h, float *logits) {
     p.h_lo = h.h_lo;
     p.ssqA = h.ssqA;
     p.ssqM = h.ssqM;
-    p.accQ = h.accQ;
-    p.accO = h.accO;
-    p.accGU = h.accGU;
-    p.accD = h.accD;
+    p.gpart = h.gpart;
+    p.gp_qkv = h.gp_qkv;
+    p.gp_o = h.gp_o;
     p.part = h.attn_part;
     p.att_cnt = h.attn_cnt;
-    p.logits = logits;
-    p.arg_val = h.lm_val;
-    p.arg_idx = h.lm_idx;
+    p.logits = h.logit_buf;
     p.cnt = h.phase_cnt;
     p.epoch = h.phase_cnt + h.n_phase_cnt;
+    p.stamps = h.stamps;
+    p.n_stamp_ph = h.n_phase_cnt + 1 + 4;  // phases, kernel start, 4 x 4 detail stamps
     return p;
 }
 
 // One decode step over the live rows: the persistent decode-step kernel (embedding, every
-// layer, lm_head with the Gumbel-max partials) followed by the sampling reduction and
-// bookkeeping kernel.
-void enqueue_decode_step(sara_handle &h, cudaStream_t s, float *logits_stage) {
-    launch_ex(s, false, true, dim3(h.sms), dim3(kMegaThreads), kMegaSmemBytes, decode_step_kernel,
-              mega_params(h, logits_stage));
-    launch(s, false, dim3(h.cfg.max_seqs), dim3(256), 0, sample_finish_kernel, h.ptrs);
+// layer, lm_head logits) followed by the Gumbel-max sampling and bookkeeping kernel.
+void enqueue_decode_step(sara_handle &h, cudaStream_t s) {
+    launch_ex(s, false, true, dim3(h.sms), dim3(kMegaThreads), kMegaSmemBytes, decode_step_kernel, mega_params(h));
+    launch(s, false, dim3(h.cfg.max_seqs, kSampleChunks), dim3(256), 0, sample_finish_kernel, h.ptrs,
+           (const float *)h.logit_buf, h.cfg.vocab);
 }
 
 // Prefill of the fresh prompts of a round: embedding, every layer up to the last layer's
@@ -455,7 +454,7 @@ void build_graph(sara_handle &h) {
         enqueue_round_start(h, h.cap_stream2, pdl);
         cudaGraph_t ib2;
         CK(cudaStreamEndCapture(h.cap_stream2, &ib2));
-        enqueue_decode_step(h, cs, nullptr);
+        enqueue_decode_step(h, cs);
     }
     cudaGraph_t b2;
     CK(cudaStreamEndCapture(cs, &b2));
@@ -475,7 +474,7 @@ void run_host_loop(sara_handle &h) {
         if (v.done || v.err) break;
         if (!h.has_model) continue;
         if (v.round_steps == 0 && v.live > 0) enqueue_round_start(h, s, h.use_pdl);
-        enqueue_decode_step(h, s, nullptr);
+        enqueue_decode_step(h, s);
     }
 }
 
@@ -568,7 +567,7 @@ void alloc_acts(sara_handle &h, Acts &A, int rows) {
 }
 
 // Decode-step buffers: residual stream, blocked hi/lo operands (rows padded to 16), the
-// fixed-point projection sums (zero between uses) and the phase counters.
+// GEMM partial tiles and the phase counters.
 void alloc_decode(sara_handle &h) {
     const sara_model_cfg &m = h.cfg;
     const int S = m.max_seqs, d = m.d_model, Hhd = m.n_heads * m.head_dim, F = m.ffn;
@@ -584,26 +583,26 @@ void alloc_decode(sara_handle &h) {
     h.h_lo = h.mem.alloc<uint8_t>(R16 * F * 2);
     h.ssqA = h.mem.alloc<float>((size_t)(d / 128) * S);
     h.ssqM = h.mem.alloc<float>((size_t)(d / 128) * S);
-    h.accQ = h.mem.alloc<unsigned long long>((size_t)S * nqkv);
-    h.accO = h.mem.alloc<unsigned long long>((size_t)S * d);
-    h.accGU = h.mem.alloc<unsigned long long>((size_t)S * 2 * F);
-    h.accD = h.mem.alloc<unsigned long long>((size_t)S * d);
+    // partial tiles: one segment per (CTA, tile) pair of a phase, at most CTAs + tiles - 1
+    const int tmax = std::max({nqkv, d, 2 * F}) / kTileN + 1;
+    h.gpart = h.mem.alloc<float>((size_t)(h.sms + tmax) * S * kTileN, false);
+    // the QKV and O projections are spread over few CTAs (each about one ring of weights)
+    auto small = [&](int N, int K) {
+        const int units = ((N + kTileN - 1) / kTileN) * (K / 64);
+        return std::max(1, std::min(h.sms, units / kSmallPhaseUnits));
+    };
+    h.gp_qkv = small(nqkv, d);
+    h.gp_o = small(d, Hhd);
     h.n_phase_cnt = 1 + kPhasesPerLayer * m.layers + 1;
     h.phase_cnt = h.mem.alloc<unsigned long long>((size_t)h.n_phase_cnt + 1);
 }
 
-// Phase counters and the fixed-point sums back to zero (start of every call: a step that
-// failed part-way may have left them anywhere).
+// Phase counters and split counters back to zero (start of every call: a step that failed
+// part-way may have left them anywhere).
 void reset_decode_state(sara_handle &h, cudaStream_t s) {
     const sara_model_cfg &m = h.cfg;
-    const size_t S = m.max_seqs, d = m.d_model;
-    const size_t nqkv = (size_t)(m.n_heads + 2 * m.n_kv_heads) * m.head_dim;
     CK(cudaMemsetAsync(h.phase_cnt, 0, ((size_t)h.n_phase_cnt + 1) * 8, s));
-    CK(cudaMemsetAsync(h.accQ, 0, S * nqkv * 8, s));
-    CK(cudaMemsetAsync(h.accO, 0, S * d * 8, s));
-    CK(cudaMemsetAsync(h.accGU, 0, S * 2 * m.ffn * 8, s));
-    CK(cudaMemsetAsync(h.accD, 0, S * d * 8, s));
-    CK(cudaMemsetAsync(h.attn_cnt, 0, S * m.n_kv_heads * 4, s));
+    CK(cudaMemsetAsync(h.attn_cnt, 0, (size_t)m.max_seqs * m.n_kv_heads * 4, s));
 }
 
 void make_tensor_maps(sara_handle &h) {
@@ -744,9 +743,10 @@ void create_impl(sara_handle &h, const sara_model_cfg *cfgp, const sara_weights 
         const int Gq = m.n_heads / KVH;
         h.attn_part = h.mem.alloc<float>((size_t)h.att_cap * KVH * Gq * (hd + 2), false);
         h.attn_cnt = h.mem.alloc<int>((size_t)S * KVH);
-        c.lm_tiles = m.vocab / 128;
-        h.lm_val = h.mem.alloc<float>((size_t)S * c.lm_tiles, false);
-        h.lm_idx = h.mem.alloc<int>((size_t)S * c.lm_tiles, false);
+        c.lm_tiles = kSampleChunks;
+        h.lm_val = h.mem.alloc<float>((size_t)S * kSampleChunks, false);
+        h.lm_idx = h.mem.alloc<int>((size_t)S * kSampleChunks, false);
+        h.logit_buf = h.mem.alloc<float>((size_t)S * m.vocab, false);
         c.arg_val = h.lm_val;
         c.arg_idx = h.lm_idx;
         load_weights(h, w);
@@ -877,7 +877,6 @@ void teacher_impl(sara_handle &h, int n, int Lp, const int32_t *prompts, int T, 
     cudaStream_t s = h.stream;
     const cudaMemcpyKind kin = on_device ? cudaMemcpyDeviceToDevice : cudaMemcpyHostToDevice;
     const cudaMemcpyKind kout = on_device ? cudaMemcpyDeviceToDevice : cudaMemcpyDeviceToHost;
-    if (!h.logit_stage) h.logit_stage = h.mem.alloc<float>((size_t)m.max_seqs * m.vocab, false);
     if ((size_t)n * T > h.forced_cap) {
         h.forced_cap = (size_t)n * T;
         h.forced = h.mem.alloc<int32_t>(h.forced_cap, false);
@@ -903,9 +902,9 @@ void teacher_impl(sara_handle &h, int n, int Lp, const int32_t *prompts, int T, 
         enqueue_prefill(h, s, false);
         enqueue_kv_fanout(h, s, false, c);
         for (int step = 0; step < T; ++step) {
-            enqueue_decode_step(h, s, h.logit_stage);
+            enqueue_decode_step(h, s);
             // rows stay in rollout order for all T steps (every rollout has length T)
-            CK(cudaMemcpy2DAsync(logits + (size_t)step * m.vocab, (size_t)T * m.vocab * 4, h.logit_stage,
+            CK(cudaMemcpy2DAsync(logits + (size_t)step * m.vocab, (size_t)T * m.vocab * 4, h.logit_buf,
                                  (size_t)m.vocab * 4, (size_t)m.vocab * 4, n, kout, s));
         }
     } catch (...) {
@@ -920,6 +919,66 @@ void teacher_impl(sara_handle &h, int n, int Lp, const int32_t *prompts, int T, 
     check_step_error(v);
     if (v.live != 0 || v.exec_steps != T) throw SaraError(SARA_EDEVICE, "teacher forcing ran an unexpected number of steps");
 }
+
+#ifdef SARA_STAMPS
+// Phase timeline of the last decode-step launch (profiling builds): for each phase kind,
+// averaged over the middle layers, the time from the previous phase's completion (last CTA
+// arrived) to this one's, the median delay until CTAs observed the dependency, and how far
+// ahead of the previous phase's completion the W producer had issued this phase's copies.
+void print_stamps(sara_handle &h, int rows, int ctx) {
+    const int NP = h.n_phase_cnt + 1 + 4, G = h.sms, L = h.cfg.layers;
+    std::vector<uint64_t> st((size_t)G * NP * 4);
+    CK(cudaMemcpy(st.data(), h.stamps, st.size() * 8, cudaMemcpyDeviceToHost));
+    auto at = [&](int c, int ph, int k) { return st[((size_t)c * NP + ph) * 4 + k]; };
+    uint64_t t0 = ~0ull;
+    for (int c = 0; c < G; ++c) t0 = std::min(t0, at(c, NP - 5, 0));
+    auto stat = [&](int ph, int k, bool mx) {
+        std::vector<double> v;
+        for (int c = 0; c < G; ++c)
+            if (at(c, ph, k) >= t0) v.push_back((double)(at(c, ph, k) - t0) * 1e-3);
+        if (v.empty()) return -1.0;
+        std::sort(v.begin(), v.end());
+        return mx ? v.back() : v[v.size() / 2];
+    };
+    const int NPH = 1 + kPhasesPerLayer * L + 1;
+    std::vector<double> done(NPH);
+    for (int ph = 0; ph < NPH; ++ph) done[ph] = stat(ph, 0, true);
+    fprintf(stderr, "rows %d ctx %d: start->embed done %.2f us, lm_head done at %.2f us\n", rows, ctx, done[0],
+            done[NPH - 1]);
+    const char *names[8] = {"QKV", "ATT", "O", "FIN_O", "GU", "FIN_GU", "DOWN", "FIN_D"};
+    const int l0 = L > 4 ? 2 : 0, l1 = L > 4 ? L - 2 : L;
+    for (int k = 0; k < kPhasesPerLayer; ++k) {
+        double span = 0, obs = 0, wahead = 0, mma = 0;
+        int n = 0;
+        for (int l = l0; l < l1; ++l) {
+            const int ph = 1 + kPhasesPerLayer * l + k;
+            span += done[ph] - done[ph - 1];
+            obs += stat(ph, 1, false) - done[ph - 1];
+            wahead += done[ph - 1] - stat(ph, 2, false);
+            mma += stat(ph, 3, false) - done[ph - 1];
+            ++n;
+        }
+        fprintf(stderr, "  %-6s span %7.2f us  dep seen +%6.2f  W issued %+7.2f before  MMA done +%6.2f\n", names[k],
+                span / n, obs / n, wahead / n, mma / n);
+    }
+    fprintf(stderr, "  LM     span %7.2f us\n", done[NPH - 1] - done[NPH - 2]);
+    // detail stamps (layer 2): median over CTAs relative to the QKV phase's completion
+    const int lq = std::min(2, L - 1);
+    const double ref = done[1 + kPhasesPerLayer * lq];
+    const char *dn[13] = {"att start", "q built", "S ready", "P ready", "O ready", "partial out", "split count",
+                          "merged", "units done", "att arrived", "fin_o start", "fin_o work", "fin_o arrived"};
+    for (int i = 0; i < 13; ++i) {
+        std::vector<double> v;
+        for (int c = 0; c < G; ++c) {
+            const uint64_t x = at(c, NP - 4 + i / 4, i % 4);
+            if (x >= t0) v.push_back((double)(x - t0) * 1e-3 - ref);
+        }
+        std::sort(v.begin(), v.end());
+        if (!v.empty())
+            fprintf(stderr, "    %-14s n=%3zu  med %+7.2f  max %+7.2f us\n", dn[i], v.size(), v[v.size() / 2], v.back());
+    }
+}
+#endif
 
 // Profiling hook: `rows` live rollouts at context `ctx` (synthetic row state), `iters`
 // launches of the whole decode step (kernel 0: decode-step kernel + sampling/bookkeeping,
@@ -967,13 +1026,17 @@ void profile_impl(sara_handle &h, int which, int rows, int ctx, int iters, doubl
     CK(cudaMemcpyAsync(c.seq_gen, zero.data(), rows * 4, cudaMemcpyHostToDevice, s));
     CK(cudaMemcpyAsync(c.seq_len, len.data(), rows * 4, cudaMemcpyHostToDevice, s));
     CK(cudaMemcpyAsync(c.seq_uid, uid.data(), rows * 8, cudaMemcpyHostToDevice, s));
+#ifdef SARA_STAMPS
+    const size_t nst = (size_t)h.sms * (h.n_phase_cnt + 1 + 4) * 4;
+    if (!h.stamps) h.stamps = h.mem.alloc<uint64_t>(nst);
+#endif
     CK(cudaStreamSynchronize(s));
     auto one = [&](cudaStream_t st) {
         if (which == 0) {
-            enqueue_decode_step(h, st, nullptr);
+            enqueue_decode_step(h, st);
         } else {
             launch_ex(st, false, true, dim3(h.sms), dim3(kMegaThreads), kMegaSmemBytes, decode_step_kernel,
-                      mega_params(h, nullptr));
+                      mega_params(h));
         }
     };
     one(s);
@@ -999,6 +1062,9 @@ void profile_impl(sara_handle &h, int which, int rows, int ctx, int iters, doubl
     CK(cudaMemcpy(&v, h.vars, sizeof(v), cudaMemcpyDeviceToHost));
     check_step_error(v);
     *ms = (double)t / iters;
+#ifdef SARA_STAMPS
+    if (which == 1) print_stamps(h, rows, ctx);
+#endif
 }
 
 int guard(sara_handle *h, const std::function<void()> &fn) {

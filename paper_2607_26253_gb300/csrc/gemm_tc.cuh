@@ -51,7 +51,7 @@ struct GemmParams {
     const int *rows_dev;       // device count of valid rows (nullptr -> rows_fixed)
     int rows_fixed;
     int decode;                // 1: a single row tile, weights prefetched before the PDL wait
-    const uint8_t *w_blk;      // non-null: W stored as pre-swizzled 16 KB tiles [Nout/128][K/64] (bulk copies)
+    const uint8_t *w_blk;      // non-null: W stored as pre-swizzled 256-row tiles (bulk copies, wblk128_off)
     int has_lo;                // 1: the activation's lo part (second tensor map) is multiplied too
     unsigned long long *ws_acc;  // [gridDim.x][kTileR * kTileM] fixed-point tile sums, zero between launches
     int *ws_cnt;               // [tiles] arrival counters, zero between launches
@@ -116,6 +116,15 @@ __device__ __forceinline__ int cta_of_unit(int64_t u, int64_t U, int G) {
 #define GEMM_STAMP(i) do { } while (0)
 #endif
 __device__ __forceinline__ int64_t min64(int64_t a, int64_t b) { return a < b ? a : b; }
+
+// Byte offset of the 128 x 64 weight sub-tile (m_tile, kc) of a weight [Nout][K] stored as
+// pre-swizzled tiles of 256 rows (the last may have 128): tile t = m_tile / 2 holds, for
+// each k-chunk, its rows at a 128-byte pitch, so the two 128-row halves are 16 KB apart.
+__device__ __forceinline__ int64_t wblk128_off(int Nout, int K, int m_tile, int kc) {
+    const int t = m_tile >> 1;
+    const int rows = min(256, Nout - 256 * t);
+    return (int64_t)t * 256 * K * 2 + (int64_t)kc * rows * 128 + (m_tile & 1) * 16384;
+}
 
 
 template <int EPI>
@@ -306,7 +315,7 @@ gemm_tc_kernel(const __grid_constant__ CUtensorMap tmW, const __grid_constant__ 
                     const int m_tile = tile % m_tiles;
                     mbar_expect_tx(&S.full[i], (uint32_t)kWStageBytes);
                     if (p.w_blk)
-                        bulk_load(sW + i * kWStageBytes, p.w_blk + ((int64_t)m_tile * kch + kc) * kWStageBytes,
+                        bulk_load(sW + i * kWStageBytes, p.w_blk + wblk128_off(m_tiles * kTileM, kch * kTileK, m_tile, kc),
                                   kWStageBytes, &S.full[i], l2_policy_evict_first());
                     else
                         tma_load_2d(sW + i * kWStageBytes, &tmW, &S.full[i], kc * kTileK, m_tile * kTileM,
@@ -333,8 +342,9 @@ gemm_tc_kernel(const __grid_constant__ CUtensorMap tmW, const __grid_constant__ 
                 if (i >= n_pre) {
                     mbar_arrive_expect_tx(&S.full[s], (uint32_t)kWStageBytes + xbytes);
                     if (p.w_blk)
-                        bulk_load(sW + (size_t)s * kWStageBytes, p.w_blk + ((int64_t)m_tile * kch + kc) * kWStageBytes,
-                                  kWStageBytes, &S.full[s], pol_w);
+                        bulk_load(sW + (size_t)s * kWStageBytes,
+                                  p.w_blk + wblk128_off(m_tiles * kTileM, kch * kTileK, m_tile, kc), kWStageBytes,
+                                  &S.full[s], pol_w);
                     else
                         tma_load_2d(sW + (size_t)s * kWStageBytes, &tmW, &S.full[s], kc * kTileK, m_tile * kTileM,
                                     pol_w);

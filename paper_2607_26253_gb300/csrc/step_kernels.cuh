@@ -63,11 +63,15 @@ __device__ __forceinline__ int scan256(int v, int &total, int *warp_tot) {
     return before + x - v;
 }
 
-// Sampling reduction + step bookkeeping.  CTA r < live reduces row r's lm_head partial
-// argmax over the vocabulary tiles (ties: lowest token id).  The last CTA to finish then
-// appends each row's token to its rollout, retires rollouts that reached their length,
-// compacts the live rows (order kept) and writes the next step's rows and attention items.
-static __global__ void __launch_bounds__(256) sample_finish_kernel(StepPtrs c) {
+constexpr int kSampleChunks = 8;  // vocabulary chunks per row (one CTA each)
+
+// Gumbel-max sampling + step bookkeeping.  CTA (r, ch), r < live, draws the Gumbel noise of
+// tokens [ch * V / 8, ..) of row r from the row's sampler key, adds it to the logits and
+// keeps the argmax (ties: lowest token id).  The last CTA to finish reduces each row's
+// chunk partials, then appends each row's token to its rollout, retires rollouts that
+// reached their length, compacts the live rows (order kept) and writes the next step's rows
+// and attention items.
+static __global__ void __launch_bounds__(256) sample_finish_kernel(StepPtrs c, const float *logits, int vocab) {
     __shared__ float sv[8];
     __shared__ int si[8];
     __shared__ int s_last;
@@ -76,15 +80,23 @@ static __global__ void __launch_bounds__(256) sample_finish_kernel(StepPtrs c) {
     pdl_allow_dependents();
     StepVars &V = *c.v;
     const int live = V.live;
-    const int r = blockIdx.x;
+    const int r = blockIdx.x, ch = blockIdx.y;
     const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
     if (r < live) {
+        const int chunk = ((vocab + kSampleChunks - 1) / kSampleChunks + 3) & ~3;
+        const int n0 = ch * chunk, n1 = min(vocab, n0 + chunk);
+        const uint64_t seed = c.row_seed[r];
+        const float *lr = logits + (int64_t)r * vocab;
         float best = -INFINITY;
         int bi = 0x7fffffff;
-        for (int t = tid; t < c.lm_tiles; t += blockDim.x) {
-            const float v = __ldcg(&c.arg_val[(int64_t)r * c.lm_tiles + t]);
-            const int i = __ldcg(&c.arg_idx[(int64_t)r * c.lm_tiles + t]);
-            if (v > best || (v == best && i < bi)) { best = v; bi = i; }
+        for (int n = n0 + 4 * tid; n < n1; n += 4 * blockDim.x) {
+            const float4 l4 = __ldcg(reinterpret_cast<const float4 *>(lr + n));
+            const float l[4] = {l4.x, l4.y, l4.z, l4.w};
+#pragma unroll
+            for (int e = 0; e < 4; ++e) {
+                const float z = l[e] + gumbel_from_hash(splitmix_at(seed, (uint64_t)(n + e) + 1));
+                if (z > best) { best = z; bi = n + e; }
+            }
         }
 #pragma unroll
         for (int o = 16; o > 0; o >>= 1) {
@@ -97,20 +109,32 @@ static __global__ void __launch_bounds__(256) sample_finish_kernel(StepPtrs c) {
         if (tid == 0) {
             for (int w = 1; w < 8; ++w)
                 if (sv[w] > best || (sv[w] == best && si[w] < bi)) { best = sv[w]; bi = si[w]; }
-            c.sampled[r] = bi;
+            c.arg_val[(int64_t)r * kSampleChunks + ch] = best;
+            c.arg_idx[(int64_t)r * kSampleChunks + ch] = bi;
         }
     }
     __threadfence();
     __syncthreads();
     if (tid == 0) {
         const int old = atomicAdd(&V.fin_count, 1);
-        s_last = (old == (int)gridDim.x - 1);
+        s_last = (old == (int)(gridDim.x * gridDim.y) - 1);
     }
     __syncthreads();
     if (!s_last) return;
     __threadfence();
     if (tid == 0) V.fin_count = 0;
     if (live == 0) return;
+    for (int i = tid; i < live; i += blockDim.x) {  // each row's token: argmax over its chunks
+        float best = __ldcg(&c.arg_val[(int64_t)i * kSampleChunks]);
+        int bi = __ldcg(&c.arg_idx[(int64_t)i * kSampleChunks]);
+        for (int q = 1; q < kSampleChunks; ++q) {
+            const float v = __ldcg(&c.arg_val[(int64_t)i * kSampleChunks + q]);
+            const int id = __ldcg(&c.arg_idx[(int64_t)i * kSampleChunks + q]);
+            if (v > best || (v == best && id < bi)) { best = v; bi = id; }
+        }
+        c.sampled[i] = bi;
+    }
+    __syncthreads();
     const StepConst &K = *c.kc;
     const int Lp = K.Lp;
     // bookkeeping over the live rows (several passes of 256)

@@ -74,9 +74,9 @@ struct StepPtrs {
     // teacher forcing
     const int32_t *forced;     // [n][T]
     int32_t *sampled_out;      // [n][T]
-    // lm_head partial argmax
-    const float *arg_val;
-    const int32_t *arg_idx;
+    // sampling partial argmax per (row, vocabulary chunk)
+    float *arg_val;
+    int32_t *arg_idx;
     int32_t lm_tiles;
     int32_t max_seqs, max_active, pre_cap, att_cap;
 };
