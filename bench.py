@@ -38,7 +38,7 @@ FALLBACK_HBM_GBS = 6800.0
 def parse():
     ap = argparse.ArgumentParser()
     ap.add_argument("--gpus", type=int, default=1)
-    ap.add_argument("--steps", type=int, default=3)
+    ap.add_argument("--steps", type=int, default=1)
     ap.add_argument("--warmup", type=int, default=3)
     ap.add_argument("--impl", default="mine", choices=["mine", "reference"])
     ap.add_argument("--workload", default="1.5b", choices=sorted(synth.WORKLOADS))
@@ -179,6 +179,7 @@ def run_mine(args):
     import torch.distributed as dist
 
     import paper_2607_26253_gb300 as pkg
+    from paper_2607_26253_gb300 import replicas
 
     world = int(os.environ.get("WORLD_SIZE", "1"))
     rank = int(os.environ.get("RANK", "0"))
@@ -190,7 +191,7 @@ def run_mine(args):
 
     w0 = synth.WORKLOADS[args.workload]
     m = w0.model
-    w = w0.with_seed_offset(1000 * rank) if rank else w0  # each replica its own prompt-stream shard
+    w = w0.with_seed_offset(replicas.seed_offset(rank))  # each replica its own prompt-stream shard
     weights = synth.model_weights(m, w.weight_seed)
     cfg = pkg.model_cfg(m, max_prompts=w.n_prompts, max_active=w.target_B, max_seqs=w.target_B * w.n0,
                         max_prompt_len=w.prompt_len, max_gen_len=w.lengths.max_len, max_k=w.k)
@@ -285,13 +286,10 @@ def run_mine(args):
     h.close()
 
     # ------------------------------------------------------------------ reduce over ranks
-    if world > 1:
-        t = torch.tensor([ms, e2e_ms], dtype=torch.float64, device=dev)
-        dist.all_reduce(t, op=dist.ReduceOp.MAX)
-        ms, e2e_ms = t.tolist()
-        s = torch.tensor([tok, groups, rollouts, e2e_tok, dec_bytes, h2d, d2h], dtype=torch.float64, device=dev)
-        dist.all_reduce(s, op=dist.ReduceOp.SUM)
-        tok, groups, rollouts, e2e_tok, dec_bytes, h2d, d2h = s.tolist()
+    if world > 1:  # the only collective: job totals (sum) over the slowest rank's time (max)
+        ms, e2e_ms = replicas.reduce_max([ms, e2e_ms], device=dev)
+        tok, groups, rollouts, e2e_tok, dec_bytes, h2d, d2h = replicas.reduce_sum(
+            [tok, groups, rollouts, e2e_tok, dec_bytes, h2d, d2h], device=dev)
     if rank != 0:
         if world > 1:
             dist.destroy_process_group()

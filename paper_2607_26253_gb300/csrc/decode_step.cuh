@@ -64,6 +64,7 @@ constexpr int kKVBlockBytes = 65536;  // K 2 x 16 KB + V^T 2 x 16 KB
 constexpr int kMegaMaxSplits = 96;
 constexpr int kPhasesPerLayer = 8;
 constexpr int kSmallPhaseUnits = 4;   // QKV / O: units per participating CTA (the ring's depth)
+constexpr int kCntStride = 16;        // phase counters 128 bytes apart (one L2 line each)
 constexpr uint32_t kTmemCols = 512;
 constexpr uint32_t kTmemS = 256;  // attention scores, 2 buffers x 16 columns
 constexpr uint32_t kTmemO = 288;  // attention output, 2 buffers x 16 columns
@@ -92,7 +93,7 @@ struct MegaParams {
     float *part;                                    // [items][KVH][Gq][hd + 2] attention split partials
     int *att_cnt;                                   // [rows_cap][KVH] split arrival counters
     float *logits;                                  // [rows_cap][V] fp32 (read by the sampling kernel)
-    unsigned long long *cnt;                        // phase arrival counters (monotonic)
+    unsigned long long *cnt;                        // phase arrival counters (monotonic), kCntStride apart
     unsigned long long *epoch;                      // launches completed since the reset
     uint64_t *stamps;                               // profiling builds: [cta][phase + 1][4] timestamps
     int n_stamp_ph;
@@ -182,8 +183,8 @@ __device__ __forceinline__ bool mwait(uint64_t *bar, uint32_t parity, int *err, 
     }
 }
 
-// Spin until a phase counter reaches `target` (acquire); bounded, gives up on abort or once
-// another CTA reported a timeout.
+// Spin until a phase counter reaches `target` (acquire loads);
+// bounded, gives up on abort or once another CTA reported a timeout.
 __device__ __forceinline__ bool spin_counter(const unsigned long long *cnt, unsigned long long target, int *err,
                                              volatile int *abort) {
     if (ld_acquire_u64(cnt) >= target) return true;
@@ -378,7 +379,7 @@ __device__ __forceinline__ void mega_x_producer(const MegaParams &p, MegaSmem &S
             if (u0 >= u1) continue;
             // the phase this operand comes from: FIN_D of l-1 / embedding, ATT, FIN_O, FIN_GU
             const int dep = (l == p.layers || k == 0) ? kPhasesPerLayer * l : 1 + kPhasesPerLayer * l + k - 1;
-            if (!spin_counter(&p.cnt[dep], S.target, err, ab)) { ok = false; break; }
+            if (!spin_counter(&p.cnt[dep * kCntStride], S.target, err, ab)) { ok = false; break; }
             MEGA_STAMP(1 + kPhasesPerLayer * l + k, 1);
             fence_proxy_async_global();
             for (int64_t u = u0; u < u1; ++u, ++xi) {
@@ -524,17 +525,25 @@ __device__ __forceinline__ void head_granule(const MegaParams &p, const GemmPh &
     float x[8], xp[8];
 #pragma unroll
     for (int e = 0; e < 8; ++e) x[e] = xp[e] = 0.f;
-#pragma unroll 4
-    for (int c = ca; c <= cb; ++c) {
-        const float *base = p.gpart + ((int64_t)(c + t) * p.rows_cap + r) * kTileN;
-        const float4 a = __ldcg(reinterpret_cast<const float4 *>(base + col));
-        const float4 b = __ldcg(reinterpret_cast<const float4 *>(base + col + 4));
-        const float4 pa = rot ? __ldcg(reinterpret_cast<const float4 *>(base + pcol)) : make_float4(0.f, 0.f, 0.f, 0.f);
-        const float4 pb = rot ? __ldcg(reinterpret_cast<const float4 *>(base + pcol + 4)) : make_float4(0.f, 0.f, 0.f, 0.f);
-        x[0] += a.x; x[1] += a.y; x[2] += a.z; x[3] += a.w;
-        x[4] += b.x; x[5] += b.y; x[6] += b.z; x[7] += b.w;
-        xp[0] += pa.x; xp[1] += pa.y; xp[2] += pa.z; xp[3] += pa.w;
-        xp[4] += pb.x; xp[5] += pb.y; xp[6] += pb.z; xp[7] += pb.w;
+    const float4 z4 = make_float4(0.f, 0.f, 0.f, 0.f);
+    for (int c0 = ca; c0 <= cb; c0 += 7) {  // 7 contributors' loads in flight, summed in CTA order
+        float4 a[7], b[7], pa[7], pb[7];
+#pragma unroll
+        for (int k = 0; k < 7; ++k) {
+            const bool ok = c0 + k <= cb;
+            const float *base = p.gpart + ((int64_t)(c0 + k + t) * p.rows_cap + r) * kTileN;
+            a[k] = ok ? __ldcg(reinterpret_cast<const float4 *>(base + col)) : z4;
+            b[k] = ok ? __ldcg(reinterpret_cast<const float4 *>(base + col + 4)) : z4;
+            pa[k] = (ok && rot) ? __ldcg(reinterpret_cast<const float4 *>(base + pcol)) : z4;
+            pb[k] = (ok && rot) ? __ldcg(reinterpret_cast<const float4 *>(base + pcol + 4)) : z4;
+        }
+#pragma unroll
+        for (int k = 0; k < 7; ++k) {
+            x[0] += a[k].x; x[1] += a[k].y; x[2] += a[k].z; x[3] += a[k].w;
+            x[4] += b[k].x; x[5] += b[k].y; x[6] += b[k].z; x[7] += b[k].w;
+            xp[0] += pa[k].x; xp[1] += pa[k].y; xp[2] += pa[k].z; xp[3] += pa[k].w;
+            xp[4] += pb[k].x; xp[5] += pb[k].y; xp[6] += pb[k].z; xp[7] += pb[k].w;
+        }
     }
     if (!rot) {
 #pragma unroll
@@ -582,21 +591,24 @@ __device__ __forceinline__ void mega_compute(const MegaParams &p, MegaSmem &S, u
         if (ctid == 0) {
             fence_acq_rel_gpu();
             MEGA_STAMP(idx, 0);
-            atomicAdd(&p.cnt[idx], 1ull);
+            atomicAdd(&p.cnt[idx * kCntStride], 1ull);
         }
     };
     auto wait_phase = [&](int idx) {
         if (ctid == 0) {
-            spin_counter(&p.cnt[idx], S.target, err, ab);
+            spin_counter(&p.cnt[idx * kCntStride], S.target, err, ab);
             MEGA_STAMP(idx + 1, 1);
         }
         named_bar_sync(1, kMegaCThreads);
     };
     auto load_rstd = [&](const float *ssq) {
-        if (ctid < R) {
+        if (ctid < R) {  // every partial load in flight at once (d <= 2048: at most 16)
+            float v[16];
+#pragma unroll
+            for (int t = 0; t < 16; ++t) v[t] = t < dt ? __ldcg(&ssq[(int64_t)t * p.rows_cap + ctid]) : 0.f;
             float s = 0.f;
-#pragma unroll 16
-            for (int t = 0; t < dt; ++t) s += __ldcg(&ssq[(int64_t)t * p.rows_cap + ctid]);
+#pragma unroll
+            for (int t = 0; t < 16; ++t) s += v[t];
             S.rstd[ctid] = rsqrtf(s / (float)d + p.eps);
         }
         named_bar_sync(1, kMegaCThreads);
@@ -640,11 +652,17 @@ __device__ __forceinline__ void mega_compute(const MegaParams &p, MegaSmem &S, u
                 int ca, cb;
                 tile_ctas(*g, gt, ca, cb);
                 float4 s = make_float4(0.f, 0.f, 0.f, 0.f);
-#pragma unroll 8
-                for (int c = ca; c <= cb; ++c) {
-                    const float4 v = __ldcg(reinterpret_cast<const float4 *>(
-                        p.gpart + ((int64_t)(c + gt) * p.rows_cap + r) * kTileN + col));
-                    s.x += v.x; s.y += v.y; s.z += v.z; s.w += v.w;
+                for (int c0 = ca; c0 <= cb; c0 += 16) {  // 16 contributors' loads in flight, summed in CTA order
+                    float4 v[16];
+#pragma unroll
+                    for (int k = 0; k < 16; ++k)
+                        v[k] = c0 + k <= cb ? __ldcg(reinterpret_cast<const float4 *>(
+                                                  p.gpart + ((int64_t)(c0 + k + gt) * p.rows_cap + r) * kTileN + col))
+                                            : make_float4(0.f, 0.f, 0.f, 0.f);
+#pragma unroll
+                    for (int k = 0; k < 16; ++k) {
+                        s.x += v[k].x; s.y += v[k].y; s.z += v[k].z; s.w += v[k].w;
+                    }
                 }
                 x.x += s.x; x.y += s.y; x.z += s.z; x.w += s.w;
                 *reinterpret_cast<float4 *>(p.x + (int64_t)r * d + f) = x;
@@ -698,12 +716,14 @@ __device__ __forceinline__ void mega_compute(const MegaParams &p, MegaSmem &S, u
         // ------------------------------------------------------------ attention
         {
             wait_phase(base + 0);
+            const bool det_layer = l == min(2, p.layers - 1);
+            if (det_layer && ctid == 0) MEGA_DETAIL(13);
             load_rstd(p.ssqA);
+            if (det_layer && ctid == 0) MEGA_DETAIL(14);
             int64_t a0, a1;
             att_range(p, S.n_items, a0, a1);
             const int n = (int)(a1 - a0);
             const uint32_t wb = wi;
-            const bool det_layer = l == min(2, p.layers - 1);
 #define DETAIL(i)                                       \
     do {                                                \
         if (det_layer && ctid == 0 && i_unit == 0) MEGA_DETAIL(i); \
@@ -934,33 +954,57 @@ __device__ __forceinline__ void mega_compute(const MegaParams &p, MegaSmem &S, u
             wait_phase(base + 4);
             load_rstd(p.ssqM);
             const int fb = p.F / 128;
-            for (int u = gw; u < R * fb; u += nw) {
-                const int r = u / fb, t = u - r * fb;
-                const float rs = S.rstd[r];
-                // h features 128 t + 4 lane .. +3: gate at tile column c, up at c + 64, with
-                // c = 4 lane (features < 64 of the tile) or 128 + 4 lane - 64 (the rest)
-                const int c0 = (lane < 16) ? 4 * lane : 128 + 4 * lane - 64;
-                int ca, cb;
-                tile_ctas(gu, t, ca, cb);
-                float4 gs = make_float4(0.f, 0.f, 0.f, 0.f), us = gs;
-#pragma unroll 4
-                for (int c = ca; c <= cb; ++c) {
-                    const float *src = p.gpart + ((int64_t)(c + t) * p.rows_cap + r) * kTileN + c0;
-                    const float4 a = __ldcg(reinterpret_cast<const float4 *>(src));
-                    const float4 bq = __ldcg(reinterpret_cast<const float4 *>(src + 64));
-                    gs.x += a.x; gs.y += a.y; gs.z += a.z; gs.w += a.w;
-                    us.x += bq.x; us.y += bq.y; us.z += bq.z; us.w += bq.w;
-                }
-                const float gv[4] = {gs.x * rs, gs.y * rs, gs.z * rs, gs.w * rs};
-                const float uv[4] = {us.x * rs, us.y * rs, us.z * rs, us.w * rs};
-                uint16_t hh[4], hl[4];
+            // unit = (row, 128 features of h) = one 256-row tile of the gate/up outputs; lane:
+            // 4 features, gate at tile column c, up at c + 64 (c = 4 lane, or 128 + 4 lane - 64
+            // for the tile's second 64 features).  A warp takes two units per pass with every
+            // partial load in flight before the sums (in CTA order).
+            const int c0 = (lane < 16) ? 4 * lane : 128 + 4 * lane - 64;
+            for (int u = gw; u < R * fb; u += 2 * nw) {
+                float4 gs[2], us[2];
+                int rr[2], tt[2];
 #pragma unroll
-                for (int e = 0; e < 4; ++e) split_bf16(gv[e] / (1.0f + expf(-gv[e])) * uv[e], hh[e], hl[e]);
-                const int64_t off = xblk_off(r, t * 128 + 4 * lane, R16c);
-                *reinterpret_cast<uint2 *>(p.h_hi + off) =
-                    make_uint2((uint32_t)hh[0] | ((uint32_t)hh[1] << 16), (uint32_t)hh[2] | ((uint32_t)hh[3] << 16));
-                *reinterpret_cast<uint2 *>(p.h_lo + off) =
-                    make_uint2((uint32_t)hl[0] | ((uint32_t)hl[1] << 16), (uint32_t)hl[2] | ((uint32_t)hl[3] << 16));
+                for (int q = 0; q < 2; ++q) {
+                    const int uq = u + q * nw;
+                    gs[q] = us[q] = make_float4(0.f, 0.f, 0.f, 0.f);
+                    rr[q] = -1;
+                    tt[q] = 0;
+                    if (uq >= R * fb) continue;
+                    const int r = uq / fb, t = uq - r * fb;
+                    rr[q] = r;
+                    tt[q] = t;
+                    int ca, cb;
+                    tile_ctas(gu, t, ca, cb);
+                    for (int cq = ca; cq <= cb; cq += 4) {
+                        float4 a4[4], b4[4];
+#pragma unroll
+                        for (int k = 0; k < 4; ++k) {
+                            const bool ok = cq + k <= cb;
+                            const float *src = p.gpart + ((int64_t)(cq + k + t) * p.rows_cap + r) * kTileN + c0;
+                            a4[k] = ok ? __ldcg(reinterpret_cast<const float4 *>(src)) : make_float4(0.f, 0.f, 0.f, 0.f);
+                            b4[k] = ok ? __ldcg(reinterpret_cast<const float4 *>(src + 64)) : make_float4(0.f, 0.f, 0.f, 0.f);
+                        }
+#pragma unroll
+                        for (int k = 0; k < 4; ++k) {
+                            gs[q].x += a4[k].x; gs[q].y += a4[k].y; gs[q].z += a4[k].z; gs[q].w += a4[k].w;
+                            us[q].x += b4[k].x; us[q].y += b4[k].y; us[q].z += b4[k].z; us[q].w += b4[k].w;
+                        }
+                    }
+                }
+#pragma unroll
+                for (int q = 0; q < 2; ++q) {
+                    if (rr[q] < 0) continue;
+                    const float rs = S.rstd[rr[q]];
+                    const float gv[4] = {gs[q].x * rs, gs[q].y * rs, gs[q].z * rs, gs[q].w * rs};
+                    const float uv[4] = {us[q].x * rs, us[q].y * rs, us[q].z * rs, us[q].w * rs};
+                    uint16_t hh[4], hl[4];
+#pragma unroll
+                    for (int e = 0; e < 4; ++e) split_bf16(gv[e] / (1.0f + expf(-gv[e])) * uv[e], hh[e], hl[e]);
+                    const int64_t off = xblk_off(rr[q], tt[q] * 128 + 4 * lane, R16c);
+                    *reinterpret_cast<uint2 *>(p.h_hi + off) =
+                        make_uint2((uint32_t)hh[0] | ((uint32_t)hh[1] << 16), (uint32_t)hh[2] | ((uint32_t)hh[3] << 16));
+                    *reinterpret_cast<uint2 *>(p.h_lo + off) =
+                        make_uint2((uint32_t)hl[0] | ((uint32_t)hl[1] << 16), (uint32_t)hl[2] | ((uint32_t)hl[3] << 16));
+                }
             }
             arrive(base + 5);
         }

@@ -369,7 +369,7 @@ MegaParams mega_params(const sara_handle &h) {
     p.att_cnt = h.attn_cnt;
     p.logits = h.logit_buf;
     p.cnt = h.phase_cnt;
-    p.epoch = h.phase_cnt + h.n_phase_cnt;
+    p.epoch = h.phase_cnt + (size_t)h.n_phase_cnt * kCntStride;
     p.stamps = h.stamps;
     p.n_stamp_ph = h.n_phase_cnt + 1 + 4;  // phases, kernel start, 4 x 4 detail stamps
     return p;
@@ -594,14 +594,14 @@ void alloc_decode(sara_handle &h) {
     h.gp_qkv = small(nqkv, d);
     h.gp_o = small(d, Hhd);
     h.n_phase_cnt = 1 + kPhasesPerLayer * m.layers + 1;
-    h.phase_cnt = h.mem.alloc<unsigned long long>((size_t)h.n_phase_cnt + 1);
+    h.phase_cnt = h.mem.alloc<unsigned long long>(((size_t)h.n_phase_cnt + 1) * kCntStride);
 }
 
 // Phase counters and split counters back to zero (start of every call: a step that failed
 // part-way may have left them anywhere).
 void reset_decode_state(sara_handle &h, cudaStream_t s) {
     const sara_model_cfg &m = h.cfg;
-    CK(cudaMemsetAsync(h.phase_cnt, 0, ((size_t)h.n_phase_cnt + 1) * 8, s));
+    CK(cudaMemsetAsync(h.phase_cnt, 0, ((size_t)h.n_phase_cnt + 1) * kCntStride * 8, s));
     CK(cudaMemsetAsync(h.attn_cnt, 0, (size_t)m.max_seqs * m.n_kv_heads * 4, s));
 }
 
@@ -623,7 +623,7 @@ void validate_cfg(const sara_model_cfg &m) {
     if (m.max_active > 8192) bad("max_active must be <= 8192");
     if (m.layers < 0) bad("layers < 0");
     if (m.layers == 0) return;
-    if (m.d_model % 128 || m.d_model < 128) bad("d_model must be a positive multiple of 128");
+    if (m.d_model % 128 || m.d_model < 128 || m.d_model > 2048) bad("d_model must be a multiple of 128 in [128, 2048]");
     if (m.head_dim != 32 && m.head_dim != 64 && m.head_dim != 128) bad("head_dim must be 32, 64 or 128");
     if (m.n_kv_heads < 1 || m.n_heads % m.n_kv_heads)
         bad("n_heads must be a multiple of n_kv_heads");
@@ -965,9 +965,10 @@ void print_stamps(sara_handle &h, int rows, int ctx) {
     // detail stamps (layer 2): median over CTAs relative to the QKV phase's completion
     const int lq = std::min(2, L - 1);
     const double ref = done[1 + kPhasesPerLayer * lq];
-    const char *dn[13] = {"att start", "q built", "S ready", "P ready", "O ready", "partial out", "split count",
-                          "merged", "units done", "att arrived", "fin_o start", "fin_o work", "fin_o arrived"};
-    for (int i = 0; i < 13; ++i) {
+    const char *dn[15] = {"att start", "q built", "S ready", "P ready", "O ready", "partial out", "split count",
+                          "merged", "units done", "att arrived", "fin_o start", "fin_o work", "fin_o arrived",
+                          "att dep seen", "att rstd"};
+    for (int i = 0; i < 15; ++i) {
         std::vector<double> v;
         for (int c = 0; c < G; ++c) {
             const uint64_t x = at(c, NP - 4 + i / 4, i % 4);
