@@ -297,7 +297,10 @@ def run_mine(args):
 
     peak, peak_kind = peaks()
     achieved = k_bytes / (k_ms * 1e-3) / 1e9
-    traffic = read_traffic(args.workload)
+    # DRAM traffic of the capture, scaled to this launch by its algorithmic bytes (weights are
+    # the same; KV grows with rows x context, which the capture read exactly once as well)
+    tr = read_traffic(args.workload)
+    traffic = None if tr is None else tr[0] * k_bytes / tr[1]
     cpu = None
     if not args.no_cpu_baseline:
         rate, secs, desc = cpu_oracle_sample(w0, weights)
@@ -327,6 +330,7 @@ def run_mine(args):
         "decode_kernel_ms": k_ms,
         "roofline": {"bound": "hbm", "achieved": achieved, "peak": peak, "unit": "GB/s",
                      "frac": achieved / peak, "traffic": traffic,
+                     "traffic_note": None if tr is None else "ncu capture at 25 rows, context 384, scaled by algorithmic bytes",
                      "kernel": f"decode_step_kernel (whole forward), {mean_rows} live rows at context {mid_ctx}",
                      "bytes_per_launch": k_bytes,
                      "peak_kind": f"{peak_kind} burst copy"},
@@ -347,15 +351,20 @@ def run_mine(args):
 
 
 def read_traffic(workload: str):
-    """DRAM bytes per launch of the dominant kernel from the committed ncu summary, if any."""
+    """(DRAM bytes, algorithmic bytes) of one launch of the dominant kernel from the committed
+    ncu summary, or None."""
     path = os.path.join(ROOT, "profiles", f"decode_step_{workload.replace('.', 'p')}_ncu.md")
+    got = {}
     try:
         for line in open(path):
-            if line.startswith("traffic_bytes_per_launch:"):
-                return float(line.split(":", 1)[1].split()[0])
+            for key in ("traffic_bytes_per_launch:", "algorithmic_bytes_per_launch:"):
+                if line.startswith(key):
+                    got[key] = float(line.split(":", 1)[1].split()[0])
     except OSError:
-        pass
-    return None
+        return None
+    if len(got) != 2:
+        return None
+    return got["traffic_bytes_per_launch:"], got["algorithmic_bytes_per_launch:"]
 
 
 # --------------------------------------------------------------------------------- ncu mode
