@@ -63,7 +63,7 @@ constexpr int kKVPos = 128;           // positions per KV block and per attentio
 constexpr int kKVBlockBytes = 65536;  // K 2 x 16 KB + V^T 2 x 16 KB
 constexpr int kMegaMaxSplits = 96;
 constexpr int kPhasesPerLayer = 8;
-constexpr int kSmallPhaseUnits = 4;   // QKV / O: units per participating CTA (the ring's depth)
+constexpr int kSmallPhaseUnits = 2;   // QKV / O: units per participating CTA
 constexpr int kCntStride = 16;        // phase counters 128 bytes apart (one L2 line each)
 constexpr uint32_t kTmemCols = 512;
 constexpr uint32_t kTmemS = 256;  // attention scores, 2 buffers x 16 columns
@@ -137,9 +137,10 @@ struct MegaSmem {
     int rows, rows16, nx, n_items;
     float rstd[128];
     float att_m[2][8], att_l[2][8];
-    float red[4][8], red2[4][8];
-    float mw[8][kMegaMaxSplits];
-    float ml[8];
+    float red[2][4][8], red2[2][4][8];  // per warp group: attention max / sum reductions
+    float mw[2][8][kMegaMaxSplits];      // per warp group: split weights of a merge
+    float ml[2][8];
+    int last_flag2[2];
 };
 
 constexpr size_t kMegaSmemBytes =
@@ -281,15 +282,15 @@ __device__ __forceinline__ AttUnit att_unit(const MegaParams &p, int64_t a) {
     AttUnit u;
     u.item = (int)(a / p.KVH);
     u.kvh = (int)(a - (int64_t)u.item * p.KVH);
-    const int2 it = p.c.att_items[u.item];
+    const int2 it = __ldg(&p.c.att_items[u.item]);
     u.row = it.x;
     u.sp = it.y;
-    u.ctx = p.c.row_pos[u.row] + 1;
+    u.ctx = __ldg(&p.c.row_pos[u.row]) + 1;
     u.p0 = u.sp * kKVPos;
     u.n = min(u.ctx - u.p0, kKVPos);
     u.nsplit = (u.ctx + kKVPos - 1) / kKVPos;
     u.last = u.p0 + u.n == u.ctx;
-    u.slot = p.c.row_slot[u.row];
+    u.slot = __ldg(&p.c.row_slot[u.row]);
     return u;
 }
 __device__ __forceinline__ void att_range(const MegaParams &p, int n_items, int64_t &a0, int64_t &a1) {
@@ -446,36 +447,41 @@ __device__ __forceinline__ void mega_mma(const MegaParams &p, MegaSmem &S, uint8
             if (g.whole) ++lmseg;
         }
     };
+    // attention units in pairs (one per compute warp group): S(i), S(i+1), PV(i), PV(i+1)
     auto att = [&](int64_t a0, int64_t a1) {
         const int n = (int)(a1 - a0);
         const uint32_t wb = wi;
-        for (int i = 0; i <= n && ok; ++i) {
-            if (i < n) {  // scores S = K q^T of unit i
-                const int g = gi + i, b = g & 1;
-                const uint32_t w0 = wb + 2 * i;
-                if (!mwait(&S.q_ready[b], (g >> 1) & 1, err, ab) || !wwait(w0)) { ok = false; break; }
-                tc_fence_after();
-                const uint32_t dS = tmem + kTmemS + 16 * b, qb = smem_u32(sQ + 4096 * b), kb = wslot(w0);
-                for (int ks = 0; ks < p.hd / 16; ++ks)
-                    tc_mma_bf16(dS, sdesc_kmajor_sw128(kb + (ks >> 2) * 16384 + (ks & 3) * 32),
-                                sdesc_kmajor_sw128(qb + (ks >> 2) * 2048 + (ks & 3) * 32), ida, ks > 0 ? 1u : 0u);
-                tc_commit(&S.s_full[b]);
-                tc_commit(&S.wempty[w0 % kWSlots]);
-            }
-            if (i >= 1) {  // output O^T = V^T P^T of unit i - 1
-                const int g = gi + i - 1, b = g & 1;
-                const uint32_t w1 = wb + 2 * (i - 1) + 1;
-                const AttUnit u = att_unit(p, a0 + i - 1);
-                if (!mwait(&S.p_ready[b], (g >> 1) & 1, err, ab) || !wwait(w1)) { ok = false; break; }
-                tc_fence_after();
-                const uint32_t dO = tmem + kTmemO + 16 * b, pb = smem_u32(sP + 4096 * b), vb = wslot(w1);
-                const int ksteps = (u.n + 15) >> 4;
-                for (int ks = 0; ks < ksteps; ++ks)
-                    tc_mma_bf16(dO, sdesc_kmajor_sw128(vb + (ks >> 2) * 16384 + (ks & 3) * 32),
-                                sdesc_kmajor_sw128(pb + (ks >> 2) * 2048 + (ks & 3) * 32), ida, ks > 0 ? 1u : 0u);
-                tc_commit(&S.o_full[b]);
-                tc_commit(&S.wempty[w1 % kWSlots]);
-            }
+        auto scores = [&](int i) -> bool {  // S = K q^T
+            const int g = gi + i, b = g & 1;
+            const uint32_t w0 = wb + 2 * i;
+            if (!mwait(&S.q_ready[b], (g >> 1) & 1, err, ab) || !wwait(w0)) return false;
+            tc_fence_after();
+            const uint32_t dS = tmem + kTmemS + 16 * b, qb = smem_u32(sQ + 4096 * b), kb = wslot(w0);
+            for (int ks = 0; ks < p.hd / 16; ++ks)
+                tc_mma_bf16(dS, sdesc_kmajor_sw128(kb + (ks >> 2) * 16384 + (ks & 3) * 32),
+                            sdesc_kmajor_sw128(qb + (ks >> 2) * 2048 + (ks & 3) * 32), ida, ks > 0 ? 1u : 0u);
+            tc_commit(&S.s_full[b]);
+            tc_commit(&S.wempty[w0 % kWSlots]);
+            return true;
+        };
+        auto pv = [&](int i) -> bool {  // O^T = V^T P^T
+            const int g = gi + i, b = g & 1;
+            const uint32_t w1 = wb + 2 * i + 1;
+            const AttUnit u = att_unit(p, a0 + i);
+            if (!mwait(&S.p_ready[b], (g >> 1) & 1, err, ab) || !wwait(w1)) return false;
+            tc_fence_after();
+            const uint32_t dO = tmem + kTmemO + 16 * b, pb = smem_u32(sP + 4096 * b), vb = wslot(w1);
+            const int ksteps = (u.n + 15) >> 4;
+            for (int ks = 0; ks < ksteps; ++ks)
+                tc_mma_bf16(dO, sdesc_kmajor_sw128(vb + (ks >> 2) * 16384 + (ks & 3) * 32),
+                            sdesc_kmajor_sw128(pb + (ks >> 2) * 2048 + (ks & 3) * 32), ida, ks > 0 ? 1u : 0u);
+            tc_commit(&S.o_full[b]);
+            tc_commit(&S.wempty[w1 % kWSlots]);
+            return true;
+        };
+        for (int i = 0; i < n && ok; i += 2) {
+            const bool two = i + 1 < n;
+            if (!scores(i) || (two && !scores(i + 1)) || !pv(i) || (two && !pv(i + 1))) ok = false;
         }
         wi = wb + 2 * n;
         gi += n;
@@ -553,7 +559,7 @@ __device__ __forceinline__ void head_granule(const MegaParams &p, const GemmPh &
     const int fr = low ? d0 : pd0;
 #pragma unroll
     for (int e = 0; e < 8; ++e) {
-        const float2 c = __ldg(&cs[fr + e]);
+        const float2 c = __ldg(&cs[fr + e]);  // (read-only table)
         y[e] = (low ? (x[e] * c.x - xp[e] * c.y) : (x[e] * c.x + xp[e] * c.y)) * scale;
     }
 }
@@ -585,8 +591,9 @@ __device__ __forceinline__ void mega_compute(const MegaParams &p, MegaSmem &S, u
 
     // phase arrival: the CTA's writes of this phase (made visible to thread 0 by the barrier)
     // are released to the other CTAs with the counter increment
-    auto arrive = [&](int idx) {
-        fence_proxy_async_global();
+    // (x_operand: this phase wrote a GEMM operand that bulk copies of other CTAs will read)
+    auto arrive = [&](int idx, bool x_operand) {
+        if (x_operand) fence_proxy_async_global();
         named_bar_sync(1, kMegaCThreads);
         if (ctid == 0) {
             fence_acq_rel_gpu();
@@ -701,7 +708,7 @@ __device__ __forceinline__ void mega_compute(const MegaParams &p, MegaSmem &S, u
     }
     __syncwarp();
     fin_resid(nullptr, p.attn_norm, p.ssqA);
-    arrive(0);
+    arrive(0, true);
 
     for (int l = 0; l < p.layers; ++l) {
         const int base = 1 + kPhasesPerLayer * l;
@@ -712,46 +719,64 @@ __device__ __forceinline__ void mega_compute(const MegaParams &p, MegaSmem &S, u
         gemm_range(gq, u0, u1);
         gemm_epi(gq, u0, u1);
         wi += (uint32_t)(u1 - u0);
-        arrive(base + 0);
+        arrive(base + 0, false);
         // ------------------------------------------------------------ attention
         {
-            wait_phase(base + 0);
-            const bool det_layer = l == min(2, p.layers - 1);
-            if (det_layer && ctid == 0) MEGA_DETAIL(13);
+            // nothing below depends on the QKV phase until the partial sums: the RMS scales
+            // (from the previous layer's finalisation, complete before QKV could start) and
+            // the units' metadata and rotary entries (read-only; touched so they sit in L1)
+            wait_phase(base - 1);
             load_rstd(p.ssqA);
-            if (det_layer && ctid == 0) MEGA_DETAIL(14);
             int64_t a0, a1;
             att_range(p, S.n_items, a0, a1);
             const int n = (int)(a1 - a0);
             const uint32_t wb = wi;
+            if (n > 0 && ctid < 128) {
+                const AttUnit u = att_unit(p, a0 + (ctid & 1) * (n > 1 ? 1 : 0));
+                const float2 c = __ldg(p.rope + (int64_t)(u.ctx - 1) * (hd / 2) + ((ctid >> 1) & 63) % (hd / 2));
+                if (c.x == 12345.f) S.last_flag = 0;  // keeps the loads
+            }
+            wait_phase(base + 0);
+            const bool det_layer = l == min(2, p.layers - 1);
+            if (det_layer && ctid == 0) MEGA_DETAIL(13);
+            if (det_layer && ctid == 0) MEGA_DETAIL(14);
 #define DETAIL(i)                                       \
     do {                                                \
         if (det_layer && ctid == 0 && i_unit == 0) MEGA_DETAIL(i); \
     } while (0)
             int i_unit = 0;
             DETAIL(0);
-            // per unit i: all compute warps build the q tile (warps 3..6) and, on a row's last
-            // split, the new position's k and v (warps 7..10); warps 3..6 then run the softmax
-            // of unit i - 1 and the output / split merge of unit i - 2
-            for (int i = 0; i < n + 2; ++i) {
-                if (i < n) {
-                    const AttUnit u = att_unit(p, a0 + i);
-                    const int b = (gi + i) & 1;
-                    const float rs = S.rstd[u.row];
-                    const float2 *cs = p.rope + (int64_t)(u.ctx - 1) * (hd / 2);
-                    if (half == 0) {  // q tile rows 0..7 (score columns 8..15 are unused)
-                        const int g = ctid >> 4, j = ctid & 15;
-                        uint4 pk = make_uint4(0, 0, 0, 0);
-                        if (g < Gq && j * 8 < hd) {
-                            float y[8];
-                            head_granule(p, gq, u.row, u.kvh * Gq + g, j, hd, cs, true, rs * p.scale_log2, y);
-                            pk = pack_f16x8(y);
-                        }
+            // units alternate between the two warp groups: group h (warps 3..6 / 7..10, named
+            // barrier 2 + h) runs the units whose buffer parity (gi + i) & 1 is h, each unit
+            // q tile (+ the new position's k, v on a row's last split) -> softmax -> output /
+            // split merge, in order; the MMA issuer interleaves the two groups' units
+            const int hb = 2 + half;     // this group's named barrier
+            const int ht = ctid & 127;   // thread index within the group
+            const int hq = ht >> 5;      // warp within the group (owns TMEM lanes 32 hq..)
+            const bool kv_spare = Gq <= 6;  // spare q-tile threads build k, v in parallel
+            for (int i = half ? 1 - (gi & 1) : (gi & 1); i < n; i += 2) {
+                const AttUnit u = att_unit(p, a0 + i);
+                const int gidx = gi + i, b = half;  // (gidx & 1) == half
+                const uint32_t ph = (uint32_t)((gidx >> 1) & 1);
+                const float rs = S.rstd[u.row];
+                const float2 *cs = p.rope + (int64_t)(u.ctx - 1) * (hd / 2);
+                // ---- q tile rows 0..7 (score columns 8..15 are unused) and k, v
+                {
+                    const int g = ht >> 4, j = ht & 15;
+                    const bool is_q = g < Gq && j * 8 < hd;
+                    if (is_q) {
+                        float y[8];
+                        head_granule(p, gq, u.row, u.kvh * Gq + g, j, hd, cs, true, rs * p.scale_log2, y);
                         *reinterpret_cast<uint4 *>(sQ + 4096 * b + (j >> 3) * 2048 + g * 128 + (((j & 7) ^ (g & 7)) << 4)) =
-                            pk;
-                    } else if (u.last && ctid < 160) {  // k, v of the new position (cache + ring slot)
-                        const int jj = ctid & 15;
-                        const bool isv = ctid >= 144;
+                            pack_f16x8(y);
+                    } else {
+                        *reinterpret_cast<uint4 *>(sQ + 4096 * b + (j >> 3) * 2048 + g * 128 + (((j & 7) ^ (g & 7)) << 4)) =
+                            make_uint4(0, 0, 0, 0);
+                    }
+                    const int kvt = kv_spare ? ht - 96 : ht;  // 0..15 k granules, 16..31 v granules
+                    if (u.last && kvt >= 0 && kvt < 32) {
+                        const int jj = kvt & 15;
+                        const bool isv = kvt >= 16;
                         if (jj * 8 < hd) {
                             const int pp = u.ctx - 1 - u.p0;
                             const int head = p.H + (isv ? p.KVH : 0) + u.kvh;
@@ -778,17 +803,14 @@ __device__ __forceinline__ void mega_compute(const MegaParams &p, MegaSmem &S, u
                         }
                     }
                     fence_proxy_async_smem();
-                    named_bar_sync(1, kMegaCThreads);
-                    i_unit = i;
-                    DETAIL(1);
-                    if (ctid == 0) mbar_arrive(&S.q_ready[b]);
+                    named_bar_sync(hb, 128);
+                    if (half == 0) { i_unit = i; DETAIL(1); }
+                    if (ht == 0) mbar_arrive(&S.q_ready[b]);
                 }
-                if (half == 0 && i >= 1 && i <= n) {  // softmax of unit i - 1 -> P
-                    const AttUnit u = att_unit(p, a0 + i - 1);
-                    const int g1 = gi + i - 1, b = g1 & 1;
-                    mwait(&S.s_full[b], (g1 >> 1) & 1, err, ab);
-                    i_unit = i - 1;
-                    DETAIL(2);
+                // ---- softmax -> P
+                {
+                    mwait(&S.s_full[b], ph, err, ab);
+                    if (half == 0) { i_unit = i; DETAIL(2); }
                     tc_fence_after();
                     float sv[8];
                     tmem_ld_32x32b_x8(tmem + lane_base + kTmemS + 16 * b, sv);
@@ -800,45 +822,43 @@ __device__ __forceinline__ void mega_compute(const MegaParams &p, MegaSmem &S, u
                         float m = sv[g];
 #pragma unroll
                         for (int o = 16; o > 0; o >>= 1) m = fmaxf(m, __shfl_xor_sync(0xffffffffu, m, o));
-                        if (lane == 0) S.red[quarter][g] = m;
+                        if (lane == 0) S.red[half][quarter][g] = m;
                     }
                     tc_fence_before();
-                    named_bar_sync(2, 128);
+                    named_bar_sync(hb, 128);
                     float M[8];
                     uint8_t *pb = sP + 4096 * b + (pos >> 6) * 2048;
                     const int pc = pos & 63;
 #pragma unroll
                     for (int g = 0; g < 8; ++g) {
-                        M[g] = fmaxf(fmaxf(S.red[0][g], S.red[1][g]), fmaxf(S.red[2][g], S.red[3][g]));
+                        M[g] = fmaxf(fmaxf(S.red[half][0][g], S.red[half][1][g]), fmaxf(S.red[half][2][g], S.red[half][3][g]));
                         const float e = valid ? exp2f(sv[g] - M[g]) : 0.f;
                         *reinterpret_cast<uint16_t *>(pb + g * 128 + ((((pc >> 3) ^ (g & 7)) << 4) | ((pc & 7) << 1))) =
                             f32_to_f16_sat(e);
                         const float se = warp_sum(e);
-                        if (lane == 0) S.red2[quarter][g] = se;
+                        if (lane == 0) S.red2[half][quarter][g] = se;
                     }
                     fence_proxy_async_smem();
-                    named_bar_sync(2, 128);
-                    DETAIL(3);
-                    if (ctid == 0) mbar_arrive(&S.p_ready[b]);
-                    if (ctid < 8) {  // read by the output step of this unit, after more barriers
+                    named_bar_sync(hb, 128);
+                    if (half == 0) DETAIL(3);
+                    if (ht == 0) mbar_arrive(&S.p_ready[b]);
+                    if (ht < 8) {
                         float mc = M[0];
 #pragma unroll
-                        for (int g = 1; g < 8; ++g) mc = (ctid == g) ? M[g] : mc;
-                        S.att_m[b][ctid] = mc;
-                        S.att_l[b][ctid] = S.red2[0][ctid] + S.red2[1][ctid] + S.red2[2][ctid] + S.red2[3][ctid];
+                        for (int g = 1; g < 8; ++g) mc = (ht == g) ? M[g] : mc;
+                        S.att_m[b][ht] = mc;
+                        S.att_l[b][ht] = S.red2[half][0][ht] + S.red2[half][1][ht] + S.red2[half][2][ht] + S.red2[half][3][ht];
                     }
                 }
-                if (half == 0 && i >= 2) {  // output of unit i - 2
-                    const AttUnit u = att_unit(p, a0 + i - 2);
-                    const int g2 = gi + i - 2, b = g2 & 1;
-                    mwait(&S.o_full[b], (g2 >> 1) & 1, err, ab);
-                    i_unit = i - 2;
-                    DETAIL(4);
+                // ---- output (single split) or partial + split merge
+                {
+                    mwait(&S.o_full[b], ph, err, ab);
+                    if (half == 0) DETAIL(4);
                     tc_fence_after();
                     float ov[8];
                     tmem_ld_32x32b_x8(tmem + lane_base + kTmemO + 16 * b, ov);
                     tc_fence_before();
-                    named_bar_sync(2, 128);  // att_m / att_l of this buffer are complete
+                    named_bar_sync(hb, 128);  // att_m / att_l of this unit are complete
                     const int dd = quarter * 32 + lane;
                     if (u.nsplit == 1) {
                         if (dd < hd) {
@@ -855,27 +875,27 @@ __device__ __forceinline__ void mega_compute(const MegaParams &p, MegaSmem &S, u
                             for (int g = 0; g < 8; ++g)
                                 if (g < Gq) mine[g * (hd + 2) + 2 + dd] = ov[g];
                         }
-                        if (ctid < Gq) {
-                            mine[ctid * (hd + 2)] = S.att_m[b][ctid];
-                            mine[ctid * (hd + 2) + 1] = S.att_l[b][ctid];
+                        if (ht < Gq) {
+                            mine[ht * (hd + 2)] = S.att_m[b][ht];
+                            mine[ht * (hd + 2) + 1] = S.att_l[b][ht];
                         }
-                        named_bar_sync(2, 128);
-                        DETAIL(5);
-                        if (ctid == 0) {
+                        named_bar_sync(hb, 128);
+                        if (half == 0) DETAIL(5);
+                        if (ht == 0) {
                             fence_acq_rel_gpu();
                             const int old = atomicAdd(&p.att_cnt[u.row * p.KVH + u.kvh], 1);
-                            S.last_flag = old == u.nsplit - 1;
-                            if (S.last_flag) p.att_cnt[u.row * p.KVH + u.kvh] = 0;
+                            S.last_flag2[half] = old == u.nsplit - 1;
+                            if (S.last_flag2[half]) p.att_cnt[u.row * p.KVH + u.kvh] = 0;
                             fence_acq_rel_gpu();
                         }
-                        named_bar_sync(2, 128);
-                        DETAIL(6);
-                        if (S.last_flag) {  // merge the row's splits in split order
+                        named_bar_sync(hb, 128);
+                        if (half == 0) DETAIL(6);
+                        if (S.last_flag2[half]) {  // merge the row's splits in split order
                             const int ns = min(u.nsplit, kMegaMaxSplits);
                             const int64_t sp_stride = (int64_t)p.KVH * Gq * (hd + 2);
-                            const float *pbase = p.part + ((int64_t)p.c.row_item0[u.row] * p.KVH + u.kvh) * Gq * (hd + 2);
-                            // split weights 2^(m_s - M) and the total weight L per head (warp cw: heads cw, cw + 4)
-                            for (int g = cw; g < Gq; g += 4) {
+                            const float *pbase = p.part + ((int64_t)__ldg(&p.c.row_item0[u.row]) * p.KVH + u.kvh) * Gq * (hd + 2);
+                            // split weights 2^(m_s - M) and the total weight L per head (warp hq: heads hq, hq + 4)
+                            for (int g = hq; g < Gq; g += 4) {
                                 float ms[3], ls[3];
                                 float Mx = -INFINITY;
 #pragma unroll
@@ -892,13 +912,13 @@ __device__ __forceinline__ void mega_compute(const MegaParams &p, MegaSmem &S, u
                                 for (int q = 0; q < 3; ++q) {
                                     const int sp = lane + 32 * q;
                                     const float w = sp < ns ? exp2f(ms[q] - Mx) : 0.f;
-                                    if (sp < ns) S.mw[g][sp] = w;
+                                    if (sp < ns) S.mw[half][g][sp] = w;
                                     L += w * ls[q];
                                 }
                                 L = warp_sum(L);
-                                if (lane == 0) S.ml[g] = L;
+                                if (lane == 0) S.ml[half][g] = L;
                             }
-                            named_bar_sync(2, 128);
+                            named_bar_sync(hb, 128);
                             if (dd < hd) {  // thread dd: output dim dd of every head
                                 float acc[8];
 #pragma unroll
@@ -910,17 +930,17 @@ __device__ __forceinline__ void mega_compute(const MegaParams &p, MegaSmem &S, u
 #pragma unroll
                                     for (int g = 0; g < 8; ++g) v[g] = g < Gq ? __ldcg(src + sp * sp_stride + g * (hd + 2)) : 0.f;
 #pragma unroll
-                                    for (int g = 0; g < 8; ++g) acc[g] += (g < Gq ? S.mw[g][sp] : 0.f) * v[g];
+                                    for (int g = 0; g < 8; ++g) acc[g] += (g < Gq ? S.mw[half][g][sp] : 0.f) * v[g];
                                 }
 #pragma unroll
                                 for (int g = 0; g < 8; ++g)
                                     if (g < Gq)
                                         store_hilo(p.att_hi, p.att_lo, xblk_off(u.row, (u.kvh * Gq + g) * hd + dd, R16c),
-                                                   acc[g] / S.ml[g]);
+                                                   acc[g] / S.ml[half][g]);
                             }
                         }
-                        named_bar_sync(2, 128);
-                        DETAIL(7);
+                        named_bar_sync(hb, 128);
+                        if (half == 0) DETAIL(7);
                     }
                 }
             }
@@ -928,7 +948,7 @@ __device__ __forceinline__ void mega_compute(const MegaParams &p, MegaSmem &S, u
             gi += n;
             i_unit = 0;
             DETAIL(8);
-            arrive(base + 1);
+            arrive(base + 1, true);
             DETAIL(9);
 #undef DETAIL
         }
@@ -936,19 +956,19 @@ __device__ __forceinline__ void mega_compute(const MegaParams &p, MegaSmem &S, u
         gemm_range(go, u0, u1);
         gemm_epi(go, u0, u1);
         wi += (uint32_t)(u1 - u0);
-        arrive(base + 2);
+        arrive(base + 2, false);
         // ------------------------------------------------------------ residual, MLP norm input
         wait_phase(base + 2);
         if (l == min(2, p.layers - 1) && ctid == 0) MEGA_DETAIL(10);
         fin_resid(&go, p.mlp_norm + (int64_t)l * d, p.ssqM);
         if (l == min(2, p.layers - 1) && ctid == 0) MEGA_DETAIL(11);
-        arrive(base + 3);
+        arrive(base + 3, true);
         if (l == min(2, p.layers - 1) && ctid == 0) MEGA_DETAIL(12);
         // ------------------------------------------------------------ gate / up
         gemm_range(gu, u0, u1);
         gemm_epi(gu, u0, u1);
         wi += (uint32_t)(u1 - u0);
-        arrive(base + 4);
+        arrive(base + 4, false);
         // ------------------------------------------------------------ SwiGLU
         {
             wait_phase(base + 4);
@@ -1006,17 +1026,17 @@ __device__ __forceinline__ void mega_compute(const MegaParams &p, MegaSmem &S, u
                         make_uint2((uint32_t)hl[0] | ((uint32_t)hl[1] << 16), (uint32_t)hl[2] | ((uint32_t)hl[3] << 16));
                 }
             }
-            arrive(base + 5);
+            arrive(base + 5, true);
         }
         // ------------------------------------------------------------ down
         gemm_range(gdn, u0, u1);
         gemm_epi(gdn, u0, u1);
         wi += (uint32_t)(u1 - u0);
-        arrive(base + 6);
+        arrive(base + 6, false);
         // ------------------------------------------------------------ residual, next norm input
         wait_phase(base + 6);
         fin_resid(&gdn, (l + 1 < p.layers) ? p.attn_norm + (int64_t)(l + 1) * d : p.final_norm, p.ssqA);
-        arrive(base + 7);
+        arrive(base + 7, true);
     }
 
     // ---------------------------------------------------------------- lm_head
