@@ -88,7 +88,7 @@ struct MegaParams {
     uint8_t *xg_hi, *xg_lo;                         // blocked [d/64][rows_cap16][64]
     uint8_t *att_hi, *att_lo;                       // blocked [H*hd/64][rows_cap16][64]
     uint8_t *h_hi, *h_lo;                           // blocked [F/64][rows_cap16][64]
-    float *ssqA, *ssqM;                             // [d/128][rows_cap] partial sums of x^2
+    float *ssqA, *ssqM;                             // [d/64][rows_cap] partial sums of x^2
     float *gpart;                                   // [segments][rows_cap][256] GEMM partial tiles
     float *part;                                    // [items][KVH][Gq][hd + 2] attention split partials
     int *att_cnt;                                   // [rows_cap][KVH] split arrival counters
@@ -424,7 +424,8 @@ __device__ __forceinline__ void mega_mma(const MegaParams &p, MegaSmem &S, uint8
             if (use_a >= 1 && !mwait(&S.acc_empty[a], (use_a - 1) & 1, err, ab)) { ok = false; break; }
             tc_fence_after();
             const uint32_t d = tmem + (uint32_t)(a * kTileN);
-            const uint32_t idg = idesc_bf16_f32(128, (uint32_t)tile_rows(g, t));
+            // M = 64 when every live row fits: same cost, rows spread over all four lane quarters
+            const uint32_t idg = idesc_bf16_f32(R16 <= 64 ? 64u : 128u, (uint32_t)tile_rows(g, t));
             bool first = true;
             for (; u < e; ++u, ++wi, ++xi) {
                 const int xs = (int)(xi % NX);
@@ -582,10 +583,14 @@ __device__ __forceinline__ void mega_compute(const MegaParams &p, MegaSmem &S, u
     const int half = cw >> 2;                    // warps 3..6 -> 0, 7..10 -> 1
     const int G = gridDim.x, cta = blockIdx.x;
     const int R = S.rows, R16c = p.rows_cap16;
-    const int d = p.d, dt = d / 128, hd = p.hd, Gq = p.Gq;
+    const int d = p.d, hd = p.hd, Gq = p.Gq;
     const int gw = cta * 8 + cw, nw = G * 8;
     const uint32_t lane_base = (uint32_t)(quarter * 32) << 16;
-    const int my_row = quarter * 32 + lane;  // GEMM accumulator lane = activation row
+    // GEMM accumulator lane -> activation row: M = 128 puts row i in lane i; M = 64 (at most 64
+    // live rows) puts row i in lane 32 (i / 16) + i % 16
+    const bool m64 = S.rows16 <= 64;
+    const int my_row = m64 ? ((lane < 16) ? quarter * 16 + lane : 1 << 20) : quarter * 32 + lane;
+    const bool quarter_live = (m64 ? quarter * 16 : quarter * 32) < R;
     uint32_t wi = 0;
     int gi = 0, cuse0 = 0, cuse1 = 0, lmseg = 0;  // accumulator buffer uses
 
@@ -609,13 +614,13 @@ __device__ __forceinline__ void mega_compute(const MegaParams &p, MegaSmem &S, u
         named_bar_sync(1, kMegaCThreads);
     };
     auto load_rstd = [&](const float *ssq) {
-        if (ctid < R) {  // every partial load in flight at once (d <= 2048: at most 16)
-            float v[16];
+        if (ctid < R) {  // every partial load in flight at once (d <= 2048: at most 32)
+            float v[32];
 #pragma unroll
-            for (int t = 0; t < 16; ++t) v[t] = t < dt ? __ldcg(&ssq[(int64_t)t * p.rows_cap + ctid]) : 0.f;
+            for (int t = 0; t < 32; ++t) v[t] = t < d / 64 ? __ldcg(&ssq[(int64_t)t * p.rows_cap + ctid]) : 0.f;
             float s = 0.f;
 #pragma unroll
-            for (int t = 0; t < 16; ++t) s += v[t];
+            for (int t = 0; t < 32; ++t) s += v[t];
             S.rstd[ctid] = rsqrtf(s / (float)d + p.eps);
         }
         named_bar_sync(1, kMegaCThreads);
@@ -628,8 +633,8 @@ __device__ __forceinline__ void mega_compute(const MegaParams &p, MegaSmem &S, u
             mwait(&S.acc_full[0], cuse0 & 1, err, ab);
             tc_fence_after();
             const int rows_t = tile_rows(g, t);
-            if (quarter * 32 < R && half * 128 < rows_t) {
-                float *dst = p.gpart + ((int64_t)(cta + t) * p.rows_cap + my_row) * kTileN + half * 128;
+            if (quarter_live && half * 128 < rows_t) {
+                float *dst = p.gpart + ((int64_t)(cta + t) * p.rows_cap + (my_row < R ? my_row : 0)) * kTileN + half * 128;
 #pragma unroll 1
                 for (int cc = 0; cc < 4; ++cc) {
                     float v[32];
@@ -650,61 +655,58 @@ __device__ __forceinline__ void mega_compute(const MegaParams &p, MegaSmem &S, u
     // x += (sum of g's partials); x_g = x * gn (blocked hi/lo); per (row, 128-feature
     // block) sum of squares of x.  g == nullptr: x as it is (embedding).
     auto fin_resid = [&](const GemmPh *g, const uint16_t *gn, float *ssq) {
-        for (int u = gw; u < R * dt; u += nw) {
-            const int r = u / dt, t = u - r * dt;
-            const int f = t * 128 + lane * 4;
-            float4 x = __ldcg(reinterpret_cast<const float4 *>(p.x + (int64_t)r * d + f));
+        // unit = (row, 64 features): lane = 2 features; up to 32 contributors' loads in
+        // flight per round, summed in CTA order.  Sums of squares per 128 features: the two
+        // 64-feature halves of a block are adjacent units of the same warp pass
+        const int d64 = d / 64;
+        for (int u = gw; u < R * d64; u += nw) {
+            const int r = u / d64, h64 = u - r * d64;
+            const int f = h64 * 64 + lane * 2;
+            float2 x = __ldcg(reinterpret_cast<const float2 *>(p.x + (int64_t)r * d + f));
             if (g) {
                 const int gt = f / kTileN, col = f - gt * kTileN;
                 int ca, cb;
                 tile_ctas(*g, gt, ca, cb);
-                float4 s = make_float4(0.f, 0.f, 0.f, 0.f);
-                for (int c0 = ca; c0 <= cb; c0 += 16) {  // 16 contributors' loads in flight, summed in CTA order
-                    float4 v[16];
+                float2 s = make_float2(0.f, 0.f);
+                for (int c0 = ca; c0 <= cb; c0 += 32) {
+                    float2 v[32];
 #pragma unroll
-                    for (int k = 0; k < 16; ++k)
-                        v[k] = c0 + k <= cb ? __ldcg(reinterpret_cast<const float4 *>(
+                    for (int k = 0; k < 32; ++k)
+                        v[k] = c0 + k <= cb ? __ldcg(reinterpret_cast<const float2 *>(
                                                   p.gpart + ((int64_t)(c0 + k + gt) * p.rows_cap + r) * kTileN + col))
-                                            : make_float4(0.f, 0.f, 0.f, 0.f);
+                                            : make_float2(0.f, 0.f);
 #pragma unroll
-                    for (int k = 0; k < 16; ++k) {
-                        s.x += v[k].x; s.y += v[k].y; s.z += v[k].z; s.w += v[k].w;
+                    for (int k = 0; k < 32; ++k) {
+                        s.x += v[k].x; s.y += v[k].y;
                     }
                 }
-                x.x += s.x; x.y += s.y; x.z += s.z; x.w += s.w;
-                *reinterpret_cast<float4 *>(p.x + (int64_t)r * d + f) = x;
+                x.x += s.x; x.y += s.y;
+                *reinterpret_cast<float2 *>(p.x + (int64_t)r * d + f) = x;
             }
-            const uint2 gb = *reinterpret_cast<const uint2 *>(gn + f);
-            const float g0 = bf16_to_f32(gb.x & 0xffff), g1 = bf16_to_f32(gb.x >> 16);
-            const float g2 = bf16_to_f32(gb.y & 0xffff), g3 = bf16_to_f32(gb.y >> 16);
-            uint16_t h[4], lo[4];
-            split_bf16(x.x * g0, h[0], lo[0]);
-            split_bf16(x.y * g1, h[1], lo[1]);
-            split_bf16(x.z * g2, h[2], lo[2]);
-            split_bf16(x.w * g3, h[3], lo[3]);
+            const uint32_t gb = *reinterpret_cast<const uint32_t *>(gn + f);
+            uint16_t h0, l0, h1, l1;
+            split_bf16(x.x * bf16_to_f32(gb & 0xffff), h0, l0);
+            split_bf16(x.y * bf16_to_f32(gb >> 16), h1, l1);
             const int64_t off = xblk_off(r, f, R16c);
-            *reinterpret_cast<uint2 *>(p.xg_hi + off) =
-                make_uint2((uint32_t)h[0] | ((uint32_t)h[1] << 16), (uint32_t)h[2] | ((uint32_t)h[3] << 16));
-            *reinterpret_cast<uint2 *>(p.xg_lo + off) =
-                make_uint2((uint32_t)lo[0] | ((uint32_t)lo[1] << 16), (uint32_t)lo[2] | ((uint32_t)lo[3] << 16));
-            const float s = warp_sum(x.x * x.x + x.y * x.y + x.z * x.z + x.w * x.w);
-            if (lane == 0) ssq[(int64_t)t * p.rows_cap + r] = s;
+            *reinterpret_cast<uint32_t *>(p.xg_hi + off) = (uint32_t)h0 | ((uint32_t)h1 << 16);
+            *reinterpret_cast<uint32_t *>(p.xg_lo + off) = (uint32_t)l0 | ((uint32_t)l1 << 16);
+            const float sq = warp_sum(x.x * x.x + x.y * x.y);
+            if (lane == 0) ssq[(int64_t)h64 * p.rows_cap + r] = sq;
         }
     };
 
     // ---------------------------------------------------------------- embedding
-    for (int u = gw; u < R * dt; u += nw) {
-        const int r = u / dt, t = u - r * dt;
+    // (same (row, 64-feature) units and lanes as the finalisation that reads them back)
+    for (int u = gw; u < R * (d / 64); u += nw) {
+        const int r = u / (d / 64), h64 = u - r * (d / 64);
         int tok = p.c.row_tok[r];
         if (tok < 0 || tok >= p.V) {
             if (lane == 0) report_error(err, ERR_BOUNDS);
             tok = 0;
         }
-        const int f = t * 128 + lane * 4;
-        const uint2 e = *reinterpret_cast<const uint2 *>(p.embed + (int64_t)tok * d + f);
-        const float4 x = make_float4(bf16_to_f32(e.x & 0xffff), bf16_to_f32(e.x >> 16), bf16_to_f32(e.y & 0xffff),
-                                     bf16_to_f32(e.y >> 16));
-        *reinterpret_cast<float4 *>(p.x + (int64_t)r * d + f) = x;
+        const int f = h64 * 64 + lane * 2;
+        const uint32_t e = *reinterpret_cast<const uint32_t *>(p.embed + (int64_t)tok * d + f);
+        *reinterpret_cast<float2 *>(p.x + (int64_t)r * d + f) = make_float2(bf16_to_f32(e & 0xffff), bf16_to_f32(e >> 16));
     }
     __syncwarp();
     fin_resid(nullptr, p.attn_norm, p.ssqA);
@@ -1055,8 +1057,8 @@ __device__ __forceinline__ void mega_compute(const MegaParams &p, MegaSmem &S, u
             const int a = lmseg & 1;
             mwait(&S.acc_full[a], (a ? cuse1 : cuse0) & 1, err, ab);
             tc_fence_after();
-            if (quarter * 32 < R && half * 128 < tile_rows(g, t)) {
-                float *dst = p.logits + (int64_t)my_row * p.V + t * kTileN + half * 128;
+            if (quarter_live && half * 128 < tile_rows(g, t)) {
+                float *dst = p.logits + (int64_t)(act ? my_row : 0) * p.V + t * kTileN + half * 128;
 #pragma unroll 1
                 for (int cc = 0; cc < 4; ++cc) {
                     float v[32];

@@ -581,8 +581,8 @@ void alloc_decode(sara_handle &h) {
     h.att_lo = h.mem.alloc<uint8_t>(R16 * Hhd * 2);
     h.h_hi = h.mem.alloc<uint8_t>(R16 * F * 2);
     h.h_lo = h.mem.alloc<uint8_t>(R16 * F * 2);
-    h.ssqA = h.mem.alloc<float>((size_t)(d / 128) * S);
-    h.ssqM = h.mem.alloc<float>((size_t)(d / 128) * S);
+    h.ssqA = h.mem.alloc<float>((size_t)(d / 64) * S);
+    h.ssqM = h.mem.alloc<float>((size_t)(d / 64) * S);
     // partial tiles: one segment per (CTA, tile) pair of a phase, at most CTAs + tiles - 1
     const int tmax = std::max({nqkv, d, 2 * F}) / kTileN + 1;
     h.gpart = h.mem.alloc<float>((size_t)(h.sms + tmax) * S * kTileN, false);
