@@ -48,6 +48,8 @@ def parse():
                          "eager decode step) on a reduced-capacity handle of the workload's shapes")
     ap.add_argument("--rows", type=int, default=25, help="live rows in --kernel-profile mode")
     ap.add_argument("--iters", type=int, default=5, help="launches in --kernel-profile mode")
+    ap.add_argument("--ctx", type=int, default=None, help="context length in --kernel-profile mode "
+                    "(default: prompt length + 128)")
     return ap.parse_args()
 
 
@@ -378,11 +380,13 @@ def run_kernel_profile(args):
     w = synth.WORKLOADS[args.workload]
     m = w.model
     weights = synth.model_weights(m, w.weight_seed)
+    ctx = args.ctx if args.ctx is not None else w.prompt_len + 128
+    gen = max(512, ctx - w.prompt_len + 2 * args.iters + 8)
     cfg = pkg.model_cfg(m, max_prompts=w.n_prompts, max_active=max(16, args.rows), max_seqs=max(32, args.rows),
-                        max_prompt_len=w.prompt_len, max_gen_len=512, max_k=w.k)
+                        max_prompt_len=w.prompt_len, max_gen_len=gen, max_k=w.k)
     with pkg.Handle(cfg, weights, stream=torch.cuda.current_stream()) as h:
-        ms = h.profile(args.kernel_profile, args.rows, w.prompt_len + 128, iters=args.iters)
-    print(json.dumps({"kernel": args.kernel_profile, "rows": args.rows, "ms_per_launch": ms}))
+        ms = h.profile(args.kernel_profile, args.rows, ctx, iters=args.iters)
+    print(json.dumps({"kernel": args.kernel_profile, "rows": args.rows, "ctx": ctx, "ms_per_launch": ms}))
 
 
 # --------------------------------------------------------------------------------- reference arm

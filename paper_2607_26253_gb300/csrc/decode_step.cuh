@@ -26,17 +26,18 @@
 //   warps 3..10  compute: GEMM epilogues, attention softmax / merge, residual + RMSNorm +
 //                SwiGLU finalisation, embedding, logits
 //
-// Phases of layer l (counter index 1 + 8l + k):
+// Phases of layer l (counter index 1 + 9l + k):
 //   0 QKV   x_g W_qkv^T -> partials        (a subset of the CTAs: few tiles)
-//   1 ATT   q, k, v = RMSNorm scale + RoPE of the summed partials; new k, v appended to
-//           the KV cache; softmax(q K^T) V on the tensor cores per 128-position split;
-//           the last split of a row to finish merges them
-//   2 O     att W_o^T -> partials           (a subset of the CTAs)
-//   3 FIN_O x += sum; x_g = x * g_mlp (bf16 hi/lo, blocked); per-row sum of squares
-//   4 GU    x_g W_gu^T -> partials          (gate / up interleaved in 64-row blocks)
-//   5 FIN_GU h = silu(r g) * (r u), r = 1/rms(x)  (bf16 hi/lo, blocked)
-//   6 DOWN  h W_down^T -> partials
-//   7 FIN_D x += sum; x_g = x * g_next; sum of squares
+//   1 FIN_Q q, k, v = RMSNorm scale + RoPE of the summed partials, fp16, once per row; the
+//           new k, v appended to the KV cache
+//   2 ATT   softmax(q K^T) V on the tensor cores per 128-position split; the last split of a
+//           row to finish merges them
+//   3 O     att W_o^T -> partials           (a subset of the CTAs)
+//   4 FIN_O x += sum; x_g = x * g_mlp (bf16 hi/lo, blocked); per-row sum of squares
+//   5 GU    x_g W_gu^T -> partials          (gate / up interleaved in 64-row blocks)
+//   6 FIN_GU h = silu(r g) * (r u), r = 1/rms(x)  (bf16 hi/lo, blocked)
+//   7 DOWN  h W_down^T -> partials
+//   8 FIN_D x += sum; x_g = x * g_next; sum of squares
 // then lm_head over whole 256-token tiles, writing the logits of the live rows.
 //
 // Layouts (all chosen so that bulk copies land MMA operands in shared memory in the
@@ -62,7 +63,11 @@ constexpr int kTileN = 256;           // weight rows (output features) per GEMM 
 constexpr int kKVPos = 128;           // positions per KV block and per attention split
 constexpr int kKVBlockBytes = 65536;  // K 2 x 16 KB + V^T 2 x 16 KB
 constexpr int kMegaMaxSplits = 96;
-constexpr int kPhasesPerLayer = 8;
+constexpr int kPhasesPerLayer = 9;
+// phases of a layer (counter index 1 + 9 l + phase)
+enum : int { kPhQKV = 0, kPhFinQ = 1, kPhAtt = 2, kPhO = 3, kPhFinO = 4, kPhGU = 5, kPhFinGU = 6, kPhDown = 7,
+             kPhFinD = 8 };
+__device__ constexpr int kGemmPhases[4] = {kPhQKV, kPhO, kPhGU, kPhDown};
 constexpr int kSmallPhaseUnits = 2;   // QKV / O: units per participating CTA
 constexpr int kCntStride = 16;        // phase counters 128 bytes apart (one L2 line each)
 constexpr uint32_t kTmemCols = 512;
@@ -90,6 +95,7 @@ struct MegaParams {
     uint8_t *h_hi, *h_lo;                           // blocked [F/64][rows_cap16][64]
     float *ssqA, *ssqM;                             // [d/64][rows_cap] partial sums of x^2
     float *gpart;                                   // [segments][rows_cap][256] GEMM partial tiles
+    uint16_t *qkv16;                                // [rows_cap][nqkv] fp16 q (scaled), k, v of the step
     float *part;                                    // [items][KVH][Gq][hd + 2] attention split partials
     int *att_cnt;                                   // [rows_cap][KVH] split arrival counters
     float *logits;                                  // [rows_cap][V] fp32 (read by the sampling kernel)
@@ -216,18 +222,18 @@ struct GemmPh {
     bool whole;  // whole tiles per CTA (lm_head: the argmax of a tile is finished in one CTA)
 };
 
-// GEMM phase k (0 QKV, 2 O, 4 GU, 6 DOWN) of layer l; l == layers: lm_head.
+// GEMM phase k (kPhQKV, kPhO, kPhGU, kPhDown) of layer l; l == layers: lm_head.
 __device__ __forceinline__ GemmPh gemm_phase(const MegaParams &p, int l, int k) {
     GemmPh g;
     g.whole = false;
     g.Gp = gridDim.x;
     if (l == p.layers) {
         g.w = p.w_lm; g.N = p.V; g.K = p.d; g.xhi = p.xg_hi; g.xlo = p.xg_lo; g.whole = true;
-    } else if (k == 0) {
+    } else if (k == kPhQKV) {
         g.w = p.w_qkv + l * p.ls_qkv; g.N = p.nqkv; g.K = p.d; g.xhi = p.xg_hi; g.xlo = p.xg_lo; g.Gp = p.gp_qkv;
-    } else if (k == 2) {
+    } else if (k == kPhO) {
         g.w = p.w_o + l * p.ls_o; g.N = p.d; g.K = p.H * p.hd; g.xhi = p.att_hi; g.xlo = p.att_lo; g.Gp = p.gp_o;
-    } else if (k == 4) {
+    } else if (k == kPhGU) {
         g.w = p.w_gu + l * p.ls_gu; g.N = 2 * p.F; g.K = p.d; g.xhi = p.xg_hi; g.xlo = p.xg_lo;
     } else {
         g.w = p.w_down + l * p.ls_down; g.N = p.d; g.K = p.F; g.xhi = p.h_hi; g.xlo = p.h_lo;
@@ -293,10 +299,13 @@ __device__ __forceinline__ AttUnit att_unit(const MegaParams &p, int64_t a) {
     u.slot = __ldg(&p.c.row_slot[u.row]);
     return u;
 }
+// Attention units in equal contiguous ranges, counted from the last CTA down: the QKV
+// projection runs on the first CTAs, so a small unit count lands on CTAs that are free
+// to prefetch during it.
 __device__ __forceinline__ void att_range(const MegaParams &p, int n_items, int64_t &a0, int64_t &a1) {
-    const int NU = n_items * p.KVH;
-    a0 = (int)blockIdx.x * NU / (int)gridDim.x;
-    a1 = ((int)blockIdx.x + 1) * NU / (int)gridDim.x;
+    const int NU = n_items * p.KVH, G = (int)gridDim.x, v = G - 1 - (int)blockIdx.x;
+    a0 = v * NU / G;
+    a1 = (v + 1) * NU / G;
 }
 __device__ __forceinline__ uint8_t *kv_block(const MegaParams &p, int l, const AttUnit &u) {
     return p.kv + l * p.kv_layer + (int64_t)u.slot * p.kv_slot + ((int64_t)u.kvh * p.kv_nblk + u.sp) * kKVBlockBytes;
@@ -313,8 +322,9 @@ __device__ __forceinline__ void mega_w_producer(const MegaParams &p, MegaSmem &S
         return i < kWSlots || mwait(&S.wempty[i % kWSlots], ((i / kWSlots) & 1) ^ 1, err, ab);
     };
     for (int l = 0; l <= p.layers && ok; ++l) {
-        for (int k = 0; k < kPhasesPerLayer && ok; k += 2) {
-            if (l == p.layers && k > 0) break;
+        for (int gp = 0; gp < 4 && ok; ++gp) {
+            if (l == p.layers && gp > 0) break;
+            const int k = kGemmPhases[gp];
             const GemmPh g = gemm_phase(p, l, k);
             int64_t u0, u1;
             gemm_range(g, u0, u1);
@@ -349,7 +359,7 @@ __device__ __forceinline__ void mega_w_producer(const MegaParams &p, MegaSmem &S
                     if (u.n > 64) bulk_load(sW + (size_t)s * kSlotBytes + 16384, blk + 49152, vb, &S.wfull[s], pol);
                     ++wi;
                 }
-                MEGA_STAMP(2 + kPhasesPerLayer * l, 2);
+                MEGA_STAMP(1 + kPhasesPerLayer * l + kPhAtt, 2);
             }
         }
     }
@@ -372,13 +382,15 @@ __device__ __forceinline__ void mega_x_producer(const MegaParams &p, MegaSmem &S
     uint32_t xi = 0;
     bool ok = true;
     for (int l = 0; l <= p.layers && ok; ++l) {
-        for (int k = 0; k < kPhasesPerLayer && ok; k += 2) {
-            if (l == p.layers && k > 0) break;
+        for (int gp = 0; gp < 4 && ok; ++gp) {
+            if (l == p.layers && gp > 0) break;
+            const int k = kGemmPhases[gp];
             const GemmPh g = gemm_phase(p, l, k);
             int64_t u0, u1;
             gemm_range(g, u0, u1);
             if (u0 >= u1) continue;
-            // the phase this operand comes from: FIN_D of l-1 / embedding, ATT, FIN_O, FIN_GU
+            // the phase this operand comes from (the one before it): FIN_D of l-1 / embedding,
+            // ATT, FIN_O, FIN_GU
             const int dep = (l == p.layers || k == 0) ? kPhasesPerLayer * l : 1 + kPhasesPerLayer * l + k - 1;
             if (!spin_counter(&p.cnt[dep * kCntStride], S.target, err, ab)) { ok = false; break; }
             MEGA_STAMP(1 + kPhasesPerLayer * l + k, 1);
@@ -488,8 +500,9 @@ __device__ __forceinline__ void mega_mma(const MegaParams &p, MegaSmem &S, uint8
         gi += n;
     };
     for (int l = 0; l <= p.layers && ok; ++l) {
-        for (int k = 0; k < kPhasesPerLayer && ok; k += 2) {
-            if (l == p.layers && k > 0) break;
+        for (int gp = 0; gp < 4 && ok; ++gp) {
+            if (l == p.layers && gp > 0) break;
+            const int k = kGemmPhases[gp];
             const GemmPh g = gemm_phase(p, l, k);
             int64_t u0, u1;
             gemm_range(g, u0, u1);
@@ -499,7 +512,7 @@ __device__ __forceinline__ void mega_mma(const MegaParams &p, MegaSmem &S, uint8
                 int64_t a0, a1;
                 att_range(p, S.n_items, a0, a1);
                 att(a0, a1);
-                MEGA_STAMP(2 + kPhasesPerLayer * l, 3);
+                MEGA_STAMP(1 + kPhasesPerLayer * l + kPhAtt, 3);
             }
         }
     }
@@ -516,62 +529,6 @@ __device__ __forceinline__ void store_hilo(uint8_t *hi, uint8_t *lo, int64_t off
     *reinterpret_cast<uint16_t *>(lo + off) = l;
 }
 
-// 8 consecutive head dims (granule j) of one head of the QKV output (sum of the tile's
-// partials in CTA order), RMSNorm-scaled by `scale`, with the rotary embedding (pairs
-// i, i + hd/2) when `rot`.  A head lies inside one 256-feature tile, so the granule and its
-// rotation partner are read in the same pass over the contributors.
-__device__ __forceinline__ void head_granule(const MegaParams &p, const GemmPh &g, int r, int head, int j, int hd,
-                                             const float2 *cs, bool rot, float scale, float (&y)[8]) {
-    const int d0 = j * 8, half = hd >> 1;
-    const bool low = d0 < half;
-    const int pd0 = low ? d0 + half : d0 - half;
-    const int f0 = head * hd + d0, t = f0 / kTileN;
-    const int col = f0 - t * kTileN, pcol = head * hd + pd0 - t * kTileN;
-    int ca, cb;
-    tile_ctas(g, t, ca, cb);
-    float x[8], xp[8];
-#pragma unroll
-    for (int e = 0; e < 8; ++e) x[e] = xp[e] = 0.f;
-    const float4 z4 = make_float4(0.f, 0.f, 0.f, 0.f);
-    for (int c0 = ca; c0 <= cb; c0 += 7) {  // 7 contributors' loads in flight, summed in CTA order
-        float4 a[7], b[7], pa[7], pb[7];
-#pragma unroll
-        for (int k = 0; k < 7; ++k) {
-            const bool ok = c0 + k <= cb;
-            const float *base = p.gpart + ((int64_t)(c0 + k + t) * p.rows_cap + r) * kTileN;
-            a[k] = ok ? __ldcg(reinterpret_cast<const float4 *>(base + col)) : z4;
-            b[k] = ok ? __ldcg(reinterpret_cast<const float4 *>(base + col + 4)) : z4;
-            pa[k] = (ok && rot) ? __ldcg(reinterpret_cast<const float4 *>(base + pcol)) : z4;
-            pb[k] = (ok && rot) ? __ldcg(reinterpret_cast<const float4 *>(base + pcol + 4)) : z4;
-        }
-#pragma unroll
-        for (int k = 0; k < 7; ++k) {
-            x[0] += a[k].x; x[1] += a[k].y; x[2] += a[k].z; x[3] += a[k].w;
-            x[4] += b[k].x; x[5] += b[k].y; x[6] += b[k].z; x[7] += b[k].w;
-            xp[0] += pa[k].x; xp[1] += pa[k].y; xp[2] += pa[k].z; xp[3] += pa[k].w;
-            xp[4] += pb[k].x; xp[5] += pb[k].y; xp[6] += pb[k].z; xp[7] += pb[k].w;
-        }
-    }
-    if (!rot) {
-#pragma unroll
-        for (int e = 0; e < 8; ++e) y[e] = x[e] * scale;
-        return;
-    }
-    const int fr = low ? d0 : pd0;
-#pragma unroll
-    for (int e = 0; e < 8; ++e) {
-        const float2 c = __ldg(&cs[fr + e]);  // (read-only table)
-        y[e] = (low ? (x[e] * c.x - xp[e] * c.y) : (x[e] * c.x + xp[e] * c.y)) * scale;
-    }
-}
-
-__device__ __forceinline__ uint4 pack_f16x8(const float (&y)[8]) {
-    uint32_t w[4];
-#pragma unroll
-    for (int e = 0; e < 4; ++e)
-        w[e] = (uint32_t)f32_to_f16_sat(y[2 * e]) | ((uint32_t)f32_to_f16_sat(y[2 * e + 1]) << 16);
-    return make_uint4(w[0], w[1], w[2], w[3]);
-}
 
 __device__ __forceinline__ void mega_compute(const MegaParams &p, MegaSmem &S, uint8_t *sW, uint8_t *sQ, uint8_t *sP,
                                              uint32_t tmem) {
@@ -715,30 +672,91 @@ __device__ __forceinline__ void mega_compute(const MegaParams &p, MegaSmem &S, u
     for (int l = 0; l < p.layers; ++l) {
         const int base = 1 + kPhasesPerLayer * l;
         int64_t u0, u1;
-        const GemmPh gq = gemm_phase(p, l, 0), go = gemm_phase(p, l, 2), gu = gemm_phase(p, l, 4),
-                     gdn = gemm_phase(p, l, 6);
+        const GemmPh gq = gemm_phase(p, l, kPhQKV), go = gemm_phase(p, l, kPhO), gu = gemm_phase(p, l, kPhGU),
+                     gdn = gemm_phase(p, l, kPhDown);
         // ------------------------------------------------------------ QKV
         gemm_range(gq, u0, u1);
         gemm_epi(gq, u0, u1);
         wi += (uint32_t)(u1 - u0);
-        arrive(base + 0, false);
+        arrive(base + kPhQKV, false);
+        // ------------------------------------------------------------ q, k, v (once per row)
+        {
+            // unit = (row, head, 64 dims): the head's QKV partials summed in CTA order, times
+            // 1/rms; RoPE on q and k; q pre-scaled by log2(e)/sqrt(hd) for the exp2 softmax;
+            // fp16 q, k, v for the attention phase; k and v appended to the KV cache at the
+            // row's position
+            wait_phase(base + kPhQKV);
+            load_rstd(p.ssqA);
+            const int nh = p.H + 2 * p.KVH, dpu = min(hd, 64), upr = hd / dpu;
+            for (int u = gw; u < R * nh * upr; u += nw) {
+                const int r = u / (nh * upr), rem = u - r * nh * upr;
+                const int head = rem / upr, d0 = (rem - head * upr) * dpu + 2 * lane;
+                if (2 * lane >= dpu) continue;
+                const bool isq = head < p.H, isk = !isq && head < p.H + p.KVH;
+                const int half_hd = hd >> 1;
+                const int pd0 = d0 < half_hd ? d0 + half_hd : d0 - half_hd;
+                const int f0 = head * hd + d0, t = f0 / kTileN;
+                const int col = f0 - t * kTileN, pcol = head * hd + pd0 - t * kTileN;
+                int ca, cb;
+                tile_ctas(gq, t, ca, cb);
+                float2 x = make_float2(0.f, 0.f), xp = x;
+                for (int c0 = ca; c0 <= cb; c0 += 16) {  // 16 contributors' loads in flight, CTA order
+                    float2 a[16], b2[16];
+#pragma unroll
+                    for (int k = 0; k < 16; ++k) {
+                        const bool ok = c0 + k <= cb;
+                        const float *src = p.gpart + ((int64_t)(c0 + k + t) * p.rows_cap + r) * kTileN;
+                        a[k] = ok ? __ldcg(reinterpret_cast<const float2 *>(src + col)) : make_float2(0.f, 0.f);
+                        b2[k] = (ok && !(head >= p.H + p.KVH)) ? __ldcg(reinterpret_cast<const float2 *>(src + pcol))
+                                                               : make_float2(0.f, 0.f);
+                    }
+#pragma unroll
+                    for (int k = 0; k < 16; ++k) {
+                        x.x += a[k].x; x.y += a[k].y;
+                        xp.x += b2[k].x; xp.y += b2[k].y;
+                    }
+                }
+                const int pos = __ldg(&p.c.row_pos[r]);
+                const float rs = S.rstd[r] * (isq ? p.scale_log2 : 1.f);
+                float y0 = x.x, y1 = x.y;
+                if (isq || isk) {  // rotate the pairs (i, i + hd/2)
+                    const int fr = d0 < half_hd ? d0 : pd0;
+                    const float2 c0r = __ldg(&p.rope[(int64_t)pos * half_hd + fr]);
+                    const float2 c1r = __ldg(&p.rope[(int64_t)pos * half_hd + fr + 1]);
+                    if (d0 < half_hd) {
+                        y0 = x.x * c0r.x - xp.x * c0r.y;
+                        y1 = x.y * c1r.x - xp.y * c1r.y;
+                    } else {
+                        y0 = x.x * c0r.x + xp.x * c0r.y;
+                        y1 = x.y * c1r.x + xp.y * c1r.y;
+                    }
+                }
+                const uint16_t h0 = f32_to_f16_sat(y0 * rs), h1 = f32_to_f16_sat(y1 * rs);
+                *reinterpret_cast<uint32_t *>(p.qkv16 + (int64_t)r * p.nqkv + head * hd + d0) =
+                    (uint32_t)h0 | ((uint32_t)h1 << 16);
+                if (!isq) {  // the new position's k / v into the cache (blocked layout)
+                    const int kvh = head - p.H - (isk ? 0 : p.KVH);
+                    const int slot = __ldg(&p.c.row_slot[r]);
+                    uint8_t *blk = p.kv + l * p.kv_layer + (int64_t)slot * p.kv_slot +
+                                   ((int64_t)kvh * p.kv_nblk + pos / kKVPos) * kKVBlockBytes;
+                    const int pp = pos % kKVPos;
+                    if (isk) {
+                        *reinterpret_cast<uint32_t *>(blk + kv_k_off(pp, d0)) = (uint32_t)h0 | ((uint32_t)h1 << 16);
+                    } else {
+                        *reinterpret_cast<uint16_t *>(blk + kv_v_off(pp, d0)) = h0;
+                        *reinterpret_cast<uint16_t *>(blk + kv_v_off(pp, d0 + 1)) = h1;
+                    }
+                }
+            }
+            arrive(base + kPhFinQ, false);
+        }
         // ------------------------------------------------------------ attention
         {
-            // nothing below depends on the QKV phase until the partial sums: the RMS scales
-            // (from the previous layer's finalisation, complete before QKV could start) and
-            // the units' metadata and rotary entries (read-only; touched so they sit in L1)
-            wait_phase(base - 1);
-            load_rstd(p.ssqA);
             int64_t a0, a1;
             att_range(p, S.n_items, a0, a1);
             const int n = (int)(a1 - a0);
             const uint32_t wb = wi;
-            if (n > 0 && ctid < 128) {
-                const AttUnit u = att_unit(p, a0 + (ctid & 1) * (n > 1 ? 1 : 0));
-                const float2 c = __ldg(p.rope + (int64_t)(u.ctx - 1) * (hd / 2) + ((ctid >> 1) & 63) % (hd / 2));
-                if (c.x == 12345.f) S.last_flag = 0;  // keeps the loads
-            }
-            wait_phase(base + 0);
+            wait_phase(base + kPhFinQ);
             const bool det_layer = l == min(2, p.layers - 1);
             if (det_layer && ctid == 0) MEGA_DETAIL(13);
             if (det_layer && ctid == 0) MEGA_DETAIL(14);
@@ -755,52 +773,38 @@ __device__ __forceinline__ void mega_compute(const MegaParams &p, MegaSmem &S, u
             const int hb = 2 + half;     // this group's named barrier
             const int ht = ctid & 127;   // thread index within the group
             const int hq = ht >> 5;      // warp within the group (owns TMEM lanes 32 hq..)
-            const bool kv_spare = Gq <= 6;  // spare q-tile threads build k, v in parallel
             for (int i = half ? 1 - (gi & 1) : (gi & 1); i < n; i += 2) {
                 const AttUnit u = att_unit(p, a0 + i);
                 const int gidx = gi + i, b = half;  // (gidx & 1) == half
                 const uint32_t ph = (uint32_t)((gidx >> 1) & 1);
-                const float rs = S.rstd[u.row];
-                const float2 *cs = p.rope + (int64_t)(u.ctx - 1) * (hd / 2);
-                // ---- q tile rows 0..7 (score columns 8..15 are unused) and k, v
+                const uint16_t *qr = p.qkv16 + (int64_t)u.row * p.nqkv;
+                // ---- q tile rows 0..7 (score columns 8..15 are unused) and, on a row's last
+                // split, the new position's k, v patched into the prefetched block (the copy
+                // may predate their append to the cache)
                 {
                     const int g = ht >> 4, j = ht & 15;
-                    const bool is_q = g < Gq && j * 8 < hd;
-                    if (is_q) {
-                        float y[8];
-                        head_granule(p, gq, u.row, u.kvh * Gq + g, j, hd, cs, true, rs * p.scale_log2, y);
-                        *reinterpret_cast<uint4 *>(sQ + 4096 * b + (j >> 3) * 2048 + g * 128 + (((j & 7) ^ (g & 7)) << 4)) =
-                            pack_f16x8(y);
-                    } else {
-                        *reinterpret_cast<uint4 *>(sQ + 4096 * b + (j >> 3) * 2048 + g * 128 + (((j & 7) ^ (g & 7)) << 4)) =
-                            make_uint4(0, 0, 0, 0);
-                    }
-                    const int kvt = kv_spare ? ht - 96 : ht;  // 0..15 k granules, 16..31 v granules
-                    if (u.last && kvt >= 0 && kvt < 32) {
-                        const int jj = kvt & 15;
-                        const bool isv = kvt >= 16;
+                    uint4 qv = make_uint4(0, 0, 0, 0);
+                    if (g < Gq && j * 8 < hd)
+                        qv = __ldcg(reinterpret_cast<const uint4 *>(qr + (u.kvh * Gq + g) * hd + j * 8));
+                    *reinterpret_cast<uint4 *>(sQ + 4096 * b + (j >> 3) * 2048 + g * 128 + (((j & 7) ^ (g & 7)) << 4)) = qv;
+                    if (u.last && ht < 32) {
+                        const int jj = ht & 15;
+                        const bool isv = ht >= 16;
                         if (jj * 8 < hd) {
                             const int pp = u.ctx - 1 - u.p0;
-                            const int head = p.H + (isv ? p.KVH : 0) + u.kvh;
-                            float y[8];
-                            head_granule(p, gq, u.row, head, jj, hd, cs, !isv, rs, y);
-                            uint8_t *gblk = kv_block(p, l, u);
+                            const uint4 kv4 = __ldcg(reinterpret_cast<const uint4 *>(
+                                qr + (p.H + (isv ? p.KVH : 0) + u.kvh) * hd + jj * 8));
                             const uint32_t ws = wb + 2 * i + (isv ? 1 : 0);
                             mwait(&S.wfull[ws % kWSlots], (ws / kWSlots) & 1, err, ab);
                             uint8_t *slot = sW + (size_t)(ws % kWSlots) * kSlotBytes;
                             if (!isv) {
-                                const uint4 kp = pack_f16x8(y);
-                                const int off = kv_k_off(pp, jj * 8);
-                                *reinterpret_cast<uint4 *>(gblk + off) = kp;
-                                *reinterpret_cast<uint4 *>(slot + off) = kp;
+                                *reinterpret_cast<uint4 *>(slot + kv_k_off(pp, jj * 8)) = kv4;
                             } else {
+                                const uint32_t w4[4] = {kv4.x, kv4.y, kv4.z, kv4.w};
 #pragma unroll
-                                for (int e = 0; e < 8; ++e) {
-                                    const uint16_t hv = f32_to_f16_sat(y[e]);
-                                    const int off = kv_v_off(pp, jj * 8 + e);
-                                    *reinterpret_cast<uint16_t *>(gblk + off) = hv;
-                                    *reinterpret_cast<uint16_t *>(slot + off - 32768) = hv;
-                                }
+                                for (int e = 0; e < 8; ++e)
+                                    *reinterpret_cast<uint16_t *>(slot + kv_v_off(pp, jj * 8 + e) - 32768) =
+                                        (uint16_t)(w4[e >> 1] >> (16 * (e & 1)));
                             }
                         }
                     }
@@ -821,9 +825,7 @@ __device__ __forceinline__ void mega_compute(const MegaParams &p, MegaSmem &S, u
 #pragma unroll
                     for (int g = 0; g < 8; ++g) {
                         sv[g] = valid ? sv[g] : -INFINITY;
-                        float m = sv[g];
-#pragma unroll
-                        for (int o = 16; o > 0; o >>= 1) m = fmaxf(m, __shfl_xor_sync(0xffffffffu, m, o));
+                        const float m = warp_max_redux(sv[g]);
                         if (lane == 0) S.red[half][quarter][g] = m;
                     }
                     tc_fence_before();
@@ -837,7 +839,7 @@ __device__ __forceinline__ void mega_compute(const MegaParams &p, MegaSmem &S, u
                         const float e = valid ? exp2f(sv[g] - M[g]) : 0.f;
                         *reinterpret_cast<uint16_t *>(pb + g * 128 + ((((pc >> 3) ^ (g & 7)) << 4) | ((pc & 7) << 1))) =
                             f32_to_f16_sat(e);
-                        const float se = warp_sum(e);
+                        const float se = warp_sum_unit_redux(e);
                         if (lane == 0) S.red2[half][quarter][g] = se;
                     }
                     fence_proxy_async_smem();
@@ -950,7 +952,7 @@ __device__ __forceinline__ void mega_compute(const MegaParams &p, MegaSmem &S, u
             gi += n;
             i_unit = 0;
             DETAIL(8);
-            arrive(base + 1, true);
+            arrive(base + kPhAtt, true);
             DETAIL(9);
 #undef DETAIL
         }
@@ -958,22 +960,22 @@ __device__ __forceinline__ void mega_compute(const MegaParams &p, MegaSmem &S, u
         gemm_range(go, u0, u1);
         gemm_epi(go, u0, u1);
         wi += (uint32_t)(u1 - u0);
-        arrive(base + 2, false);
+        arrive(base + kPhO, false);
         // ------------------------------------------------------------ residual, MLP norm input
-        wait_phase(base + 2);
+        wait_phase(base + kPhO);
         if (l == min(2, p.layers - 1) && ctid == 0) MEGA_DETAIL(10);
         fin_resid(&go, p.mlp_norm + (int64_t)l * d, p.ssqM);
         if (l == min(2, p.layers - 1) && ctid == 0) MEGA_DETAIL(11);
-        arrive(base + 3, true);
+        arrive(base + kPhFinO, true);
         if (l == min(2, p.layers - 1) && ctid == 0) MEGA_DETAIL(12);
         // ------------------------------------------------------------ gate / up
         gemm_range(gu, u0, u1);
         gemm_epi(gu, u0, u1);
         wi += (uint32_t)(u1 - u0);
-        arrive(base + 4, false);
+        arrive(base + kPhGU, false);
         // ------------------------------------------------------------ SwiGLU
         {
-            wait_phase(base + 4);
+            wait_phase(base + kPhGU);
             load_rstd(p.ssqM);
             const int fb = p.F / 128;
             // unit = (row, 128 features of h) = one 256-row tile of the gate/up outputs; lane:
@@ -1028,17 +1030,17 @@ __device__ __forceinline__ void mega_compute(const MegaParams &p, MegaSmem &S, u
                         make_uint2((uint32_t)hl[0] | ((uint32_t)hl[1] << 16), (uint32_t)hl[2] | ((uint32_t)hl[3] << 16));
                 }
             }
-            arrive(base + 5, true);
+            arrive(base + kPhFinGU, true);
         }
         // ------------------------------------------------------------ down
         gemm_range(gdn, u0, u1);
         gemm_epi(gdn, u0, u1);
         wi += (uint32_t)(u1 - u0);
-        arrive(base + 6, false);
+        arrive(base + kPhDown, false);
         // ------------------------------------------------------------ residual, next norm input
-        wait_phase(base + 6);
+        wait_phase(base + kPhDown);
         fin_resid(&gdn, (l + 1 < p.layers) ? p.attn_norm + (int64_t)(l + 1) * d : p.final_norm, p.ssqA);
-        arrive(base + 7, true);
+        arrive(base + kPhFinD, true);
     }
 
     // ---------------------------------------------------------------- lm_head

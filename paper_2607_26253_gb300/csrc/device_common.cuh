@@ -278,6 +278,23 @@ __device__ __forceinline__ void named_bar_sync(int id, int nthreads) {
     asm volatile("bar.sync %0, %1;" ::"r"(id), "r"(nthreads) : "memory");
 }
 
+// Warp maximum of a float in one redux.sync: floats mapped to order-preserving signed ints.
+__device__ __forceinline__ float warp_max_redux(float v) {
+    int k = __float_as_int(v);
+    k ^= (k >> 31) & 0x7fffffff;
+    int m;
+    asm volatile("redux.sync.max.s32 %0, %1, 0xffffffff;" : "=r"(m) : "r"(k));
+    m ^= (m >> 31) & 0x7fffffff;
+    return __int_as_float(m);
+}
+// Warp sum of values in [0, 1] in one redux.sync, as 2^-24 fixed point (exact for 32 lanes).
+__device__ __forceinline__ float warp_sum_unit_redux(float v) {
+    const unsigned q = (unsigned)__float2uint_rn(v * 16777216.0f);
+    unsigned s;
+    asm volatile("redux.sync.add.u32 %0, %1, 0xffffffff;" : "=r"(s) : "r"(q));
+    return (float)s * 5.9604644775390625e-08f;
+}
+
 __device__ __forceinline__ float warp_sum(float v) {
 #pragma unroll
     for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);

@@ -82,6 +82,7 @@ struct sara_handle {
     float *dx = nullptr, *ssqA = nullptr, *ssqM = nullptr;
     uint8_t *xg_hi = nullptr, *xg_lo = nullptr, *att_hi = nullptr, *att_lo = nullptr, *h_hi = nullptr, *h_lo = nullptr;
     float *gpart = nullptr;  // GEMM partial tiles of the decode step
+    uint16_t *qkv16 = nullptr;  // the step's q (scaled), k, v in fp16
     int gp_qkv = 0, gp_o = 0;
     unsigned long long *phase_cnt = nullptr;  // [1 + 8 layers + 1] then the epoch
     int n_phase_cnt = 0;
@@ -363,6 +364,7 @@ MegaParams mega_params(const sara_handle &h) {
     p.ssqA = h.ssqA;
     p.ssqM = h.ssqM;
     p.gpart = h.gpart;
+    p.qkv16 = h.qkv16;
     p.gp_qkv = h.gp_qkv;
     p.gp_o = h.gp_o;
     p.part = h.attn_part;
@@ -586,6 +588,7 @@ void alloc_decode(sara_handle &h) {
     // partial tiles: one segment per (CTA, tile) pair of a phase, at most CTAs + tiles - 1
     const int tmax = std::max({nqkv, d, 2 * F}) / kTileN + 1;
     h.gpart = h.mem.alloc<float>((size_t)(h.sms + tmax) * S * kTileN, false);
+    h.qkv16 = h.mem.alloc<uint16_t>((size_t)S * nqkv, false);
     // the QKV and O projections are spread over few CTAs (each about one ring of weights)
     auto small = [&](int N, int K) {
         const int units = ((N + kTileN - 1) / kTileN) * (K / 64);
@@ -945,7 +948,7 @@ void print_stamps(sara_handle &h, int rows, int ctx) {
     for (int ph = 0; ph < NPH; ++ph) done[ph] = stat(ph, 0, true);
     fprintf(stderr, "rows %d ctx %d: start->embed done %.2f us, lm_head done at %.2f us\n", rows, ctx, done[0],
             done[NPH - 1]);
-    const char *names[8] = {"QKV", "ATT", "O", "FIN_O", "GU", "FIN_GU", "DOWN", "FIN_D"};
+    const char *names[kPhasesPerLayer] = {"QKV", "FIN_Q", "ATT", "O", "FIN_O", "GU", "FIN_GU", "DOWN", "FIN_D"};
     const int l0 = L > 4 ? 2 : 0, l1 = L > 4 ? L - 2 : L;
     for (int k = 0; k < kPhasesPerLayer; ++k) {
         double span = 0, obs = 0, wahead = 0, mma = 0;
