@@ -227,7 +227,9 @@ static __device__ void ctl_round_setup(const StepConst &K, StepVars &V, const St
     __syncthreads();
     if (R > c.max_seqs) { if (threadIdx.x == 0) report_error(&V.err, ERR_CAPACITY); return; }
     // first decode step: input = last prompt token at position Lp - 1
-    const int nsplit = (Lp + K.attn_chunk - 1) / K.attn_chunk;
+    const int nblk = (Lp + K.attn_chunk - 1) / K.attn_chunk;
+    const int span = att_span_for((int64_t)R * nblk, K.att_slots);
+    const int nsplit = (nblk + span - 1) / span;
     int maxL = 0;
     for (int r = threadIdx.x; r < R; r += kCtlThreads) {
         const int q = c.seq_q[r];
@@ -256,6 +258,7 @@ static __device__ void ctl_round_setup(const StepConst &K, StepVars &V, const St
     if (threadIdx.x == 0) {
         V.live = R;
         V.att_items = R * nsplit;
+        V.att_span = span;
         V.pre_rows = pre_rows;
         V.n_fresh = n_fresh;
         V.round_maxL = maxL;

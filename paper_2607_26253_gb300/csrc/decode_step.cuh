@@ -44,7 +44,7 @@
 // 128-byte-swizzled K-major form the tensor core reads):
 //   weights       tiles of 256 rows (the last may have 128): [N/256][K/64][rows][64],
 //                 16-byte granule j of row r at granule j ^ (r % 8)
-//   activations   [K/64][rows16][64] bf16 (hi and lo planes), same swizzle
+//   activations   [K/64][2 rows16][64] bf16, 8-row groups alternating hi / lo parts, same swizzle
 //   KV cache      per (layer, slot, kv head, 128-position block): K as [d/64][128 pos][64 d]
 //                 and V transposed as [pos/64][128 d][64 pos], fp16, head dim padded to 128
 #pragma once
@@ -55,9 +55,10 @@ namespace sara {
 
 constexpr int kMegaThreads = 352;
 constexpr int kMegaCThreads = 256;  // compute warps 3..10
-constexpr int kWSlots = 4;
+constexpr int kMaxWSlots = 5;
+constexpr int kDetailRows = 16;  // profiling builds: rows of 4 detail stamps per CTA
 constexpr int kSlotBytes = 32768;
-constexpr int kXRingBytes = 65536;
+constexpr int kRingBytes = 4 * 32768 + 65536;  // W slots + X stages share it
 constexpr int kMaxXStages = 8;
 constexpr int kTileN = 256;           // weight rows (output features) per GEMM tile
 constexpr int kKVPos = 128;           // positions per KV block and per attention split
@@ -90,9 +91,9 @@ struct MegaParams {
     int rows_cap, rows_cap16;
     int gp_qkv, gp_o;                               // CTAs taking part in the QKV / O projections
     float *x;                                       // [rows_cap][d] residual stream
-    uint8_t *xg_hi, *xg_lo;                         // blocked [d/64][rows_cap16][64]
-    uint8_t *att_hi, *att_lo;                       // blocked [H*hd/64][rows_cap16][64]
-    uint8_t *h_hi, *h_lo;                           // blocked [F/64][rows_cap16][64]
+    uint8_t *xg;                                    // pair-blocked [d/64][2 rows_cap16][64]
+    uint8_t *att;                                   // pair-blocked [H*hd/64][2 rows_cap16][64]
+    uint8_t *hm;                                    // pair-blocked [F/64][2 rows_cap16][64]
     float *ssqA, *ssqM;                             // [d/64][rows_cap] partial sums of x^2
     float *gpart;                                   // [segments][rows_cap][256] GEMM partial tiles
     uint16_t *qkv16;                                // [rows_cap][nqkv] fp16 q (scaled), k, v of the step
@@ -113,13 +114,15 @@ struct MegaParams {
     do {                                                                                                  \
         if (p.stamps) p.stamps[((size_t)blockIdx.x * p.n_stamp_ph + (ph)) * 4 + (kind)] = globaltimer_ns(); \
     } while (0)
-// Detail stamps of the attention and first finalize phases of one layer (layer 2), first
-// unit of each CTA: the last four phase slots of the same array (the fifth-last holds the
-// kernel start).
-#define MEGA_DETAIL(i)                                                                                          \
-    do {                                                                                                        \
-        if (p.stamps) p.stamps[((size_t)blockIdx.x * p.n_stamp_ph + p.n_stamp_ph - 4 + ((i) >> 2)) * 4 + ((i) & 3)] = \
-                          globaltimer_ns();                                                                       \
+// Detail stamps of one layer (layer 2): the attention and first finalize phases (first unit
+// of each CTA, ids 0-15) and the first 12 units of the gate / up GEMM (ids 16-63: W copy
+// issued, W slot full and X stage full as seen by the MMA issuer, MMAs committed); the last
+// kDetailRows phase slots of the same array (the one before them holds the kernel start).
+#define MEGA_DETAIL(i)                                                                                    \
+    do {                                                                                                  \
+        if (p.stamps)                                                                                     \
+            p.stamps[((size_t)blockIdx.x * p.n_stamp_ph + p.n_stamp_ph - kDetailRows + ((i) >> 2)) * 4 + \
+                     ((i) & 3)] = globaltimer_ns();                                                       \
     } while (0)
 #else
 #define MEGA_STAMP(ph, kind) \
@@ -131,7 +134,7 @@ struct MegaParams {
 #endif
 
 struct MegaSmem {
-    uint64_t wfull[kWSlots], wempty[kWSlots];
+    uint64_t wfull[kMaxWSlots], wempty[kMaxWSlots];
     uint64_t xfull[kMaxXStages], xempty[kMaxXStages];
     uint64_t acc_full[2], acc_empty[2];
     uint64_t q_ready[2], s_full[2], p_ready[2], o_full[2];
@@ -140,9 +143,8 @@ struct MegaSmem {
     uint32_t tmem_base;
     int abort;
     int last_flag;
-    int rows, rows16, nx, n_items;
+    int rows, rows16, nws, nx, n_items, att_span;
     float rstd[128];
-    float att_m[2][8], att_l[2][8];
     float red[2][4][8], red2[2][4][8];  // per warp group: attention max / sum reductions
     float mw[2][8][kMegaMaxSplits];      // per warp group: split weights of a merge
     float ml[2][8];
@@ -150,13 +152,20 @@ struct MegaSmem {
 };
 
 constexpr size_t kMegaSmemBytes =
-    1024 + (size_t)kWSlots * kSlotBytes + kXRingBytes + 4 * 4096 + sizeof(MegaSmem);
+    1024 + (size_t)kRingBytes + 4 * 4096 + sizeof(MegaSmem);
 
 // ------------------------------------------------------------------------------ layouts
-// Byte offset of element (r, k) of a blocked activation plane with rows16 rows per chunk.
+// Pair-blocked activation (a GEMM operand held as bf16 hi + lo parts): per 64-wide k-chunk,
+// 2 rows16 rows of 128 B (64 bf16, 128-byte swizzle) in 8-row groups that alternate between
+// the hi parts of rows 8g..8g+7 and their lo parts.  Byte offset of the hi part of element
+// (r, k); the lo part sits kLoOff bytes after it.  One MMA over the chunk's first 2 R16 rows
+// multiplies hi and lo parts at once (rows16 <= 64); with a 2048-byte group stride the hi
+// (lo) groups alone form a 128-row operand.
+constexpr int kLoOff = 1024;
 __host__ __device__ __forceinline__ int64_t xblk_off(int r, int k, int rows16) {
     const int chunk = k >> 6, col = k & 63;
-    return ((int64_t)chunk * rows16 + r) * 128 + ((((col >> 3) ^ (r & 7)) << 4) | ((col & 7) << 1));
+    return ((int64_t)chunk * 2 * rows16 + 16 * (r >> 3) + (r & 7)) * 128 +
+           ((((col >> 3) ^ (r & 7)) << 4) | ((col & 7) << 1));
 }
 // Byte offsets of K(pp, d) and V(pp, d) inside one 128-position KV block.
 __host__ __device__ __forceinline__ int kv_k_off(int pp, int d) {
@@ -218,7 +227,7 @@ __device__ __forceinline__ bool spin_counter(const unsigned long long *cnt, unsi
 struct GemmPh {
     const uint8_t *w;
     int N, K, kch, T, Gp;
-    const uint8_t *xhi, *xlo;
+    const uint8_t *x;  // pair-blocked operand
     bool whole;  // whole tiles per CTA (lm_head: the argmax of a tile is finished in one CTA)
 };
 
@@ -228,15 +237,15 @@ __device__ __forceinline__ GemmPh gemm_phase(const MegaParams &p, int l, int k) 
     g.whole = false;
     g.Gp = gridDim.x;
     if (l == p.layers) {
-        g.w = p.w_lm; g.N = p.V; g.K = p.d; g.xhi = p.xg_hi; g.xlo = p.xg_lo; g.whole = true;
+        g.w = p.w_lm; g.N = p.V; g.K = p.d; g.x = p.xg; g.whole = true;
     } else if (k == kPhQKV) {
-        g.w = p.w_qkv + l * p.ls_qkv; g.N = p.nqkv; g.K = p.d; g.xhi = p.xg_hi; g.xlo = p.xg_lo; g.Gp = p.gp_qkv;
+        g.w = p.w_qkv + l * p.ls_qkv; g.N = p.nqkv; g.K = p.d; g.x = p.xg; g.Gp = p.gp_qkv;
     } else if (k == kPhO) {
-        g.w = p.w_o + l * p.ls_o; g.N = p.d; g.K = p.H * p.hd; g.xhi = p.att_hi; g.xlo = p.att_lo; g.Gp = p.gp_o;
+        g.w = p.w_o + l * p.ls_o; g.N = p.d; g.K = p.H * p.hd; g.x = p.att; g.Gp = p.gp_o;
     } else if (k == kPhGU) {
-        g.w = p.w_gu + l * p.ls_gu; g.N = 2 * p.F; g.K = p.d; g.xhi = p.xg_hi; g.xlo = p.xg_lo;
+        g.w = p.w_gu + l * p.ls_gu; g.N = 2 * p.F; g.K = p.d; g.x = p.xg;
     } else {
-        g.w = p.w_down + l * p.ls_down; g.N = p.d; g.K = p.F; g.xhi = p.h_hi; g.xlo = p.h_lo;
+        g.w = p.w_down + l * p.ls_down; g.N = p.d; g.K = p.F; g.x = p.hm;
     }
     g.kch = g.K / 64;
     g.T = (g.N + kTileN - 1) / kTileN;
@@ -280,11 +289,13 @@ __device__ __forceinline__ void tile_ctas(const GemmPh &g, int t, int &ca, int &
     cb = unit_owner((t + 1) * g.kch - 1, U, g.Gp);
 }
 
+// Attention unit: one split of one row for one kv head.  Split sp covers the `span` KV
+// blocks from block sp * span on: positions [p0, p0 + n) of the row's ctx, in nb blocks.
 struct AttUnit {
-    int item, kvh, row, sp, ctx, p0, n, nsplit, slot;
+    int item, kvh, row, sp, ctx, p0, n, nb, nsplit, slot;
     bool last;
 };
-__device__ __forceinline__ AttUnit att_unit(const MegaParams &p, int64_t a) {
+__device__ __forceinline__ AttUnit att_unit(const MegaParams &p, int64_t a, int span) {
     AttUnit u;
     u.item = (int)(a / p.KVH);
     u.kvh = (int)(a - (int64_t)u.item * p.KVH);
@@ -292,9 +303,10 @@ __device__ __forceinline__ AttUnit att_unit(const MegaParams &p, int64_t a) {
     u.row = it.x;
     u.sp = it.y;
     u.ctx = __ldg(&p.c.row_pos[u.row]) + 1;
-    u.p0 = u.sp * kKVPos;
-    u.n = min(u.ctx - u.p0, kKVPos);
-    u.nsplit = (u.ctx + kKVPos - 1) / kKVPos;
+    u.p0 = u.sp * span * kKVPos;
+    u.n = min(u.ctx - u.p0, span * kKVPos);
+    u.nb = (u.n + kKVPos - 1) / kKVPos;
+    u.nsplit = ((u.ctx + kKVPos - 1) / kKVPos + span - 1) / span;
     u.last = u.p0 + u.n == u.ctx;
     u.slot = __ldg(&p.c.row_slot[u.row]);
     return u;
@@ -307,8 +319,10 @@ __device__ __forceinline__ void att_range(const MegaParams &p, int n_items, int6
     a0 = v * NU / G;
     a1 = (v + 1) * NU / G;
 }
-__device__ __forceinline__ uint8_t *kv_block(const MegaParams &p, int l, const AttUnit &u) {
-    return p.kv + l * p.kv_layer + (int64_t)u.slot * p.kv_slot + ((int64_t)u.kvh * p.kv_nblk + u.sp) * kKVBlockBytes;
+// Block j of unit u in layer l's KV cache.
+__device__ __forceinline__ uint8_t *kv_block(const MegaParams &p, int l, const AttUnit &u, int j) {
+    return p.kv + l * p.kv_layer + (int64_t)u.slot * p.kv_slot +
+           ((int64_t)u.kvh * p.kv_nblk + u.p0 / kKVPos + j) * kKVBlockBytes;
 }
 
 // ------------------------------------------------------------------------------ W producer
@@ -316,10 +330,11 @@ __device__ __forceinline__ void mega_w_producer(const MegaParams &p, MegaSmem &S
     volatile int *ab = &S.abort;
     int *err = &p.c.v->err;
     const uint64_t pol = l2_policy_evict_first();
+    const uint32_t nws = (uint32_t)S.nws;
     uint32_t wi = 0;
     bool ok = true;
     auto acquire = [&](uint32_t i) -> bool {
-        return i < kWSlots || mwait(&S.wempty[i % kWSlots], ((i / kWSlots) & 1) ^ 1, err, ab);
+        return i < nws || mwait(&S.wempty[i % nws], ((i / nws) & 1) ^ 1, err, ab);
     };
     for (int l = 0; l <= p.layers && ok; ++l) {
         for (int gp = 0; gp < 4 && ok; ++gp) {
@@ -330,43 +345,68 @@ __device__ __forceinline__ void mega_w_producer(const MegaParams &p, MegaSmem &S
             gemm_range(g, u0, u1);
             for (int64_t u = u0; u < u1; ++u, ++wi) {
                 if (!acquire(wi)) { ok = false; break; }
-                const int s = (int)(wi % kWSlots);
+                const int s = (int)(wi % nws);
                 const int t = (int)(u / g.kch), kc = (int)(u - (int64_t)t * g.kch);
                 const uint32_t bytes = (uint32_t)tile_rows(g, t) * 128;
                 mbar_arrive_expect_tx(&S.wfull[s], bytes);
                 bulk_load(sW + (size_t)s * kSlotBytes, g.w + wblk_off(g.N, g.K, t, kc), bytes, &S.wfull[s], pol);
+                if (k == kPhGU && l == min(2, p.layers - 1) && u - u0 < 12) MEGA_DETAIL(16 + (int)(u - u0));
             }
             MEGA_STAMP(1 + kPhasesPerLayer * l + k, 2);
             if (k == 0 && l < p.layers && ok) {
-                // the attention phase's KV blocks follow the QKV weights in ring order:
-                // slot 1 = K (d < 64 | d >= 64), slot 2 = V^T (positions < 64 | >= 64)
+                // the attention phase's KV blocks follow the QKV weights in ring order: unit
+                // pairs (one unit per compute warp group), block by block, K then V^T of the
+                // pair's first unit, then of its second; each one ring entry (K: d < 64 |
+                // d >= 64 halves, V^T: positions < 64 | >= 64).  The block holding a row's
+                // new position is copied once the q / k / v phase has appended it to the cache.
                 int64_t a0, a1;
                 att_range(p, S.n_items, a0, a1);
-                for (int64_t a = a0; a < a1 && ok; ++a) {
-                    const AttUnit u = att_unit(p, a);
-                    const uint8_t *blk = kv_block(p, l, u);
-                    const uint32_t kb = (uint32_t)(((u.n + 7) & ~7) * 128), vb = (uint32_t)(p.hd * 128);
-                    if (!acquire(wi)) { ok = false; break; }
-                    int s = (int)(wi % kWSlots);
-                    mbar_arrive_expect_tx(&S.wfull[s], p.hd > 64 ? 2 * kb : kb);
-                    bulk_load(sW + (size_t)s * kSlotBytes, blk, kb, &S.wfull[s], pol);
-                    if (p.hd > 64) bulk_load(sW + (size_t)s * kSlotBytes + 16384, blk + 16384, kb, &S.wfull[s], pol);
-                    ++wi;
-                    if (!acquire(wi)) { ok = false; break; }
-                    s = (int)(wi % kWSlots);
-                    mbar_arrive_expect_tx(&S.wfull[s], u.n > 64 ? 2 * vb : vb);
-                    bulk_load(sW + (size_t)s * kSlotBytes, blk + 32768, vb, &S.wfull[s], pol);
-                    if (u.n > 64) bulk_load(sW + (size_t)s * kSlotBytes + 16384, blk + 49152, vb, &S.wfull[s], pol);
-                    ++wi;
+                const int span = S.att_span;
+                bool finq_seen = false;
+                for (int64_t a = a0; a < a1 && ok; a += 2) {
+                    const bool two = a + 1 < a1;
+                    const AttUnit ua = att_unit(p, a, span);
+                    const AttUnit ub = two ? att_unit(p, a + 1, span) : ua;
+                    const int nbb = two ? ub.nb : 0;
+                    for (int j = 0; j < max(ua.nb, nbb) && ok; ++j) {
+                        for (int w = 0; w < 2 && ok; ++w) {
+                            const AttUnit &u = w ? ub : ua;
+                            if (j >= (w ? nbb : ua.nb)) continue;
+                            if (u.last && j == u.nb - 1 && !finq_seen) {
+                                if (!spin_counter(&p.cnt[(1 + kPhasesPerLayer * l + kPhFinQ) * kCntStride], S.target,
+                                                  err, ab)) {
+                                    ok = false;
+                                    break;
+                                }
+                                fence_proxy_async_global();
+                                finq_seen = true;
+                            }
+                            const uint8_t *blk = kv_block(p, l, u, j);
+                            const int nj = min(kKVPos, u.n - j * kKVPos);
+                            const uint32_t kb = (uint32_t)(((nj + 7) & ~7) * 128), vb = (uint32_t)(p.hd * 128);
+                            if (!acquire(wi)) { ok = false; break; }
+                            int s = (int)(wi % nws);
+                            mbar_arrive_expect_tx(&S.wfull[s], p.hd > 64 ? 2 * kb : kb);
+                            bulk_load(sW + (size_t)s * kSlotBytes, blk, kb, &S.wfull[s], pol);
+                            if (p.hd > 64) bulk_load(sW + (size_t)s * kSlotBytes + 16384, blk + 16384, kb, &S.wfull[s], pol);
+                            ++wi;
+                            if (!acquire(wi)) { ok = false; break; }
+                            s = (int)(wi % nws);
+                            mbar_arrive_expect_tx(&S.wfull[s], nj > 64 ? 2 * vb : vb);
+                            bulk_load(sW + (size_t)s * kSlotBytes, blk + 32768, vb, &S.wfull[s], pol);
+                            if (nj > 64) bulk_load(sW + (size_t)s * kSlotBytes + 16384, blk + 49152, vb, &S.wfull[s], pol);
+                            ++wi;
+                        }
+                    }
                 }
                 MEGA_STAMP(1 + kPhasesPerLayer * l + kPhAtt, 2);
             }
         }
     }
     if (!ok) {  // every copy already issued lands before the CTA exits
-        for (uint32_t s = 0; s < kWSlots && s < wi; ++s) {
-            const uint32_t last = ((wi - 1 - s) / kWSlots) * kWSlots + s;
-            mbar_wait(&S.wfull[s], (last / kWSlots) & 1, err);
+        for (uint32_t s = 0; s < nws && s < wi; ++s) {
+            const uint32_t last = ((wi - 1 - s) / nws) * nws + s;
+            mbar_wait(&S.wfull[s], (last / nws) & 1, err);
         }
     }
 }
@@ -377,8 +417,8 @@ __device__ __forceinline__ void mega_x_producer(const MegaParams &p, MegaSmem &S
     int *err = &p.c.v->err;
     const uint64_t pol = l2_policy_evict_last();
     const int NX = S.nx, R16 = S.rows16;
-    const uint32_t plane = (uint32_t)R16 * 128, stage = 2 * plane;
-    const int64_t chunk_stride = (int64_t)p.rows_cap16 * 128;
+    const uint32_t stage = (uint32_t)R16 * 256;  // hi + lo parts of the live rows' groups
+    const int64_t chunk_stride = (int64_t)p.rows_cap16 * 256;
     uint32_t xi = 0;
     bool ok = true;
     for (int l = 0; l <= p.layers && ok; ++l) {
@@ -400,9 +440,7 @@ __device__ __forceinline__ void mega_x_producer(const MegaParams &p, MegaSmem &S
                 if (xi >= (uint32_t)NX && !mwait(&S.xempty[s], ((xi / NX) & 1) ^ 1, err, ab)) { ok = false; break; }
                 const int kc = (int)(u % g.kch);
                 mbar_arrive_expect_tx(&S.xfull[s], stage);
-                uint8_t *dst = sX + (size_t)s * stage;
-                bulk_load(dst, g.xhi + kc * chunk_stride, plane, &S.xfull[s], pol);
-                bulk_load(dst + plane, g.xlo + kc * chunk_stride, plane, &S.xfull[s], pol);
+                bulk_load(sX + (size_t)s * stage, g.x + kc * chunk_stride, stage, &S.xfull[s], pol);
             }
         }
     }
@@ -420,14 +458,20 @@ __device__ __forceinline__ void mega_mma(const MegaParams &p, MegaSmem &S, uint8
     volatile int *ab = &S.abort;
     int *err = &p.c.v->err;
     const int NX = S.nx, R16 = S.rows16;
-    const uint32_t plane = (uint32_t)R16 * 128, stage = 2 * plane;
+    const uint32_t stage = (uint32_t)R16 * 256;
     const uint32_t ida = idesc_f16_f32(128, 16);
+    // at most 64 live rows: one MMA per k-step over the stacked hi / lo groups (M = 2 R16
+    // rounded up to 64 or 128: the rows past the stage only feed accumulator rows nobody
+    // reads); more: the hi and the lo groups as two 128-row operands into one accumulator
+    const bool stacked = R16 <= 64;
     uint32_t wi = 0, xi = 0;
     int gi = 0, use0 = 0, use1 = 0, lmseg = 0;  // accumulator buffer uses
     bool ok = true;
-    auto wslot = [&](uint32_t i) -> uint32_t { return smem_u32(sW + (size_t)(i % kWSlots) * kSlotBytes); };
-    auto wwait = [&](uint32_t i) -> bool { return mwait(&S.wfull[i % kWSlots], (i / kWSlots) & 1, err, ab); };
-    auto gemm = [&](const GemmPh &g, int64_t u0, int64_t u1) {
+    const uint32_t nws = (uint32_t)S.nws;
+    auto wslot = [&](uint32_t i) -> uint32_t { return smem_u32(sW + (size_t)(i % nws) * kSlotBytes); };
+    auto wwait = [&](uint32_t i) -> bool { return mwait(&S.wfull[i % nws], (i / nws) & 1, err, ab); };
+    auto gemm = [&](const GemmPh &g, int64_t u0, int64_t u1, bool det) {
+        const int64_t ub = u0;
         for (int64_t u = u0; u < u1 && ok;) {
             const int t = (int)(u / g.kch);
             const int64_t e = min(u1, (int64_t)(t + 1) * g.kch);
@@ -436,23 +480,32 @@ __device__ __forceinline__ void mega_mma(const MegaParams &p, MegaSmem &S, uint8
             if (use_a >= 1 && !mwait(&S.acc_empty[a], (use_a - 1) & 1, err, ab)) { ok = false; break; }
             tc_fence_after();
             const uint32_t d = tmem + (uint32_t)(a * kTileN);
-            // M = 64 when every live row fits: same cost, rows spread over all four lane quarters
-            const uint32_t idg = idesc_bf16_f32(R16 <= 64 ? 64u : 128u, (uint32_t)tile_rows(g, t));
+            const uint32_t idg = idesc_bf16_f32(R16 <= 32 ? 64u : 128u, (uint32_t)tile_rows(g, t));
             bool first = true;
             for (; u < e; ++u, ++wi, ++xi) {
                 const int xs = (int)(xi % NX);
-                if (!wwait(wi) || !mwait(&S.xfull[xs], (xi / NX) & 1, err, ab)) { ok = false; break; }
+                const bool dj = det && u - ub < 12;
+                if (!wwait(wi)) { ok = false; break; }
+                if (dj) MEGA_DETAIL(28 + (int)(u - ub));
+                if (!mwait(&S.xfull[xs], (xi / NX) & 1, err, ab)) { ok = false; break; }
+                if (dj) MEGA_DETAIL(40 + (int)(u - ub));
                 tc_fence_after();
                 const uint32_t aw = wslot(wi), ax = smem_u32(sX + (size_t)xs * stage);
 #pragma unroll
                 for (int kk = 0; kk < 4; ++kk) {
                     const uint64_t bd = sdesc_kmajor_sw128(aw + kk * 32);
-                    tc_mma_bf16(d, sdesc_kmajor_sw128(ax + kk * 32), bd, idg, (first && kk == 0) ? 0u : 1u);
-                    tc_mma_bf16(d, sdesc_kmajor_sw128(ax + plane + kk * 32), bd, idg, 1u);
+                    const uint32_t acc = (first && kk == 0) ? 0u : 1u;
+                    if (stacked) {
+                        tc_mma_bf16(d, sdesc_kmajor_sw128(ax + kk * 32), bd, idg, acc);
+                    } else {
+                        tc_mma_bf16(d, sdesc_kmajor_sw128(ax + kk * 32, 2048), bd, idg, acc);
+                        tc_mma_bf16(d, sdesc_kmajor_sw128(ax + kLoOff + kk * 32, 2048), bd, idg, 1u);
+                    }
                 }
                 first = false;
-                tc_commit(&S.wempty[wi % kWSlots]);
+                tc_commit(&S.wempty[wi % nws]);
                 tc_commit(&S.xempty[xs]);
+                if (dj) MEGA_DETAIL(52 + (int)(u - ub));
             }
             if (!ok) break;
             tc_commit(&S.acc_full[a]);
@@ -460,43 +513,63 @@ __device__ __forceinline__ void mega_mma(const MegaParams &p, MegaSmem &S, uint8
             if (g.whole) ++lmseg;
         }
     };
-    // attention units in pairs (one per compute warp group): S(i), S(i+1), PV(i), PV(i+1)
+    // attention: unit pairs (one unit per compute warp group, group (gi + i) & 1), block by
+    // block in lockstep: S(a, j), S(b, j), PV(a, j), PV(b, j).  S(x, j > 0) may overwrite the
+    // score buffer once PV(x, j - 1) was issued (the group had read the scores before it
+    // released P); PV(x, j) waits for P(x, j), which the group publishes only after reading
+    // O(x, j - 1).  Per group: units (q_ready) and blocks (s_full / p_ready / o_full) counted
+    // for the barrier parities.
+    uint32_t aq0 = 0, aq1 = 0, ab0 = 0, ab1 = 0;
     auto att = [&](int64_t a0, int64_t a1) {
-        const int n = (int)(a1 - a0);
-        const uint32_t wb = wi;
-        auto scores = [&](int i) -> bool {  // S = K q^T
-            const int g = gi + i, b = g & 1;
-            const uint32_t w0 = wb + 2 * i;
-            if (!mwait(&S.q_ready[b], (g >> 1) & 1, err, ab) || !wwait(w0)) return false;
+        const int n = (int)(a1 - a0), span = S.att_span;
+        uint32_t w = wi;
+        auto scores = [&](int b, uint32_t e, bool first_blk) -> bool {  // S = K q^T
+            uint32_t &cq = b ? aq1 : aq0;
+            if (first_blk) {
+                if (!mwait(&S.q_ready[b], cq & 1, err, ab)) return false;
+                ++cq;
+            }
+            if (!wwait(e)) return false;
             tc_fence_after();
-            const uint32_t dS = tmem + kTmemS + 16 * b, qb = smem_u32(sQ + 4096 * b), kb = wslot(w0);
+            const uint32_t dS = tmem + kTmemS + 16 * b, qb = smem_u32(sQ + 4096 * b), kb = wslot(e);
             for (int ks = 0; ks < p.hd / 16; ++ks)
                 tc_mma_bf16(dS, sdesc_kmajor_sw128(kb + (ks >> 2) * 16384 + (ks & 3) * 32),
                             sdesc_kmajor_sw128(qb + (ks >> 2) * 2048 + (ks & 3) * 32), ida, ks > 0 ? 1u : 0u);
             tc_commit(&S.s_full[b]);
-            tc_commit(&S.wempty[w0 % kWSlots]);
+            tc_commit(&S.wempty[e % nws]);
             return true;
         };
-        auto pv = [&](int i) -> bool {  // O^T = V^T P^T
-            const int g = gi + i, b = g & 1;
-            const uint32_t w1 = wb + 2 * i + 1;
-            const AttUnit u = att_unit(p, a0 + i);
-            if (!mwait(&S.p_ready[b], (g >> 1) & 1, err, ab) || !wwait(w1)) return false;
+        auto pv = [&](int b, uint32_t e, int nj) -> bool {  // O^T = V^T P^T
+            uint32_t &cb = b ? ab1 : ab0;
+            if (!mwait(&S.p_ready[b], cb & 1, err, ab)) return false;
+            ++cb;
+            if (!wwait(e)) return false;
             tc_fence_after();
-            const uint32_t dO = tmem + kTmemO + 16 * b, pb = smem_u32(sP + 4096 * b), vb = wslot(w1);
-            const int ksteps = (u.n + 15) >> 4;
+            const uint32_t dO = tmem + kTmemO + 16 * b, pb = smem_u32(sP + 4096 * b), vb = wslot(e);
+            const int ksteps = (nj + 15) >> 4;
             for (int ks = 0; ks < ksteps; ++ks)
                 tc_mma_bf16(dO, sdesc_kmajor_sw128(vb + (ks >> 2) * 16384 + (ks & 3) * 32),
                             sdesc_kmajor_sw128(pb + (ks >> 2) * 2048 + (ks & 3) * 32), ida, ks > 0 ? 1u : 0u);
             tc_commit(&S.o_full[b]);
-            tc_commit(&S.wempty[w1 % kWSlots]);
+            tc_commit(&S.wempty[e % nws]);
             return true;
         };
         for (int i = 0; i < n && ok; i += 2) {
             const bool two = i + 1 < n;
-            if (!scores(i) || (two && !scores(i + 1)) || !pv(i) || (two && !pv(i + 1))) ok = false;
+            const AttUnit ua = att_unit(p, a0 + i, span);
+            const AttUnit ub = two ? att_unit(p, a0 + i + 1, span) : ua;
+            const int nba = ua.nb, nbb = two ? ub.nb : 0;
+            const int ba = (gi + i) & 1, bb = ba ^ 1;
+            for (int j = 0; j < max(nba, nbb) && ok; ++j) {
+                const uint32_t ea = w, eb = w + (j < nba ? 2u : 0u);
+                w += 2u * ((j < nba ? 1u : 0u) + (j < nbb ? 1u : 0u));
+                if (j < nba && !scores(ba, ea, j == 0)) ok = false;
+                if (ok && j < nbb && !scores(bb, eb, j == 0)) ok = false;
+                if (ok && j < nba && !pv(ba, ea + 1, min(kKVPos, ua.n - j * kKVPos))) ok = false;
+                if (ok && j < nbb && !pv(bb, eb + 1, min(kKVPos, ub.n - j * kKVPos))) ok = false;
+            }
         }
-        wi = wb + 2 * n;
+        wi = w;
         gi += n;
     };
     for (int l = 0; l <= p.layers && ok; ++l) {
@@ -506,7 +579,7 @@ __device__ __forceinline__ void mega_mma(const MegaParams &p, MegaSmem &S, uint8
             const GemmPh g = gemm_phase(p, l, k);
             int64_t u0, u1;
             gemm_range(g, u0, u1);
-            gemm(g, u0, u1);
+            gemm(g, u0, u1, k == kPhGU && l == min(2, p.layers - 1));
             MEGA_STAMP(1 + kPhasesPerLayer * l + k, 3);
             if (k == 0 && l < p.layers && ok) {
                 int64_t a0, a1;
@@ -522,11 +595,11 @@ __device__ __forceinline__ void mega_mma(const MegaParams &p, MegaSmem &S, uint8
 }
 
 // ------------------------------------------------------------------------------ compute
-__device__ __forceinline__ void store_hilo(uint8_t *hi, uint8_t *lo, int64_t off, float v) {
+__device__ __forceinline__ void store_hilo(uint8_t *base, int64_t off, float v) {
     uint16_t h, l;
     split_bf16(v, h, l);
-    *reinterpret_cast<uint16_t *>(hi + off) = h;
-    *reinterpret_cast<uint16_t *>(lo + off) = l;
+    *reinterpret_cast<uint16_t *>(base + off) = h;
+    *reinterpret_cast<uint16_t *>(base + off + kLoOff) = l;
 }
 
 
@@ -543,12 +616,19 @@ __device__ __forceinline__ void mega_compute(const MegaParams &p, MegaSmem &S, u
     const int d = p.d, hd = p.hd, Gq = p.Gq;
     const int gw = cta * 8 + cw, nw = G * 8;
     const uint32_t lane_base = (uint32_t)(quarter * 32) << 16;
-    // GEMM accumulator lane -> activation row: M = 128 puts row i in lane i; M = 64 (at most 64
-    // live rows) puts row i in lane 32 (i / 16) + i % 16
-    const bool m64 = S.rows16 <= 64;
-    const int my_row = m64 ? ((lane < 16) ? quarter * 16 + lane : 1 << 20) : quarter * 32 + lane;
-    const bool quarter_live = (m64 ? quarter * 16 : quarter * 32) < R;
-    uint32_t wi = 0;
+    // GEMM accumulator lane -> activation row.  Stacked operand (at most 64 live rows): operand
+    // row m holds the hi (lo) part of row 8 (m / 16) + m % 8 for m % 16 < 8 (>= 8); M = 128
+    // puts operand row m in lane m, M = 64 (at most 32 rows) in lane 32 (m / 16) + m % 16.
+    // The hi and lo accumulators of a row are lanes i and i ^ 8 of one warp (pair sum by a
+    // shuffle; the hi lane stores).  Otherwise (M = 128, hi and lo accumulated together) row
+    // i is lane i.
+    const int R16 = S.rows16;
+    const bool pair = R16 <= 64;
+    const int my_row = R16 <= 32   ? ((lane & 0x18) == 0 ? quarter * 8 + lane : 1 << 20)
+                       : pair      ? ((lane & 8) == 0 ? quarter * 16 + 8 * (lane >> 4) + (lane & 7) : 1 << 20)
+                                   : quarter * 32 + lane;
+    const bool quarter_live = (R16 <= 32 ? quarter * 8 : pair ? quarter * 16 : quarter * 32) < R;
+    uint32_t att_blk = 0;  // attention blocks this warp group ran (barrier parities)
     int gi = 0, cuse0 = 0, cuse1 = 0, lmseg = 0;  // accumulator buffer uses
 
     // phase arrival: the CTA's writes of this phase (made visible to thread 0 by the barrier)
@@ -596,6 +676,10 @@ __device__ __forceinline__ void mega_compute(const MegaParams &p, MegaSmem &S, u
                 for (int cc = 0; cc < 4; ++cc) {
                     float v[32];
                     tmem_ld_32x32b_x32(tmem + lane_base + (uint32_t)(half * 128 + cc * 32), v);
+                    if (pair) {
+#pragma unroll
+                        for (int e = 0; e < 32; ++e) v[e] += __shfl_xor_sync(0xffffffffu, v[e], 8);
+                    }
                     if (my_row < R) {
                         float4 *q = reinterpret_cast<float4 *>(dst + cc * 32);
 #pragma unroll
@@ -645,8 +729,8 @@ __device__ __forceinline__ void mega_compute(const MegaParams &p, MegaSmem &S, u
             split_bf16(x.x * bf16_to_f32(gb & 0xffff), h0, l0);
             split_bf16(x.y * bf16_to_f32(gb >> 16), h1, l1);
             const int64_t off = xblk_off(r, f, R16c);
-            *reinterpret_cast<uint32_t *>(p.xg_hi + off) = (uint32_t)h0 | ((uint32_t)h1 << 16);
-            *reinterpret_cast<uint32_t *>(p.xg_lo + off) = (uint32_t)l0 | ((uint32_t)l1 << 16);
+            *reinterpret_cast<uint32_t *>(p.xg + off) = (uint32_t)h0 | ((uint32_t)h1 << 16);
+            *reinterpret_cast<uint32_t *>(p.xg + off + kLoOff) = (uint32_t)l0 | ((uint32_t)l1 << 16);
             const float sq = warp_sum(x.x * x.x + x.y * x.y);
             if (lane == 0) ssq[(int64_t)h64 * p.rows_cap + r] = sq;
         }
@@ -677,7 +761,6 @@ __device__ __forceinline__ void mega_compute(const MegaParams &p, MegaSmem &S, u
         // ------------------------------------------------------------ QKV
         gemm_range(gq, u0, u1);
         gemm_epi(gq, u0, u1);
-        wi += (uint32_t)(u1 - u0);
         arrive(base + kPhQKV, false);
         // ------------------------------------------------------------ q, k, v (once per row)
         {
@@ -755,7 +838,6 @@ __device__ __forceinline__ void mega_compute(const MegaParams &p, MegaSmem &S, u
             int64_t a0, a1;
             att_range(p, S.n_items, a0, a1);
             const int n = (int)(a1 - a0);
-            const uint32_t wb = wi;
             wait_phase(base + kPhFinQ);
             const bool det_layer = l == min(2, p.layers - 1);
             if (det_layer && ctid == 0) MEGA_DETAIL(13);
@@ -767,61 +849,43 @@ __device__ __forceinline__ void mega_compute(const MegaParams &p, MegaSmem &S, u
             int i_unit = 0;
             DETAIL(0);
             // units alternate between the two warp groups: group h (warps 3..6 / 7..10, named
-            // barrier 2 + h) runs the units whose buffer parity (gi + i) & 1 is h, each unit
-            // q tile (+ the new position's k, v on a row's last split) -> softmax -> output /
-            // split merge, in order; the MMA issuer interleaves the two groups' units
+            // barrier 2 + h) runs the units (gi + i) & 1 == h, each unit: q tile, then per KV
+            // block scores -> running max -> P -> rescaled output sum (online softmax over
+            // the unit's blocks), then output / split partial + merge, in order
             const int hb = 2 + half;     // this group's named barrier
             const int ht = ctid & 127;   // thread index within the group
             const int hq = ht >> 5;      // warp within the group (owns TMEM lanes 32 hq..)
+            const int span = S.att_span;
             for (int i = half ? 1 - (gi & 1) : (gi & 1); i < n; i += 2) {
-                const AttUnit u = att_unit(p, a0 + i);
-                const int gidx = gi + i, b = half;  // (gidx & 1) == half
-                const uint32_t ph = (uint32_t)((gidx >> 1) & 1);
+                const AttUnit u = att_unit(p, a0 + i, span);
+                const int b = half;
                 const uint16_t *qr = p.qkv16 + (int64_t)u.row * p.nqkv;
-                // ---- q tile rows 0..7 (score columns 8..15 are unused) and, on a row's last
-                // split, the new position's k, v patched into the prefetched block (the copy
-                // may predate their append to the cache)
+                // ---- q tile rows 0..7 (score columns 8..15 are unused)
                 {
                     const int g = ht >> 4, j = ht & 15;
                     uint4 qv = make_uint4(0, 0, 0, 0);
                     if (g < Gq && j * 8 < hd)
                         qv = __ldcg(reinterpret_cast<const uint4 *>(qr + (u.kvh * Gq + g) * hd + j * 8));
                     *reinterpret_cast<uint4 *>(sQ + 4096 * b + (j >> 3) * 2048 + g * 128 + (((j & 7) ^ (g & 7)) << 4)) = qv;
-                    if (u.last && ht < 32) {
-                        const int jj = ht & 15;
-                        const bool isv = ht >= 16;
-                        if (jj * 8 < hd) {
-                            const int pp = u.ctx - 1 - u.p0;
-                            const uint4 kv4 = __ldcg(reinterpret_cast<const uint4 *>(
-                                qr + (p.H + (isv ? p.KVH : 0) + u.kvh) * hd + jj * 8));
-                            const uint32_t ws = wb + 2 * i + (isv ? 1 : 0);
-                            mwait(&S.wfull[ws % kWSlots], (ws / kWSlots) & 1, err, ab);
-                            uint8_t *slot = sW + (size_t)(ws % kWSlots) * kSlotBytes;
-                            if (!isv) {
-                                *reinterpret_cast<uint4 *>(slot + kv_k_off(pp, jj * 8)) = kv4;
-                            } else {
-                                const uint32_t w4[4] = {kv4.x, kv4.y, kv4.z, kv4.w};
-#pragma unroll
-                                for (int e = 0; e < 8; ++e)
-                                    *reinterpret_cast<uint16_t *>(slot + kv_v_off(pp, jj * 8 + e) - 32768) =
-                                        (uint16_t)(w4[e >> 1] >> (16 * (e & 1)));
-                            }
-                        }
-                    }
                     fence_proxy_async_smem();
                     named_bar_sync(hb, 128);
                     if (half == 0) { i_unit = i; DETAIL(1); }
                     if (ht == 0) mbar_arrive(&S.q_ready[b]);
                 }
-                // ---- softmax -> P
-                {
+                // ---- per block: softmax with the running max, P, rescaled output sum
+                float mrun[8], lrun[8], oacc[8];
+#pragma unroll
+                for (int g = 0; g < 8; ++g) { mrun[g] = -INFINITY; lrun[g] = 0.f; oacc[g] = 0.f; }
+                const int pos = quarter * 32 + lane;  // score row (position in the block)
+                for (int jb = 0; jb < u.nb; ++jb) {
+                    const uint32_t ph = att_blk & 1u;
+                    ++att_blk;
+                    const bool valid = pos < min(kKVPos, u.n - jb * kKVPos);
                     mwait(&S.s_full[b], ph, err, ab);
-                    if (half == 0) { i_unit = i; DETAIL(2); }
+                    if (half == 0 && jb == 0) DETAIL(2);
                     tc_fence_after();
                     float sv[8];
                     tmem_ld_32x32b_x8(tmem + lane_base + kTmemS + 16 * b, sv);
-                    const int pos = quarter * 32 + lane;
-                    const bool valid = pos < u.n;
 #pragma unroll
                     for (int g = 0; g < 8; ++g) {
                         sv[g] = valid ? sv[g] : -INFINITY;
@@ -830,13 +894,14 @@ __device__ __forceinline__ void mega_compute(const MegaParams &p, MegaSmem &S, u
                     }
                     tc_fence_before();
                     named_bar_sync(hb, 128);
-                    float M[8];
+                    float mnew[8];
                     uint8_t *pb = sP + 4096 * b + (pos >> 6) * 2048;
                     const int pc = pos & 63;
 #pragma unroll
                     for (int g = 0; g < 8; ++g) {
-                        M[g] = fmaxf(fmaxf(S.red[half][0][g], S.red[half][1][g]), fmaxf(S.red[half][2][g], S.red[half][3][g]));
-                        const float e = valid ? exp2f(sv[g] - M[g]) : 0.f;
+                        mnew[g] = fmaxf(mrun[g], fmaxf(fmaxf(S.red[half][0][g], S.red[half][1][g]),
+                                                       fmaxf(S.red[half][2][g], S.red[half][3][g])));
+                        const float e = valid ? exp2f(sv[g] - mnew[g]) : 0.f;
                         *reinterpret_cast<uint16_t *>(pb + g * 128 + ((((pc >> 3) ^ (g & 7)) << 4) | ((pc & 7) << 1))) =
                             f32_to_f16_sat(e);
                         const float se = warp_sum_unit_redux(e);
@@ -844,44 +909,52 @@ __device__ __forceinline__ void mega_compute(const MegaParams &p, MegaSmem &S, u
                     }
                     fence_proxy_async_smem();
                     named_bar_sync(hb, 128);
-                    if (half == 0) DETAIL(3);
+                    if (half == 0 && jb == 0) DETAIL(3);
                     if (ht == 0) mbar_arrive(&S.p_ready[b]);
-                    if (ht < 8) {
-                        float mc = M[0];
+                    float alpha[8];
 #pragma unroll
-                        for (int g = 1; g < 8; ++g) mc = (ht == g) ? M[g] : mc;
-                        S.att_m[b][ht] = mc;
-                        S.att_l[b][ht] = S.red2[half][0][ht] + S.red2[half][1][ht] + S.red2[half][2][ht] + S.red2[half][3][ht];
+                    for (int g = 0; g < 8; ++g) {
+                        alpha[g] = exp2f(mrun[g] - mnew[g]);  // 0 on the first block
+                        lrun[g] = lrun[g] * alpha[g] + (S.red2[half][0][g] + S.red2[half][1][g]) +
+                                  (S.red2[half][2][g] + S.red2[half][3][g]);
+                        mrun[g] = mnew[g];
                     }
-                }
-                // ---- output (single split) or partial + split merge
-                {
                     mwait(&S.o_full[b], ph, err, ab);
-                    if (half == 0) DETAIL(4);
+                    if (half == 0 && jb == 0) DETAIL(4);
                     tc_fence_after();
                     float ov[8];
                     tmem_ld_32x32b_x8(tmem + lane_base + kTmemO + 16 * b, ov);
+#pragma unroll
+                    for (int g = 0; g < 8; ++g) oacc[g] = oacc[g] * alpha[g] + ov[g];
                     tc_fence_before();
-                    named_bar_sync(hb, 128);  // att_m / att_l of this unit are complete
-                    const int dd = quarter * 32 + lane;
+                }
+                // ---- output (single split) or partial + split merge
+                {
+                    const int dd = quarter * 32 + lane;  // output dim of this thread
                     if (u.nsplit == 1) {
                         if (dd < hd) {
 #pragma unroll
                             for (int g = 0; g < 8; ++g)
                                 if (g < Gq)
-                                    store_hilo(p.att_hi, p.att_lo, xblk_off(u.row, (u.kvh * Gq + g) * hd + dd, R16c),
-                                               ov[g] / S.att_l[b][g]);
+                                    store_hilo(p.att, xblk_off(u.row, (u.kvh * Gq + g) * hd + dd, R16c),
+                                               oacc[g] / lrun[g]);
                         }
                     } else {
                         float *mine = p.part + ((int64_t)u.item * p.KVH + u.kvh) * Gq * (hd + 2);
                         if (dd < hd) {
 #pragma unroll
                             for (int g = 0; g < 8; ++g)
-                                if (g < Gq) mine[g * (hd + 2) + 2 + dd] = ov[g];
+                                if (g < Gq) mine[g * (hd + 2) + 2 + dd] = oacc[g];
                         }
                         if (ht < Gq) {
-                            mine[ht * (hd + 2)] = S.att_m[b][ht];
-                            mine[ht * (hd + 2) + 1] = S.att_l[b][ht];
+                            float mc = mrun[0], lc = lrun[0];
+#pragma unroll
+                            for (int g = 1; g < 8; ++g) {
+                                mc = (ht == g) ? mrun[g] : mc;
+                                lc = (ht == g) ? lrun[g] : lc;
+                            }
+                            mine[ht * (hd + 2)] = mc;
+                            mine[ht * (hd + 2) + 1] = lc;
                         }
                         named_bar_sync(hb, 128);
                         if (half == 0) DETAIL(5);
@@ -939,7 +1012,7 @@ __device__ __forceinline__ void mega_compute(const MegaParams &p, MegaSmem &S, u
 #pragma unroll
                                 for (int g = 0; g < 8; ++g)
                                     if (g < Gq)
-                                        store_hilo(p.att_hi, p.att_lo, xblk_off(u.row, (u.kvh * Gq + g) * hd + dd, R16c),
+                                        store_hilo(p.att, xblk_off(u.row, (u.kvh * Gq + g) * hd + dd, R16c),
                                                    acc[g] / S.ml[half][g]);
                             }
                         }
@@ -948,7 +1021,6 @@ __device__ __forceinline__ void mega_compute(const MegaParams &p, MegaSmem &S, u
                     }
                 }
             }
-            wi = wb + 2 * n;
             gi += n;
             i_unit = 0;
             DETAIL(8);
@@ -959,7 +1031,6 @@ __device__ __forceinline__ void mega_compute(const MegaParams &p, MegaSmem &S, u
         // ------------------------------------------------------------ O projection
         gemm_range(go, u0, u1);
         gemm_epi(go, u0, u1);
-        wi += (uint32_t)(u1 - u0);
         arrive(base + kPhO, false);
         // ------------------------------------------------------------ residual, MLP norm input
         wait_phase(base + kPhO);
@@ -971,7 +1042,6 @@ __device__ __forceinline__ void mega_compute(const MegaParams &p, MegaSmem &S, u
         // ------------------------------------------------------------ gate / up
         gemm_range(gu, u0, u1);
         gemm_epi(gu, u0, u1);
-        wi += (uint32_t)(u1 - u0);
         arrive(base + kPhGU, false);
         // ------------------------------------------------------------ SwiGLU
         {
@@ -1024,9 +1094,9 @@ __device__ __forceinline__ void mega_compute(const MegaParams &p, MegaSmem &S, u
 #pragma unroll
                     for (int e = 0; e < 4; ++e) split_bf16(gv[e] / (1.0f + expf(-gv[e])) * uv[e], hh[e], hl[e]);
                     const int64_t off = xblk_off(rr[q], tt[q] * 128 + 4 * lane, R16c);
-                    *reinterpret_cast<uint2 *>(p.h_hi + off) =
+                    *reinterpret_cast<uint2 *>(p.hm + off) =
                         make_uint2((uint32_t)hh[0] | ((uint32_t)hh[1] << 16), (uint32_t)hh[2] | ((uint32_t)hh[3] << 16));
-                    *reinterpret_cast<uint2 *>(p.h_lo + off) =
+                    *reinterpret_cast<uint2 *>(p.hm + off + kLoOff) =
                         make_uint2((uint32_t)hl[0] | ((uint32_t)hl[1] << 16), (uint32_t)hl[2] | ((uint32_t)hl[3] << 16));
                 }
             }
@@ -1035,7 +1105,6 @@ __device__ __forceinline__ void mega_compute(const MegaParams &p, MegaSmem &S, u
         // ------------------------------------------------------------ down
         gemm_range(gdn, u0, u1);
         gemm_epi(gdn, u0, u1);
-        wi += (uint32_t)(u1 - u0);
         arrive(base + kPhDown, false);
         // ------------------------------------------------------------ residual, next norm input
         wait_phase(base + kPhDown);
@@ -1065,6 +1134,10 @@ __device__ __forceinline__ void mega_compute(const MegaParams &p, MegaSmem &S, u
                 for (int cc = 0; cc < 4; ++cc) {
                     float v[32];
                     tmem_ld_32x32b_x32(tmem + lane_base + (uint32_t)(a * kTileN + half * 128 + cc * 32), v);
+                    if (pair) {
+#pragma unroll
+                        for (int e = 0; e < 32; ++e) v[e] += __shfl_xor_sync(0xffffffffu, v[e], 8);
+                    }
                     if (act) {
                         float4 *q = reinterpret_cast<float4 *>(dst + cc * 32);
 #pragma unroll
@@ -1089,15 +1162,14 @@ __global__ void __launch_bounds__(kMegaThreads, 1) decode_step_kernel(const __gr
     extern __shared__ uint8_t smem_raw[];
     uint8_t *base = reinterpret_cast<uint8_t *>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~(uintptr_t)1023);
     uint8_t *sW = base;
-    uint8_t *sX = sW + (size_t)kWSlots * kSlotBytes;
-    uint8_t *sQ = sX + kXRingBytes;
+    uint8_t *sQ = sW + kRingBytes;
     uint8_t *sP = sQ + 8192;
     MegaSmem &S = *reinterpret_cast<MegaSmem *>(sP + 8192);
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     StepVars *V = p.c.v;
 
     if (threadIdx.x == 0) {
-        for (int s = 0; s < kWSlots; ++s) { mbar_init(&S.wfull[s], 1); mbar_init(&S.wempty[s], 1); }
+        for (int s = 0; s < kMaxWSlots; ++s) { mbar_init(&S.wfull[s], 1); mbar_init(&S.wempty[s], 1); }
         for (int s = 0; s < kMaxXStages; ++s) { mbar_init(&S.xfull[s], 1); mbar_init(&S.xempty[s], 1); }
         for (int a = 0; a < 2; ++a) {
             mbar_init(&S.acc_full[a], 1);
@@ -1112,14 +1184,18 @@ __global__ void __launch_bounds__(kMegaThreads, 1) decode_step_kernel(const __gr
         const int rows = max(0, min(live, p.rows_cap));
         S.rows = rows;
         S.rows16 = max(16, (rows + 15) & ~15);
-        S.nx = min(kMaxXStages, kXRingBytes / (S.rows16 * 256));
+        // the ring holds 5 weight slots while the activation stages are small (at most 64
+        // rows: 16 KB), else 4; the X stages take the rest
+        S.nws = S.rows16 <= 64 ? 5 : 4;
+        S.nx = min(kMaxXStages, (kRingBytes - S.nws * kSlotBytes) / (S.rows16 * 256));
         S.n_items = *(volatile int *)&V->att_items;
+        S.att_span = max(1, *(volatile int *)&V->att_span);
         S.target = (*(volatile unsigned long long *)p.epoch + 1ull) * gridDim.x;
         S.abort = (*(volatile int *)&V->err & ERR_WAIT_TIMEOUT) != 0;
         S.last_flag = 0;
         fence_mbar_init();
     }
-    if (threadIdx.x == 0) MEGA_STAMP(p.n_stamp_ph - 5, 0);  // kernel start
+    if (threadIdx.x == 0) MEGA_STAMP(p.n_stamp_ph - kDetailRows - 1, 0);  // kernel start
     if (warp == 1) {
         tmem_alloc(&S.tmem_base, kTmemCols);
         tmem_relinquish();
@@ -1128,6 +1204,7 @@ __global__ void __launch_bounds__(kMegaThreads, 1) decode_step_kernel(const __gr
     __syncthreads();
     tc_fence_after();
     const uint32_t tmem = S.tmem_base;
+    uint8_t *sX = sW + (size_t)S.nws * kSlotBytes;
     const bool run = !S.abort && S.rows > 0;
     if (run) {
         if (warp == 0) {

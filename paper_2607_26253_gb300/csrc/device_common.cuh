@@ -251,11 +251,12 @@ __device__ __forceinline__ void tmem_ld_32x32b_x8(uint32_t taddr, float (&v)[8])
 // tile base 1024-byte aligned.  Fields: start address >> 4 (bits 0-13), leading-byte offset
 // >> 4 (16-29, unused for swizzled K-major), stride-byte offset >> 4 (32-45), descriptor
 // version 1 (46-47), swizzle mode 2 = 128B (61-63).
-__device__ __forceinline__ uint64_t sdesc_kmajor_sw128(uint32_t smem_addr) {
+// (sbo: the byte distance between consecutive 8-row atoms, 1024 when they are packed)
+__device__ __forceinline__ uint64_t sdesc_kmajor_sw128(uint32_t smem_addr, uint32_t sbo = 1024) {
     uint64_t d = 0;
     d |= (uint64_t)((smem_addr & 0x3FFFFu) >> 4);
     d |= (uint64_t)(16u >> 4) << 16;
-    d |= (uint64_t)(1024u >> 4) << 32;
+    d |= (uint64_t)(sbo >> 4) << 32;
     d |= (uint64_t)1 << 46;
     d |= (uint64_t)2 << 61;
     return d;

@@ -80,7 +80,7 @@ struct sara_handle {
     // decode-step activations (blocked operands) and phase counters
     int rows_cap16 = 0;
     float *dx = nullptr, *ssqA = nullptr, *ssqM = nullptr;
-    uint8_t *xg_hi = nullptr, *xg_lo = nullptr, *att_hi = nullptr, *att_lo = nullptr, *h_hi = nullptr, *h_lo = nullptr;
+    uint8_t *xg = nullptr, *att = nullptr, *hm = nullptr;  // pair-blocked GEMM operands of the decode step
     float *gpart = nullptr;  // GEMM partial tiles of the decode step
     uint16_t *qkv16 = nullptr;  // the step's q (scaled), k, v in fp16
     int gp_qkv = 0, gp_o = 0;
@@ -355,12 +355,9 @@ MegaParams mega_params(const sara_handle &h) {
     p.rows_cap = m.max_seqs;
     p.rows_cap16 = h.rows_cap16;
     p.x = h.dx;
-    p.xg_hi = h.xg_hi;
-    p.xg_lo = h.xg_lo;
-    p.att_hi = h.att_hi;
-    p.att_lo = h.att_lo;
-    p.h_hi = h.h_hi;
-    p.h_lo = h.h_lo;
+    p.xg = h.xg;
+    p.att = h.att;
+    p.hm = h.hm;
     p.ssqA = h.ssqA;
     p.ssqM = h.ssqM;
     p.gpart = h.gpart;
@@ -373,7 +370,7 @@ MegaParams mega_params(const sara_handle &h) {
     p.cnt = h.phase_cnt;
     p.epoch = h.phase_cnt + (size_t)h.n_phase_cnt * kCntStride;
     p.stamps = h.stamps;
-    p.n_stamp_ph = h.n_phase_cnt + 1 + 4;  // phases, kernel start, 4 x 4 detail stamps
+    p.n_stamp_ph = h.n_phase_cnt + 1 + kDetailRows;  // phases, kernel start, detail stamps
     return p;
 }
 
@@ -577,12 +574,9 @@ void alloc_decode(sara_handle &h) {
     h.rows_cap16 = (S + 15) & ~15;
     const size_t R16 = h.rows_cap16;
     h.dx = h.mem.alloc<float>((size_t)S * d);
-    h.xg_hi = h.mem.alloc<uint8_t>(R16 * d * 2);
-    h.xg_lo = h.mem.alloc<uint8_t>(R16 * d * 2);
-    h.att_hi = h.mem.alloc<uint8_t>(R16 * Hhd * 2);
-    h.att_lo = h.mem.alloc<uint8_t>(R16 * Hhd * 2);
-    h.h_hi = h.mem.alloc<uint8_t>(R16 * F * 2);
-    h.h_lo = h.mem.alloc<uint8_t>(R16 * F * 2);
+    h.xg = h.mem.alloc<uint8_t>(R16 * d * 4);
+    h.att = h.mem.alloc<uint8_t>(R16 * Hhd * 4);
+    h.hm = h.mem.alloc<uint8_t>(R16 * F * 4);
     h.ssqA = h.mem.alloc<float>((size_t)(d / 64) * S);
     h.ssqM = h.mem.alloc<float>((size_t)(d / 64) * S);
     // partial tiles: one segment per (CTA, tile) pair of a phase, at most CTAs + tiles - 1
@@ -602,6 +596,12 @@ void alloc_decode(sara_handle &h) {
 
 // Phase counters and split counters back to zero (start of every call: a step that failed
 // part-way may have left them anywhere).
+// Decode attention units run at once per kv head: one per compute warp group (two per SM).
+int att_slots(const sara_handle &h) {
+    const int kvh = h.has_model ? std::max(1, h.cfg.n_kv_heads) : 1;
+    return std::max(1, 2 * h.sms / kvh);
+}
+
 void reset_decode_state(sara_handle &h, cudaStream_t s) {
     const sara_model_cfg &m = h.cfg;
     CK(cudaMemsetAsync(h.phase_cnt, 0, ((size_t)h.n_phase_cnt + 1) * kCntStride * 8, s));
@@ -814,6 +814,7 @@ void collect_impl(sara_handle &h, const sara_prompts *pr, int64_t N, int32_t k, 
     K.teacher = 0;
     K.max_gen = m.max_gen_len;
     K.attn_chunk = kDecodeChunk;
+    K.att_slots = att_slots(h);
 
     CK(cudaEventRecord(h.ev0, s));
     CK(cudaMemcpyAsync(h.kc, &K, sizeof(K), cudaMemcpyHostToDevice, s));
@@ -889,7 +890,7 @@ void teacher_impl(sara_handle &h, int n, int Lp, const int32_t *prompts, int T, 
     StepConst K{};
     K.P = n; K.Lp = Lp; K.k = 2; K.n0 = 1; K.commit_min = 2; K.a0 = 1; K.b0 = 1; K.B = n; K.N = n;
     K.tau_num = 0; K.tau_den = 1; K.sample_seed = sample_seed; K.decode = 1; K.teacher = 1; K.T_forced = T;
-    K.max_gen = m.max_gen_len; K.attn_chunk = kDecodeChunk;
+    K.max_gen = m.max_gen_len; K.attn_chunk = kDecodeChunk; K.att_slots = att_slots(h);
     CK(cudaMemcpyAsync(h.kc, &K, sizeof(K), cudaMemcpyHostToDevice, s));
     CK(cudaMemcpyAsync(h.p_tok, prompts, (size_t)n * Lp * 4, kin, s));
     CK(cudaMemcpyAsync(h.forced, forced, (size_t)n * T * 4, kin, s));
@@ -929,12 +930,12 @@ void teacher_impl(sara_handle &h, int n, int Lp, const int32_t *prompts, int T, 
 // arrived) to this one's, the median delay until CTAs observed the dependency, and how far
 // ahead of the previous phase's completion the W producer had issued this phase's copies.
 void print_stamps(sara_handle &h, int rows, int ctx) {
-    const int NP = h.n_phase_cnt + 1 + 4, G = h.sms, L = h.cfg.layers;
+    const int NP = h.n_phase_cnt + 1 + kDetailRows, G = h.sms, L = h.cfg.layers;
     std::vector<uint64_t> st((size_t)G * NP * 4);
     CK(cudaMemcpy(st.data(), h.stamps, st.size() * 8, cudaMemcpyDeviceToHost));
     auto at = [&](int c, int ph, int k) { return st[((size_t)c * NP + ph) * 4 + k]; };
     uint64_t t0 = ~0ull;
-    for (int c = 0; c < G; ++c) t0 = std::min(t0, at(c, NP - 5, 0));
+    for (int c = 0; c < G; ++c) t0 = std::min(t0, at(c, NP - kDetailRows - 1, 0));
     auto stat = [&](int ph, int k, bool mx) {
         std::vector<double> v;
         for (int c = 0; c < G; ++c)
@@ -974,12 +975,31 @@ void print_stamps(sara_handle &h, int rows, int ctx) {
     for (int i = 0; i < 15; ++i) {
         std::vector<double> v;
         for (int c = 0; c < G; ++c) {
-            const uint64_t x = at(c, NP - 4 + i / 4, i % 4);
+            const uint64_t x = at(c, NP - kDetailRows + i / 4, i % 4);
             if (x >= t0) v.push_back((double)(x - t0) * 1e-3 - ref);
         }
         std::sort(v.begin(), v.end());
         if (!v.empty())
             fprintf(stderr, "    %-14s n=%3zu  med %+7.2f  max %+7.2f us\n", dn[i], v.size(), v[v.size() / 2], v.back());
+    }
+    // gate / up units of layer 2 (medians over CTAs, relative to FIN_O's completion)
+    const double ref_fo = done[1 + kPhasesPerLayer * lq + kPhFinO];
+    fprintf(stderr, "    GU unit: W issued / W full / X full / MMA committed (us after FIN_O)\n");
+    for (int j = 0; j < 12; ++j) {
+        double med[4];
+        int nn = 0;
+        for (int kind = 0; kind < 4; ++kind) {
+            std::vector<double> v;
+            const int i = 16 + 12 * kind + j;
+            for (int c = 0; c < G; ++c) {
+                const uint64_t x = at(c, NP - kDetailRows + i / 4, i % 4);
+                if (x >= t0) v.push_back((double)(x - t0) * 1e-3 - ref_fo);
+            }
+            std::sort(v.begin(), v.end());
+            med[kind] = v.empty() ? 0.0 : v[v.size() / 2];
+            nn = std::max(nn, (int)v.size());
+        }
+        fprintf(stderr, "      %2d n=%3d  %+7.2f %+7.2f %+7.2f %+7.2f\n", j, nn, med[0], med[1], med[2], med[3]);
     }
 }
 #endif
@@ -999,7 +1019,10 @@ void profile_impl(sara_handle &h, int which, int rows, int ctx, int iters, doubl
     StepConst K{};
     K.P = 1; K.Lp = ctx; K.k = 2; K.n0 = 1; K.commit_min = 2; K.a0 = 1; K.b0 = 1; K.B = 1; K.N = 1;
     K.tau_num = 0; K.tau_den = 1; K.decode = 1; K.max_gen = m.max_gen_len; K.attn_chunk = kDecodeChunk;
-    const int nsplit = (ctx + kDecodeChunk - 1) / kDecodeChunk;
+    K.att_slots = att_slots(h);
+    const int nblk = (ctx + kDecodeChunk - 1) / kDecodeChunk;
+    const int span = att_span_for((int64_t)rows * nblk, K.att_slots);
+    const int nsplit = (nblk + span - 1) / span;
     std::vector<int> slot(rows), pos(rows, ctx - 1), tok(rows, 0), item0(rows), zero(rows, 0), len(rows, m.max_gen_len);
     std::vector<uint64_t> seed(rows);
     std::vector<int64_t> uid(rows);
@@ -1014,6 +1037,7 @@ void profile_impl(sara_handle &h, int which, int rows, int ctx, int iters, doubl
     StepVars v{};
     v.live = rows;
     v.att_items = rows * nsplit;
+    v.att_span = span;
     v.round_maxL = 1 << 30;
     const StepPtrs &c = h.ptrs;
     reset_decode_state(h, s);
@@ -1031,7 +1055,7 @@ void profile_impl(sara_handle &h, int which, int rows, int ctx, int iters, doubl
     CK(cudaMemcpyAsync(c.seq_len, len.data(), rows * 4, cudaMemcpyHostToDevice, s));
     CK(cudaMemcpyAsync(c.seq_uid, uid.data(), rows * 8, cudaMemcpyHostToDevice, s));
 #ifdef SARA_STAMPS
-    const size_t nst = (size_t)h.sms * (h.n_phase_cnt + 1 + 4) * 4;
+    const size_t nst = (size_t)h.sms * (h.n_phase_cnt + 1 + kDetailRows) * 4;
     if (!h.stamps) h.stamps = h.mem.alloc<uint64_t>(nst);
 #endif
     CK(cudaStreamSynchronize(s));

@@ -170,11 +170,19 @@ static __global__ void __launch_bounds__(256) sample_finish_kernel(StepPtrs c, c
         __syncthreads();
         out += tot;
     }
-    // attention items of the next step
+    // attention items of the next step: splits of `span` KV blocks
+    int blocks = 0;
+    for (int base = 0; base < out; base += 256) {
+        const int i = base + tid;
+        int tot;
+        scan256(i < out ? (c.row_pos[i] + K.attn_chunk) / K.attn_chunk : 0, tot, warp_tot);
+        blocks += tot;
+    }
+    const int span = att_span_for(blocks, K.att_slots);
     int items = 0;
     for (int base = 0; base < out; base += 256) {
         const int i = base + tid;
-        const int ns = (i < out) ? (c.row_pos[i] + 1 + K.attn_chunk - 1) / K.attn_chunk : 0;
+        const int ns = (i < out) ? ((c.row_pos[i] + K.attn_chunk) / K.attn_chunk + span - 1) / span : 0;
         int tot;
         const int before = scan256(ns, tot, warp_tot);
         if (i < out) {
@@ -190,6 +198,7 @@ static __global__ void __launch_bounds__(256) sample_finish_kernel(StepPtrs c, c
     if (tid == 0) {
         V.live = out;
         V.att_items = min(items, c.att_cap);
+        V.att_span = span;
         V.exec_steps += 1;
         V.round_steps += 1;
     }
@@ -201,7 +210,9 @@ static __global__ void __launch_bounds__(kCtlThreads, 1) teacher_setup_kernel(St
     const StepConst &K = *c.kc;
     StepVars &V = *c.v;
     const int Lp = K.Lp, Lpre = Lp - 1;
-    const int nsplit = (Lp + K.attn_chunk - 1) / K.attn_chunk;
+    const int nblk = (Lp + K.attn_chunk - 1) / K.attn_chunk;
+    const int span = att_span_for((int64_t)n * nblk, K.att_slots);
+    const int nsplit = (nblk + span - 1) / span;
     for (int r = threadIdx.x; r < n; r += kCtlThreads) {
         c.seq_q[r] = r;
         c.seq_j[r] = 0;
@@ -230,6 +241,7 @@ static __global__ void __launch_bounds__(kCtlThreads, 1) teacher_setup_kernel(St
         z.round = 0;
         z.live = n;
         z.att_items = n * nsplit;
+        z.att_span = span;
         z.pre_rows = n * Lpre;
         z.n_fresh = n;
         z.round_maxL = K.T_forced;

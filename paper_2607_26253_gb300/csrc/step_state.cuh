@@ -21,8 +21,8 @@ struct StepConst {
     int32_t teacher;      // 1: teacher forcing (one round, forced tokens)
     int32_t T_forced;     // teacher: generated tokens per rollout
     int32_t max_gen;      // stride of the generated-token output
-    int32_t attn_chunk;   // decode attention positions per split
-    int32_t pad_;
+    int32_t attn_chunk;   // decode attention: positions per KV block
+    int32_t att_slots;    // decode attention: units one step runs at once, per kv head
 };
 
 // Scalar progress of the step (device, reset by the init kernel).
@@ -39,9 +39,17 @@ struct StepVars {
     int32_t err;
     int32_t fin_count;     // arrival counter of the sample/finish kernel
     int32_t iters;         // loop iterations
-    int32_t pad_;
+    int32_t att_span;      // KV blocks per decode attention split of the next step
     int64_t used, C, cursor, drawn, gen_tokens, sched_steps, exec_steps, rounds_done;
 };
+
+// KV blocks per decode attention split: the smallest span that leaves at most `slots` split
+// units per kv head when `blocks` blocks (summed over the rows) are to be covered.
+__host__ __device__ inline int att_span_for(int64_t blocks, int slots) {
+    if (slots < 1) slots = 1;
+    const int64_t s = (blocks + slots - 1) / slots;
+    return s < 1 ? 1 : (int)s;
+}
 
 struct StepPtrs {
     StepConst *kc;
