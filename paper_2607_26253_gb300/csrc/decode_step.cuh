@@ -55,10 +55,10 @@ namespace sara {
 
 constexpr int kMegaThreads = 352;
 constexpr int kMegaCThreads = 256;  // compute warps 3..10
-constexpr int kMaxWSlots = 5;
+constexpr int kWSlots = 4;  // weight / KV ring entries (a power of two: slot = index & 3)
 constexpr int kDetailRows = 16;  // profiling builds: rows of 4 detail stamps per CTA
 constexpr int kSlotBytes = 32768;
-constexpr int kRingBytes = 4 * 32768 + 65536;  // W slots + X stages share it
+constexpr int kRingBytes = 4 * 32768 + 65536;  // W slots, then the X stages
 constexpr int kMaxXStages = 8;
 constexpr int kTileN = 256;           // weight rows (output features) per GEMM tile
 constexpr int kKVPos = 128;           // positions per KV block and per attention split
@@ -134,7 +134,7 @@ struct MegaParams {
 #endif
 
 struct MegaSmem {
-    uint64_t wfull[kMaxWSlots], wempty[kMaxWSlots];
+    uint64_t wfull[kWSlots], wempty[kWSlots];
     uint64_t xfull[kMaxXStages], xempty[kMaxXStages];
     uint64_t acc_full[2], acc_empty[2];
     uint64_t q_ready[2], s_full[2], p_ready[2], o_full[2];
@@ -143,7 +143,7 @@ struct MegaSmem {
     uint32_t tmem_base;
     int abort;
     int last_flag;
-    int rows, rows16, nws, nx, n_items, att_span;
+    int rows, rows16, nx, nx_lg, n_items, att_span;  // nx = 2^nx_lg X stages
     float rstd[128];
     float red[2][4][8], red2[2][4][8];  // per warp group: attention max / sum reductions
     float mw[2][8][kMegaMaxSplits];      // per warp group: split weights of a merge
@@ -330,7 +330,7 @@ __device__ __forceinline__ void mega_w_producer(const MegaParams &p, MegaSmem &S
     volatile int *ab = &S.abort;
     int *err = &p.c.v->err;
     const uint64_t pol = l2_policy_evict_first();
-    const uint32_t nws = (uint32_t)S.nws;
+    constexpr uint32_t nws = kWSlots;
     uint32_t wi = 0;
     bool ok = true;
     auto acquire = [&](uint32_t i) -> bool {
@@ -416,7 +416,7 @@ __device__ __forceinline__ void mega_x_producer(const MegaParams &p, MegaSmem &S
     volatile int *ab = &S.abort;
     int *err = &p.c.v->err;
     const uint64_t pol = l2_policy_evict_last();
-    const int NX = S.nx, R16 = S.rows16;
+    const int NX = S.nx, R16 = S.rows16, nxl = S.nx_lg;
     const uint32_t stage = (uint32_t)R16 * 256;  // hi + lo parts of the live rows' groups
     const int64_t chunk_stride = (int64_t)p.rows_cap16 * 256;
     uint32_t xi = 0;
@@ -436,8 +436,8 @@ __device__ __forceinline__ void mega_x_producer(const MegaParams &p, MegaSmem &S
             MEGA_STAMP(1 + kPhasesPerLayer * l + k, 1);
             fence_proxy_async_global();
             for (int64_t u = u0; u < u1; ++u, ++xi) {
-                const int s = (int)(xi % NX);
-                if (xi >= (uint32_t)NX && !mwait(&S.xempty[s], ((xi / NX) & 1) ^ 1, err, ab)) { ok = false; break; }
+                const int s = (int)(xi & (uint32_t)(NX - 1));
+                if (xi >= (uint32_t)NX && !mwait(&S.xempty[s], ((xi >> nxl) & 1) ^ 1, err, ab)) { ok = false; break; }
                 const int kc = (int)(u % g.kch);
                 mbar_arrive_expect_tx(&S.xfull[s], stage);
                 bulk_load(sX + (size_t)s * stage, g.x + kc * chunk_stride, stage, &S.xfull[s], pol);
@@ -446,8 +446,8 @@ __device__ __forceinline__ void mega_x_producer(const MegaParams &p, MegaSmem &S
     }
     if (!ok) {
         for (uint32_t s = 0; s < (uint32_t)NX && s < xi; ++s) {
-            const uint32_t last = ((xi - 1 - s) / NX) * NX + s;
-            mbar_wait(&S.xfull[s], (last / NX) & 1, err);
+            const uint32_t last = (((xi - 1 - s) >> nxl) << nxl) + s;
+            mbar_wait(&S.xfull[s], (last >> nxl) & 1, err);
         }
     }
 }
@@ -457,7 +457,7 @@ __device__ __forceinline__ void mega_mma(const MegaParams &p, MegaSmem &S, uint8
                                          uint8_t *sP, uint32_t tmem) {
     volatile int *ab = &S.abort;
     int *err = &p.c.v->err;
-    const int NX = S.nx, R16 = S.rows16;
+    const int NX = S.nx, R16 = S.rows16, nxl = S.nx_lg;
     const uint32_t stage = (uint32_t)R16 * 256;
     const uint32_t ida = idesc_f16_f32(128, 16);
     // at most 64 live rows: one MMA per k-step over the stacked hi / lo groups (M = 2 R16
@@ -467,7 +467,7 @@ __device__ __forceinline__ void mega_mma(const MegaParams &p, MegaSmem &S, uint8
     uint32_t wi = 0, xi = 0;
     int gi = 0, use0 = 0, use1 = 0, lmseg = 0;  // accumulator buffer uses
     bool ok = true;
-    const uint32_t nws = (uint32_t)S.nws;
+    constexpr uint32_t nws = kWSlots;
     auto wslot = [&](uint32_t i) -> uint32_t { return smem_u32(sW + (size_t)(i % nws) * kSlotBytes); };
     auto wwait = [&](uint32_t i) -> bool { return mwait(&S.wfull[i % nws], (i / nws) & 1, err, ab); };
     auto gemm = [&](const GemmPh &g, int64_t u0, int64_t u1, bool det) {
@@ -483,11 +483,11 @@ __device__ __forceinline__ void mega_mma(const MegaParams &p, MegaSmem &S, uint8
             const uint32_t idg = idesc_bf16_f32(R16 <= 32 ? 64u : 128u, (uint32_t)tile_rows(g, t));
             bool first = true;
             for (; u < e; ++u, ++wi, ++xi) {
-                const int xs = (int)(xi % NX);
+                const int xs = (int)(xi & (uint32_t)(NX - 1));
                 const bool dj = det && u - ub < 12;
                 if (!wwait(wi)) { ok = false; break; }
                 if (dj) MEGA_DETAIL(28 + (int)(u - ub));
-                if (!mwait(&S.xfull[xs], (xi / NX) & 1, err, ab)) { ok = false; break; }
+                if (!mwait(&S.xfull[xs], (xi >> nxl) & 1, err, ab)) { ok = false; break; }
                 if (dj) MEGA_DETAIL(40 + (int)(u - ub));
                 tc_fence_after();
                 const uint32_t aw = wslot(wi), ax = smem_u32(sX + (size_t)xs * stage);
@@ -769,12 +769,13 @@ __device__ __forceinline__ void mega_compute(const MegaParams &p, MegaSmem &S, u
             // fp16 q, k, v for the attention phase; k and v appended to the KV cache at the
             // row's position
             wait_phase(base + kPhQKV);
-            load_rstd(p.ssqA);
             const int nh = p.H + 2 * p.KVH, dpu = min(hd, 64), upr = hd / dpu;
             for (int u = gw; u < R * nh * upr; u += nw) {
                 const int r = u / (nh * upr), rem = u - r * nh * upr;
-                const int head = rem / upr, d0 = (rem - head * upr) * dpu + 2 * lane;
-                if (2 * lane >= dpu) continue;
+                // lanes past the unit's dims (head dim 32) repeat lane 0's loads and store nothing:
+                // every lane takes part in the row's sum-of-squares reduction
+                const bool live = 2 * lane < dpu;
+                const int head = rem / upr, d0 = (rem - head * upr) * dpu + (live ? 2 * lane : 0);
                 const bool isq = head < p.H, isk = !isq && head < p.H + p.KVH;
                 const int half_hd = hd >> 1;
                 const int pd0 = d0 < half_hd ? d0 + half_hd : d0 - half_hd;
@@ -782,6 +783,8 @@ __device__ __forceinline__ void mega_compute(const MegaParams &p, MegaSmem &S, u
                 const int col = f0 - t * kTileN, pcol = head * hd + pd0 - t * kTileN;
                 int ca, cb;
                 tile_ctas(gq, t, ca, cb);
+                // the row's sum-of-squares partials load with the first batch of QKV partials
+                const float sq = lane < d / 64 ? __ldcg(&p.ssqA[(int64_t)lane * p.rows_cap + r]) : 0.f;
                 float2 x = make_float2(0.f, 0.f), xp = x;
                 for (int c0 = ca; c0 <= cb; c0 += 16) {  // 16 contributors' loads in flight, CTA order
                     float2 a[16], b2[16];
@@ -800,7 +803,8 @@ __device__ __forceinline__ void mega_compute(const MegaParams &p, MegaSmem &S, u
                     }
                 }
                 const int pos = __ldg(&p.c.row_pos[r]);
-                const float rs = S.rstd[r] * (isq ? p.scale_log2 : 1.f);
+                const float rs = rsqrtf(warp_sum(sq) / (float)d + p.eps) * (isq ? p.scale_log2 : 1.f);
+                if (!live) continue;
                 float y0 = x.x, y1 = x.y;
                 if (isq || isk) {  // rotate the pairs (i, i + hd/2)
                     const int fr = d0 < half_hd ? d0 : pd0;
@@ -1046,7 +1050,6 @@ __device__ __forceinline__ void mega_compute(const MegaParams &p, MegaSmem &S, u
         // ------------------------------------------------------------ SwiGLU
         {
             wait_phase(base + kPhGU);
-            load_rstd(p.ssqM);
             const int fb = p.F / 128;
             // unit = (row, 128 features of h) = one 256-row tile of the gate/up outputs; lane:
             // 4 features, gate at tile column c, up at c + 64 (c = 4 lane, or 128 + 4 lane - 64
@@ -1056,16 +1059,19 @@ __device__ __forceinline__ void mega_compute(const MegaParams &p, MegaSmem &S, u
             for (int u = gw; u < R * fb; u += 2 * nw) {
                 float4 gs[2], us[2];
                 int rr[2], tt[2];
+                float sq[2];  // the rows' sum-of-squares partials, loaded with the gate / up partials
 #pragma unroll
                 for (int q = 0; q < 2; ++q) {
                     const int uq = u + q * nw;
                     gs[q] = us[q] = make_float4(0.f, 0.f, 0.f, 0.f);
                     rr[q] = -1;
                     tt[q] = 0;
+                    sq[q] = 0.f;
                     if (uq >= R * fb) continue;
                     const int r = uq / fb, t = uq - r * fb;
                     rr[q] = r;
                     tt[q] = t;
+                    sq[q] = lane < d / 64 ? __ldcg(&p.ssqM[(int64_t)lane * p.rows_cap + r]) : 0.f;
                     int ca, cb;
                     tile_ctas(gu, t, ca, cb);
                     for (int cq = ca; cq <= cb; cq += 4) {
@@ -1084,10 +1090,13 @@ __device__ __forceinline__ void mega_compute(const MegaParams &p, MegaSmem &S, u
                         }
                     }
                 }
+                float rsq[2];
+#pragma unroll
+                for (int q = 0; q < 2; ++q) rsq[q] = rsqrtf(warp_sum(sq[q]) / (float)d + p.eps);
 #pragma unroll
                 for (int q = 0; q < 2; ++q) {
                     if (rr[q] < 0) continue;
-                    const float rs = S.rstd[rr[q]];
+                    const float rs = rsq[q];
                     const float gv[4] = {gs[q].x * rs, gs[q].y * rs, gs[q].z * rs, gs[q].w * rs};
                     const float uv[4] = {us[q].x * rs, us[q].y * rs, us[q].z * rs, us[q].w * rs};
                     uint16_t hh[4], hl[4];
@@ -1169,7 +1178,7 @@ __global__ void __launch_bounds__(kMegaThreads, 1) decode_step_kernel(const __gr
     StepVars *V = p.c.v;
 
     if (threadIdx.x == 0) {
-        for (int s = 0; s < kMaxWSlots; ++s) { mbar_init(&S.wfull[s], 1); mbar_init(&S.wempty[s], 1); }
+        for (int s = 0; s < kWSlots; ++s) { mbar_init(&S.wfull[s], 1); mbar_init(&S.wempty[s], 1); }
         for (int s = 0; s < kMaxXStages; ++s) { mbar_init(&S.xfull[s], 1); mbar_init(&S.xempty[s], 1); }
         for (int a = 0; a < 2; ++a) {
             mbar_init(&S.acc_full[a], 1);
@@ -1184,10 +1193,14 @@ __global__ void __launch_bounds__(kMegaThreads, 1) decode_step_kernel(const __gr
         const int rows = max(0, min(live, p.rows_cap));
         S.rows = rows;
         S.rows16 = max(16, (rows + 15) & ~15);
-        // the ring holds 5 weight slots while the activation stages are small (at most 64
-        // rows: 16 KB), else 4; the X stages take the rest
-        S.nws = S.rows16 <= 64 ? 5 : 4;
-        S.nx = min(kMaxXStages, (kRingBytes - S.nws * kSlotBytes) / (S.rows16 * 256));
+        // X stages: the largest power of two (at most kMaxXStages) that fits after the W slots
+        {
+            const int fit = min(kMaxXStages, (kRingBytes - kWSlots * kSlotBytes) / (S.rows16 * 256));
+            int lg = 0;
+            while ((2 << lg) <= fit) ++lg;
+            S.nx = 1 << lg;
+            S.nx_lg = lg;
+        }
         S.n_items = *(volatile int *)&V->att_items;
         S.att_span = max(1, *(volatile int *)&V->att_span);
         S.target = (*(volatile unsigned long long *)p.epoch + 1ull) * gridDim.x;
@@ -1204,7 +1217,7 @@ __global__ void __launch_bounds__(kMegaThreads, 1) decode_step_kernel(const __gr
     __syncthreads();
     tc_fence_after();
     const uint32_t tmem = S.tmem_base;
-    uint8_t *sX = sW + (size_t)S.nws * kSlotBytes;
+    uint8_t *sX = sW + (size_t)kWSlots * kSlotBytes;
     const bool run = !S.abort && S.rows > 0;
     if (run) {
         if (warp == 0) {
