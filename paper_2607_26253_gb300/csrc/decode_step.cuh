@@ -465,7 +465,7 @@ __device__ __forceinline__ void mega_mma(const MegaParams &p, MegaSmem &S, uint8
     // reads); more: the hi and the lo groups as two 128-row operands into one accumulator
     const bool stacked = R16 <= 64;
     uint32_t wi = 0, xi = 0;
-    int gi = 0, use0 = 0, use1 = 0, lmseg = 0;  // accumulator buffer uses
+    int gi = 0, use0 = 0, use1 = 0, tseg = 0;  // accumulator buffer uses, GEMM tiles so far
     bool ok = true;
     constexpr uint32_t nws = kWSlots;
     auto wslot = [&](uint32_t i) -> uint32_t { return smem_u32(sW + (size_t)(i % nws) * kSlotBytes); };
@@ -475,7 +475,7 @@ __device__ __forceinline__ void mega_mma(const MegaParams &p, MegaSmem &S, uint8
         for (int64_t u = u0; u < u1 && ok;) {
             const int t = (int)(u / g.kch);
             const int64_t e = min(u1, (int64_t)(t + 1) * g.kch);
-            const int a = g.whole ? (lmseg & 1) : 0;  // lm_head alternates two accumulators
+            const int a = tseg & 1;  // tiles alternate between two accumulators (epilogue overlaps)
             const int use_a = a ? use1 : use0;
             if (use_a >= 1 && !mwait(&S.acc_empty[a], (use_a - 1) & 1, err, ab)) { ok = false; break; }
             tc_fence_after();
@@ -510,7 +510,7 @@ __device__ __forceinline__ void mega_mma(const MegaParams &p, MegaSmem &S, uint8
             if (!ok) break;
             tc_commit(&S.acc_full[a]);
             if (a) ++use1; else ++use0;
-            if (g.whole) ++lmseg;
+            ++tseg;
         }
     };
     // attention: unit pairs (one unit per compute warp group, group (gi + i) & 1), block by
@@ -629,7 +629,7 @@ __device__ __forceinline__ void mega_compute(const MegaParams &p, MegaSmem &S, u
                                    : quarter * 32 + lane;
     const bool quarter_live = (R16 <= 32 ? quarter * 8 : pair ? quarter * 16 : quarter * 32) < R;
     uint32_t att_blk = 0;  // attention blocks this warp group ran (barrier parities)
-    int gi = 0, cuse0 = 0, cuse1 = 0, lmseg = 0;  // accumulator buffer uses
+    int gi = 0, cuse0 = 0, cuse1 = 0, tseg = 0;  // accumulator buffer uses, GEMM tiles so far
 
     // phase arrival: the CTA's writes of this phase (made visible to thread 0 by the barrier)
     // are released to the other CTAs with the counter increment
@@ -667,7 +667,8 @@ __device__ __forceinline__ void mega_compute(const MegaParams &p, MegaSmem &S, u
         for (int64_t u = u0; u < u1;) {
             const int t = (int)(u / g.kch);
             u = min(u1, (int64_t)(t + 1) * g.kch);
-            mwait(&S.acc_full[0], cuse0 & 1, err, ab);
+            const int a = tseg & 1;
+            mwait(&S.acc_full[a], (a ? cuse1 : cuse0) & 1, err, ab);
             tc_fence_after();
             const int rows_t = tile_rows(g, t);
             if (quarter_live && half * 128 < rows_t) {
@@ -675,7 +676,7 @@ __device__ __forceinline__ void mega_compute(const MegaParams &p, MegaSmem &S, u
 #pragma unroll 1
                 for (int cc = 0; cc < 4; ++cc) {
                     float v[32];
-                    tmem_ld_32x32b_x32(tmem + lane_base + (uint32_t)(half * 128 + cc * 32), v);
+                    tmem_ld_32x32b_x32(tmem + lane_base + (uint32_t)(a * kTileN + half * 128 + cc * 32), v);
                     if (pair) {
 #pragma unroll
                         for (int e = 0; e < 32; ++e) v[e] += __shfl_xor_sync(0xffffffffu, v[e], 8);
@@ -689,8 +690,9 @@ __device__ __forceinline__ void mega_compute(const MegaParams &p, MegaSmem &S, u
             }
             tc_fence_before();
             __syncwarp();
-            if (lane == 0) mbar_arrive(&S.acc_empty[0]);
-            ++cuse0;
+            if (lane == 0) mbar_arrive(&S.acc_empty[a]);
+            if (a) ++cuse1; else ++cuse0;
+            ++tseg;
         }
     };
     // x += (sum of g's partials); x_g = x * gn (blocked hi/lo); per (row, 128-feature
@@ -962,12 +964,10 @@ __device__ __forceinline__ void mega_compute(const MegaParams &p, MegaSmem &S, u
                         }
                         named_bar_sync(hb, 128);
                         if (half == 0) DETAIL(5);
-                        if (ht == 0) {
-                            fence_acq_rel_gpu();
-                            const int old = atomicAdd(&p.att_cnt[u.row * p.KVH + u.kvh], 1);
+                        if (ht == 0) {  // one acquire-release count: publishes this split, sees the others
+                            const int old = atom_add_acq_rel_gpu(&p.att_cnt[u.row * p.KVH + u.kvh], 1);
                             S.last_flag2[half] = old == u.nsplit - 1;
                             if (S.last_flag2[half]) p.att_cnt[u.row * p.KVH + u.kvh] = 0;
-                            fence_acq_rel_gpu();
                         }
                         named_bar_sync(hb, 128);
                         if (half == 0) DETAIL(6);
@@ -1134,7 +1134,7 @@ __device__ __forceinline__ void mega_compute(const MegaParams &p, MegaSmem &S, u
         const float rs = act ? S.rstd[my_row] : 0.f;
         for (int64_t u = u0; u < u1; u += g.kch) {
             const int t = (int)(u / g.kch);
-            const int a = lmseg & 1;
+            const int a = tseg & 1;
             mwait(&S.acc_full[a], (a ? cuse1 : cuse0) & 1, err, ab);
             tc_fence_after();
             if (quarter_live && half * 128 < tile_rows(g, t)) {
@@ -1159,7 +1159,7 @@ __device__ __forceinline__ void mega_compute(const MegaParams &p, MegaSmem &S, u
             __syncwarp();
             if (lane == 0) mbar_arrive(&S.acc_empty[a]);
             if (a) ++cuse1; else ++cuse0;
-            ++lmseg;
+            ++tseg;
         }
         named_bar_sync(1, kMegaCThreads);
         if (ctid == 0) MEGA_STAMP(1 + kPhasesPerLayer * p.layers, 0);

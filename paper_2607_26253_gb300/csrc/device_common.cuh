@@ -187,6 +187,7 @@ __device__ __forceinline__ void tc_commit(uint64_t *bar) {
 // 32 lanes x 32 consecutive fp32 columns: thread l of the warp receives lane (base + l).
 __device__ __forceinline__ void tmem_ld_32x32b_x32(uint32_t taddr, float (&v)[32]) {
     uint32_t r[32];
+    __syncwarp();  // .aligned: the whole warp converged (lanes may leave a preceding wait loop apart)
     asm volatile(
         "tcgen05.ld.sync.aligned.32x32b.x32.b32 "
         "{%0,%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15,"
@@ -222,6 +223,13 @@ __device__ __forceinline__ void fence_proxy_async_global() { asm volatile("fence
 // __threadfence): orders this thread's prior accesses, and those of its CTA made visible to
 // it by a barrier, before its later ones.
 __device__ __forceinline__ void fence_acq_rel_gpu() { asm volatile("fence.acq_rel.gpu;" ::: "memory"); }
+// Atomic add with acquire-release semantics at GPU scope (a release of the caller's prior
+// writes, and of writes ordered before them by a barrier, plus an acquire): returns the old value.
+__device__ __forceinline__ int atom_add_acq_rel_gpu(int *p, int v) {
+    int old;
+    asm volatile("atom.acq_rel.gpu.global.add.s32 %0, [%1], %2;" : "=r"(old) : "l"(p), "r"(v) : "memory");
+    return old;
+}
 
 __device__ __forceinline__ unsigned long long ld_relaxed_u64(const unsigned long long *p) {
     unsigned long long v;
@@ -237,6 +245,7 @@ __device__ __forceinline__ unsigned long long ld_acquire_u64(const unsigned long
 // 32 lanes x 8 consecutive fp32 columns.
 __device__ __forceinline__ void tmem_ld_32x32b_x8(uint32_t taddr, float (&v)[8]) {
     uint32_t r[8];
+    __syncwarp();  // .aligned: the whole warp converged
     asm volatile("tcgen05.ld.sync.aligned.32x32b.x8.b32 {%0,%1,%2,%3,%4,%5,%6,%7}, [%8];"
                  : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]), "=r"(r[7])
                  : "r"(taddr)
