@@ -638,9 +638,8 @@ __device__ __forceinline__ void mega_compute(const MegaParams &p, MegaSmem &S, u
         if (x_operand) fence_proxy_async_global();
         named_bar_sync(1, kMegaCThreads);
         if (ctid == 0) {
-            fence_acq_rel_gpu();
             MEGA_STAMP(idx, 0);
-            atomicAdd(&p.cnt[idx * kCntStride], 1ull);
+            red_add_release_gpu(&p.cnt[idx * kCntStride], 1ull);
         }
     };
     auto wait_phase = [&](int idx) {

@@ -223,6 +223,11 @@ __device__ __forceinline__ void fence_proxy_async_global() { asm volatile("fence
 // __threadfence): orders this thread's prior accesses, and those of its CTA made visible to
 // it by a barrier, before its later ones.
 __device__ __forceinline__ void fence_acq_rel_gpu() { asm volatile("fence.acq_rel.gpu;" ::: "memory"); }
+// Reduction (no return) with release semantics at GPU scope: publishes the caller's prior
+// writes and those ordered before them by a barrier.
+__device__ __forceinline__ void red_add_release_gpu(unsigned long long *p, unsigned long long v) {
+    asm volatile("red.release.gpu.global.add.u64 [%0], %1;" ::"l"(p), "l"(v) : "memory");
+}
 // Atomic add with acquire-release semantics at GPU scope (a release of the caller's prior
 // writes, and of writes ordered before them by a barrier, plus an acquire): returns the old value.
 __device__ __forceinline__ int atom_add_acq_rel_gpu(int *p, int v) {
