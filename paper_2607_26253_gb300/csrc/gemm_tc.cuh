@@ -136,122 +136,122 @@ __device__ __forceinline__ void gemm_epilogue_chunk(const GemmParams &p, GemmSme
 #pragma unroll
         for (int c = 0; c < 32; ++c)
             if (c < ncols) p.y_f32[(int64_t)(r_base + c0 + c) * p.ld + n] = v[c];
-        return;
-    }
-    if constexpr (EPI == EPI_QKV || EPI == EPI_SWIGLU || EPI == EPI_LMHEAD) {
+    } else {
+        if constexpr (EPI == EPI_QKV || EPI == EPI_SWIGLU || EPI == EPI_LMHEAD) {
 #pragma unroll
-        for (int c = 0; c < 32; ++c) v[c] *= S.inv_rms[c0 + c];
-    }
-    if constexpr (EPI == EPI_RESID) {
-        const float g = bf16_to_f32(p.g_next[n]);
-        float xo[32];
-#pragma unroll
-        for (int c = 0; c < 32; ++c)  // every load before any store (the stores may alias)
-            xo[c] = (c < ncols) ? __ldcg(&p.x_f32[(int64_t)(r_base + c0 + c) * p.ld + n]) : 0.f;
-#pragma unroll
-        for (int c = 0; c < 32; ++c) {
-            if (c < ncols) {
-                const int64_t idx = (int64_t)(r_base + c0 + c) * p.ld + n;
-                const float x = xo[c] + v[c];
-                p.x_f32[idx] = x;
-                uint16_t hi, lo;
-                split_bf16(x * g, hi, lo);
-                p.xg_out[idx] = hi;
-                p.xg_lo[idx] = lo;
-                v[c] = x * x;
-            }
+            for (int c = 0; c < 32; ++c) v[c] *= S.inv_rms[c0 + c];
         }
-    }
-    if constexpr (EPI == EPI_LMHEAD) {
+        if constexpr (EPI == EPI_RESID) {
+            const float g = bf16_to_f32(p.g_next[n]);
+            float xo[32];
 #pragma unroll
-        for (int c = 0; c < 32; ++c) {
-            if (c < ncols) {
-                const int r = r_base + c0 + c;
-                if (p.y_f32) p.y_f32[(int64_t)r * p.ld + n] = v[c];
-                v[c] += gumbel_from_hash(splitmix_at(S.row_seed[c0 + c], (uint64_t)n + 1));
-            }
-        }
-    }
-    // stage the chunk in shared memory for the cross-feature exchanges / reductions
-#pragma unroll
-    for (int c = 0; c < 32; ++c) S.xch[mrow * kEpiLd + c] = v[c];
-    named_bar_sync(1, 128);
-    if constexpr (EPI == EPI_QKV) {
-        const int hd = p.head_dim, half = hd >> 1;
-        const int head = n / hd, i = n - head * hd;
-        const int partner = (i < half) ? mrow + half : mrow - half;
-        const int fi = (i < half) ? i : i - half;
-        const int nq = p.n_heads, nkv = p.n_kv;
-        const bool rot = head < nq + nkv;  // q or k: rotate the pair (i, i + hd/2)
-        float2 cs[32];
-#pragma unroll
-        for (int c = 0; c < 32; ++c)  // every table load before any store
-            cs[c] = (rot && c < ncols) ? __ldg(&p.rope[(int64_t)S.row_pos[c0 + c] * half + fi]) : make_float2(1.f, 0.f);
-#pragma unroll
-        for (int c = 0; c < 32; ++c) {
-            if (c < ncols) {
-                const int r = r_base + c0 + c;
-                float y = v[c];
-                if (rot) {
-                    const float o = S.xch[partner * kEpiLd + c];
-                    y = (i < half) ? (y * cs[c].x - o * cs[c].y) : (y * cs[c].x + o * cs[c].y);
-                }
-                if (head < nq) {
-                    p.q_out[(int64_t)r * (nq * hd) + n] = f32_to_f16_sat(y);
-                } else {
-                    const int isv = head >= nq + nkv;
-                    const int kvh = head - nq - isv * nkv;
-                    uint16_t *dst = p.kv + (int64_t)S.row_slot[c0 + c] * p.kv_slot_stride +
-                                    ((int64_t)(isv * nkv + kvh) * p.kv_cap + S.row_pos[c0 + c]) * hd + i;
-                    *dst = f32_to_f16_sat(y);
-                }
-            }
-        }
-    } else if constexpr (EPI == EPI_SWIGLU) {
-        if (mrow < 64) {
-            const int f = m_tile * 64 + mrow;
+            for (int c = 0; c < 32; ++c)  // every load before any store (the stores may alias)
+                xo[c] = (c < ncols) ? __ldcg(&p.x_f32[(int64_t)(r_base + c0 + c) * p.ld + n]) : 0.f;
 #pragma unroll
             for (int c = 0; c < 32; ++c) {
                 if (c < ncols) {
-                    const float g = v[c], u = S.xch[(mrow + 64) * kEpiLd + c];
-                    const float h = g / (1.0f + expf(-g)) * u;
+                    const int64_t idx = (int64_t)(r_base + c0 + c) * p.ld + n;
+                    const float x = xo[c] + v[c];
+                    p.x_f32[idx] = x;
                     uint16_t hi, lo;
-                    split_bf16(h, hi, lo);
-                    p.h_out[(int64_t)(r_base + c0 + c) * p.ld + f] = hi;
-                    p.h_lo[(int64_t)(r_base + c0 + c) * p.ld + f] = lo;
+                    split_bf16(x * g, hi, lo);
+                    p.xg_out[idx] = hi;
+                    p.xg_lo[idx] = lo;
+                    v[c] = x * x;
                 }
             }
         }
-    } else if constexpr (EPI == EPI_RESID || EPI == EPI_LMHEAD) {
-        // thread etid reduces column c = etid / 4 over features [32 * (etid % 4), +32)
-        const int c = etid >> 2, part = etid & 3;
-        if constexpr (EPI == EPI_RESID) {
-            float s = 0.f;
-            for (int f = 0; f < 32; ++f) s += S.xch[(part * 32 + f) * kEpiLd + c];
-            s += __shfl_xor_sync(0xffffffffu, s, 1);
-            s += __shfl_xor_sync(0xffffffffu, s, 2);
-            if (part == 0 && c < ncols) p.ssq_out[(int64_t)m_tile * p.rows_cap + r_base + c0 + c] = s;
-        } else {
-            float best = -INFINITY;
-            int bi = 0x7fffffff;
-            for (int f = 0; f < 32; ++f) {
-                const float z = S.xch[(part * 32 + f) * kEpiLd + c];
-                if (z > best) { best = z; bi = m_tile * kTileM + part * 32 + f; }
-            }
+        if constexpr (EPI == EPI_LMHEAD) {
 #pragma unroll
-            for (int o = 1; o <= 2; o <<= 1) {
-                const float ob = __shfl_xor_sync(0xffffffffu, best, o);
-                const int oi = __shfl_xor_sync(0xffffffffu, bi, o);
-                if (ob > best || (ob == best && oi < bi)) { best = ob; bi = oi; }
-            }
-            if (part == 0 && c < ncols) {
-                const int r = r_base + c0 + c;
-                p.arg_val[(int64_t)r * p.m_tiles + m_tile] = best;
-                p.arg_idx[(int64_t)r * p.m_tiles + m_tile] = bi;
+            for (int c = 0; c < 32; ++c) {
+                if (c < ncols) {
+                    const int r = r_base + c0 + c;
+                    if (p.y_f32) p.y_f32[(int64_t)r * p.ld + n] = v[c];
+                    v[c] += gumbel_from_hash(splitmix_at(S.row_seed[c0 + c], (uint64_t)n + 1));
+                }
             }
         }
+        // stage the chunk in shared memory for the cross-feature exchanges / reductions
+#pragma unroll
+        for (int c = 0; c < 32; ++c) S.xch[mrow * kEpiLd + c] = v[c];
+        named_bar_sync(1, 128);
+        if constexpr (EPI == EPI_QKV) {
+            const int hd = p.head_dim, half = hd >> 1;
+            const int head = n / hd, i = n - head * hd;
+            const int partner = (i < half) ? mrow + half : mrow - half;
+            const int fi = (i < half) ? i : i - half;
+            const int nq = p.n_heads, nkv = p.n_kv;
+            const bool rot = head < nq + nkv;  // q or k: rotate the pair (i, i + hd/2)
+            float2 cs[32];
+#pragma unroll
+            for (int c = 0; c < 32; ++c)  // every table load before any store
+                cs[c] = (rot && c < ncols) ? __ldg(&p.rope[(int64_t)S.row_pos[c0 + c] * half + fi]) : make_float2(1.f, 0.f);
+#pragma unroll
+            for (int c = 0; c < 32; ++c) {
+                if (c < ncols) {
+                    const int r = r_base + c0 + c;
+                    float y = v[c];
+                    if (rot) {
+                        const float o = S.xch[partner * kEpiLd + c];
+                        y = (i < half) ? (y * cs[c].x - o * cs[c].y) : (y * cs[c].x + o * cs[c].y);
+                    }
+                    if (head < nq) {
+                        p.q_out[(int64_t)r * (nq * hd) + n] = f32_to_f16_sat(y);
+                    } else {
+                        const int isv = head >= nq + nkv;
+                        const int kvh = head - nq - isv * nkv;
+                        uint16_t *dst = p.kv + (int64_t)S.row_slot[c0 + c] * p.kv_slot_stride +
+                                        ((int64_t)(isv * nkv + kvh) * p.kv_cap + S.row_pos[c0 + c]) * hd + i;
+                        *dst = f32_to_f16_sat(y);
+                    }
+                }
+            }
+        } else if constexpr (EPI == EPI_SWIGLU) {
+            if (mrow < 64) {
+                const int f = m_tile * 64 + mrow;
+#pragma unroll
+                for (int c = 0; c < 32; ++c) {
+                    if (c < ncols) {
+                        const float g = v[c], u = S.xch[(mrow + 64) * kEpiLd + c];
+                        const float h = g / (1.0f + expf(-g)) * u;
+                        uint16_t hi, lo;
+                        split_bf16(h, hi, lo);
+                        p.h_out[(int64_t)(r_base + c0 + c) * p.ld + f] = hi;
+                        p.h_lo[(int64_t)(r_base + c0 + c) * p.ld + f] = lo;
+                    }
+                }
+            }
+        } else if constexpr (EPI == EPI_RESID || EPI == EPI_LMHEAD) {
+            // thread etid reduces column c = etid / 4 over features [32 * (etid % 4), +32)
+            const int c = etid >> 2, part = etid & 3;
+            if constexpr (EPI == EPI_RESID) {
+                float s = 0.f;
+                for (int f = 0; f < 32; ++f) s += S.xch[(part * 32 + f) * kEpiLd + c];
+                s += __shfl_xor_sync(0xffffffffu, s, 1);
+                s += __shfl_xor_sync(0xffffffffu, s, 2);
+                if (part == 0 && c < ncols) p.ssq_out[(int64_t)m_tile * p.rows_cap + r_base + c0 + c] = s;
+            } else {
+                float best = -INFINITY;
+                int bi = 0x7fffffff;
+                for (int f = 0; f < 32; ++f) {
+                    const float z = S.xch[(part * 32 + f) * kEpiLd + c];
+                    if (z > best) { best = z; bi = m_tile * kTileM + part * 32 + f; }
+                }
+#pragma unroll
+                for (int o = 1; o <= 2; o <<= 1) {
+                    const float ob = __shfl_xor_sync(0xffffffffu, best, o);
+                    const int oi = __shfl_xor_sync(0xffffffffu, bi, o);
+                    if (ob > best || (ob == best && oi < bi)) { best = ob; bi = oi; }
+                }
+                if (part == 0 && c < ncols) {
+                    const int r = r_base + c0 + c;
+                    p.arg_val[(int64_t)r * p.m_tiles + m_tile] = best;
+                    p.arg_idx[(int64_t)r * p.m_tiles + m_tile] = bi;
+                }
+            }
+        }
+        named_bar_sync(1, 128);  // xch reused by the next chunk
     }
-    named_bar_sync(1, 128);  // xch reused by the next chunk
 }
 
 template <int EPI>
