@@ -64,3 +64,13 @@ def test_working_set_equal_to_pool(handle):
     w = synth.sweep_workload(8, 2, 0.45, 0, n_prompts=8192, target_B=8192)
     out = _compare(handle, w)
     assert out.counters["committed"] == 0
+
+
+def test_ds_and_uniform_parameterisations(handle):
+    # the comparison baselines as Algorithm 1 parameterisations (probe n0 = k, tau_low = 0;
+    # uniform: a pool of B prompts with a budget of B k rollouts), bit-exact against the oracle
+    from dataclasses import replace
+    for k in (4, 8, 16):
+        w = synth.sweep_workload(k, 2, 0.45, 5, n_prompts=8192, target_B=1024)
+        _compare(handle, replace(w, n0=k, tau=0.0))
+        _compare(handle, replace(w, n0=k, tau=0.0, n_prompts=1024, budget_N=1024 * k))
