@@ -105,13 +105,17 @@ SHAPE_3B = ModelShape("3B-shaped", layers=36, d_model=2048, n_heads=16, n_kv_hea
 
 @dataclass(frozen=True)
 class Lengths:
-    """Rollout-length law: 'uniform' on [lo, hi] or 'lognormal' with median/sigma, capped."""
+    """Rollout-length law: 'uniform' on [lo, hi] or 'lognormal' with median/sigma, capped.
+    hard_scale > 0 (lognormal only) ties length to difficulty: prompt q's median becomes
+    median * (1 + hard_scale * (1 - p_q)), p_q its latent success rate, so the rollouts of
+    all-fail prompts are the longest (hard_scale = 1: twice the all-pass median)."""
     kind: str
     lo: int = 1
     hi: int = 1
     median: float = 1.0
     sigma: float = 0.5
     cap: int = 1
+    hard_scale: float = 0.0
 
     @property
     def max_len(self) -> int:
@@ -228,7 +232,11 @@ def rollout_lengths(w: Workload) -> np.ndarray:
     if L.kind == "uniform":
         return rng.integers(L.lo, L.hi + 1, size=shape, dtype=np.int64).astype(np.int32)
     z = rng.standard_normal(shape)
-    x = np.rint(np.exp(math.log(L.median) + L.sigma * z))
+    log_med = math.log(L.median)
+    if L.hard_scale > 0:
+        p = latent_thresholds(w).astype(np.float64) / 4294967296.0
+        log_med = np.log(L.median * (1.0 + L.hard_scale * (1.0 - p)))[:, None]
+    x = np.rint(np.exp(log_med + L.sigma * z))
     return np.clip(x, 1, L.cap).astype(np.int32)
 
 

@@ -74,3 +74,17 @@ def test_ds_and_uniform_parameterisations(handle):
         w = synth.sweep_workload(k, 2, 0.45, 5, n_prompts=8192, target_B=1024)
         _compare(handle, replace(w, n0=k, tau=0.0))
         _compare(handle, replace(w, n0=k, tau=0.0, n_prompts=1024, budget_N=1024 * k))
+
+
+def test_length_difficulty_workload_sara_and_ds():
+    # lengths tied to difficulty (all-fail prompts longest): token counts bit-exact for SARA and DS
+    from dataclasses import replace
+    import paper_2607_26253_gb300 as pkg
+    cfg = pkg.model_cfg(None, max_prompts=8192, max_active=1024, max_seqs=1, max_prompt_len=1, max_gen_len=4096,
+                        max_k=8)
+    L = synth.Lengths("lognormal", median=1024, sigma=0.5, cap=4096, hard_scale=1.0)
+    with pkg.Handle(cfg) as h:
+        for rep in range(2):
+            w = replace(synth.sweep_workload(8, 2, 0.45, rep, n_prompts=8192, target_B=1024), lengths=L)
+            _compare(h, w)
+            _compare(h, replace(w, n0=8, tau=0.0))

@@ -91,3 +91,31 @@ def test_sara_spends_fewer_rollouts_than_ds_for_the_same_target():
         assert sara["committed"] >= w.target_B and ds["committed"] >= w.target_B
         saved.append(1 - sara["rollouts"] / ds["rollouts"])
     assert min(saved) > 0.12, saved
+
+
+def test_hard_prompts_run_longest_in_the_length_generator():
+    # median * (1 + hard_scale (1 - p)): all-fail prompts (p = 0) twice the all-pass median at
+    # hard_scale = 1, so their mean lengths (same sigma, no cap in reach) are in ratio 2
+    w = replace(synth.sweep_workload(8, 2, 0.45, 0, n_prompts=8192, target_B=1024),
+                lengths=synth.Lengths("lognormal", median=1024, sigma=0.5, cap=10 ** 7, hard_scale=1.0))
+    si = synth.step_inputs(w)
+    p = si.thresholds.astype(np.float64) / 2.0 ** 32
+    Lm = si.lengths.astype(np.float64).mean(axis=1)
+    ratio = Lm[p == 0].mean() / Lm[p >= 1].mean()
+    assert abs(ratio - 2.0) < 0.05, ratio
+    base = synth.step_inputs(replace(w, lengths=replace(w.lengths, hard_scale=0.0)))
+    assert abs(base.lengths[p == 0].mean() / base.lengths[p >= 1].mean() - 1.0) < 0.05
+
+
+def test_token_savings_exceed_rollout_savings_when_hard_prompts_run_longest():
+    # abandoned all-fail groups are the longest, so cutting them after the probe saves a larger
+    # share of tokens than of rollouts (the paper's Fig. 6 observation)
+    L = synth.Lengths("lognormal", median=1024, sigma=0.5, cap=4096, hard_scale=1.0)
+    tot = np.zeros(4)
+    for rep in range(4):
+        w = replace(synth.sweep_workload(8, 2, 0.45, rep, n_prompts=8192, target_B=1024), lengths=L)
+        sara = oc.collect_workload(w).counters
+        ds = oc.collect_workload(_ds(w)).counters
+        tot += [sara["rollouts"], ds["rollouts"], sara["gen_tokens"], ds["gen_tokens"]]
+    roll_saving, tok_saving = 1 - tot[0] / tot[1], 1 - tot[2] / tot[3]
+    assert roll_saving > 0.15 and tok_saving > roll_saving, (roll_saving, tok_saving)
