@@ -10,6 +10,8 @@ method's arithmetic.
                      rational arithmetic, plain C (oracle/controller.c).
   oracle.decode      O2: the decoder policy forward pass and Gumbel-max
                      sampling in float64 numpy.
+  oracle.async_schedule  O1a: the asynchronous per-prompt variant of the step
+                     (no round barrier), on O1's predictor and rule.
 """
 import os
 import subprocess
