@@ -9,11 +9,11 @@
 // activations) ahead of the consumers through a ring of 32 KB shared-memory slots, across
 // phase boundaries.  Only the small activation operands wait for the previous phase.
 //
-// GEMM orientation: the activation rows are the MMA's M (128, rows beyond the live count
-// are don't-care) and 256 weight rows its N, so one tcgen05.mma (K = 16) consumes 8 KB of
-// weights.  The instruction's cost hardly depends on N, so this keeps the tensor pipe off
-// the critical path at the HBM rate even with the activation split into a bf16 hi/lo pair
-// (two MMAs per k-step, ~16 mantissa bits of the activation).
+// GEMM orientation: the activation rows are the MMA's M and 256 weight rows its N, so one
+// tcgen05.mma (K = 16) consumes 8 KB of weights (~133 cycles at M = 64 or 128 alike).  The
+// activation is a bf16 hi/lo pair (~16 mantissa bits); up to 64 live rows both parts sit in
+// one stacked operand and a k-step is one MMA, above that two MMAs (hi, lo) accumulate.
+// Rows beyond the live count are don't-care.
 //
 // Split-K: a phase's (tile, k-chunk) units are cut into equal contiguous ranges over its
 // CTAs; each CTA stores its fp32 partial tile with plain stores and the consuming phase
@@ -30,8 +30,8 @@
 //   0 QKV   x_g W_qkv^T -> partials        (a subset of the CTAs: few tiles)
 //   1 FIN_Q q, k, v = RMSNorm scale + RoPE of the summed partials, fp16, once per row; the
 //           new k, v appended to the KV cache
-//   2 ATT   softmax(q K^T) V on the tensor cores per 128-position split; the last split of a
-//           row to finish merges them
+//   2 ATT   softmax(q K^T) V on the tensor cores, 128-position KV blocks, online softmax
+//           over a split's blocks; the last split of a row to finish merges the splits
 //   3 O     att W_o^T -> partials           (a subset of the CTAs)
 //   4 FIN_O x += sum; x_g = x * g_mlp (bf16 hi/lo, blocked); per-row sum of squares
 //   5 GU    x_g W_gu^T -> partials          (gate / up interleaved in 64-row blocks)
@@ -61,9 +61,9 @@ constexpr int kSlotBytes = 32768;
 constexpr int kRingBytes = 4 * 32768 + 65536;  // W slots, then the X stages
 constexpr int kMaxXStages = 8;
 constexpr int kTileN = 256;           // weight rows (output features) per GEMM tile
-constexpr int kKVPos = 128;           // positions per KV block and per attention split
+constexpr int kKVPos = 128;           // positions per KV block (an attention split holds `span` blocks)
 constexpr int kKVBlockBytes = 65536;  // K 2 x 16 KB + V^T 2 x 16 KB
-constexpr int kMegaMaxSplits = 96;
+constexpr int kMegaMaxSplits = 96;    // splits per row a merge handles (context <= 96 blocks)
 constexpr int kPhasesPerLayer = 9;
 // phases of a layer (counter index 1 + 9 l + phase)
 enum : int { kPhQKV = 0, kPhFinQ = 1, kPhAtt = 2, kPhO = 3, kPhFinO = 4, kPhGU = 5, kPhFinGU = 6, kPhDown = 7,
