@@ -110,6 +110,15 @@ typedef struct {
     int32_t alpha0, beta0;     /* integer Beta prior, each 1..8 (default 1, 1) */
     int32_t target_B;          /* effective groups wanted, 1..max_active */
     uint64_t sample_seed;      /* seed of the temperature-1 Gumbel-max sampler */
+    int32_t schedule;          /* 0: synchronised rounds (Algorithm 1, the default);
+                                  1: asynchronous per-prompt: a prompt is decided when its own
+                                     rollouts finish and refill happens at the next decode step;
+                                  2: as 1, drawing a fresh prompt only if the budget covers it
+                                     and every prompt in flight running to k rollouts.
+                                  1 and 2 run on controller-only handles (layers == 0): decode
+                                  time comes from the length table (decode_steps), rounds
+                                  counts the step boundaries with decisions and decided_round
+                                  holds the index of the deciding one (capped at 32767). */
 } sara_thresholds;
 
 /* Results of one step.  Array pointers may be NULL (not written); they are host or device

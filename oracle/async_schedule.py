@@ -47,6 +47,7 @@ class AsyncResult:
     n: np.ndarray             # uint8[P] rollouts spent on each prompt
     s: np.ndarray             # uint8[P] successes observed
     decided_step: np.ndarray  # int32[P]: end of the decode step of the commit / abandon, else -1
+    decided_event: np.ndarray  # int32[P]: index of that step boundary among those with decisions
     counters: dict
 
     @property
@@ -74,6 +75,7 @@ def collect_step(thresholds: np.ndarray, lengths: np.ndarray, *, k: int, n0: int
     n = np.zeros(P, np.int64)
     s = np.zeros(P, np.int64)
     decided = np.full(P, -1, np.int32)
+    decided_ev = np.full(P, -1, np.int32)
     batch = {}  # q -> rollouts of its batch in flight
     heap = []   # (decision step, q)
     used = tokens = drawn = 0
@@ -110,6 +112,7 @@ def collect_step(thresholds: np.ndarray, lengths: np.ndarray, *, k: int, n0: int
         while heap and heap[0][0] == t:
             done.append(heapq.heappop(heap)[1])
         done.sort()
+        ev = events
         events += 1
         last_step = t
         cont = []
@@ -121,10 +124,12 @@ def collect_step(thresholds: np.ndarray, lengths: np.ndarray, *, k: int, n0: int
             if d == oc.COMMIT:
                 status[q] = oc.COMMITTED
                 decided[q] = t
+                decided_ev[q] = ev
                 C += 1
             elif d == oc.ABANDON:
                 status[q] = oc.ABANDONED
                 decided[q] = t
+                decided_ev[q] = ev
             else:
                 cont.append(q)
         if stopped or C >= target_B:
@@ -146,7 +151,7 @@ def collect_step(thresholds: np.ndarray, lengths: np.ndarray, *, k: int, n0: int
         "committed": int((status == oc.COMMITTED).sum()), "abandoned": int((status == oc.ABANDONED).sum()),
         "incomplete": int((status == oc.INCOMPLETE).sum()), "prompts_drawn": drawn,
     }
-    return AsyncResult(status, n.astype(np.uint8), s.astype(np.uint8), decided, counters)
+    return AsyncResult(status, n.astype(np.uint8), s.astype(np.uint8), decided, decided_ev, counters)
 
 
 def collect_workload(w, si=None, reserve: bool = False) -> AsyncResult:

@@ -474,3 +474,151 @@ static __global__ void __launch_bounds__(kCtlThreads, 1) ctl_init_kernel(StepPtr
 }
 
 }  // namespace sara
+
+namespace sara {
+
+// ------------------------------------------------------------------------------------------
+// Asynchronous per-prompt schedule (controller-only handles: decode-step time comes from the
+// length table, nothing is decoded).  Algorithm 1 without the round barrier: a prompt is
+// decided at the end of the decode step in which its batch in flight (the n0-rollout probe, or
+// the one rollout of a continue decision) finishes; a rollout of length L started at step t0
+// occupies steps t0 .. t0 + L - 1.  The prompts decided at one step boundary follow the round
+// rules as one round: DECIDE (Eq. decide) in stream order, stop issuing once |C| >= B,
+// otherwise fund the continuing ones by p_eff rank (ties: stream order) while the budget
+// allows (else INCOMPLETE), then draw fresh prompts in stream order while fewer than B - |C|
+// are in flight and a whole probe fits the budget; new rollouts start at the next step.  No
+// cancellation: after the stop, rollouts in flight finish and their prompts are decided.
+// reserve: a fresh prompt is drawn only if the budget covers it and every prompt in flight
+// running to k rollouts.  decided_round receives the index of the deciding event (step
+// boundary with decisions), capped at 32767.  One thread runs the event loop over a binary
+// min-heap of (decision step << 32 | prompt) in dynamic shared memory (prompts in flight
+// <= B <= max_active entries).
+constexpr int kAsyncMaxInFlight = 8192;
+
+static __global__ void __launch_bounds__(kCtlThreads, 1) ctl_async_kernel(StepPtrs c, int reserve, int heap_cap) {
+    extern __shared__ uint64_t heap[];
+    pdl_wait_prior_grids();
+    if (threadIdx.x != 0) return;
+    const StepConst K = *c.kc;
+    StepVars &V = *c.v;
+    const int k = K.k, n0 = K.n0, B = K.B, P = K.P;
+    const int64_t N = K.N;
+    int hn = 0;
+    int64_t used = 0, tokens = 0, resv = 0, last = -1;
+    int C = 0, cursor = 0, drawn = 0, events = 0;
+    bool stopped = false, bad = false;
+
+    auto push = [&](uint64_t key) {
+        int i = hn++;
+        while (i > 0) {
+            const int par = (i - 1) >> 1;
+            if (heap[par] <= key) break;
+            heap[i] = heap[par];
+            i = par;
+        }
+        heap[i] = key;
+    };
+    auto pop = [&]() -> uint64_t {
+        const uint64_t top = heap[0];
+        const uint64_t x = heap[--hn];
+        int i = 0;
+        for (;;) {
+            int ch = 2 * i + 1;
+            if (ch >= hn) break;
+            if (ch + 1 < hn && heap[ch + 1] < heap[ch]) ++ch;
+            if (heap[ch] >= x) break;
+            heap[i] = heap[ch];
+            i = ch;
+        }
+        if (hn > 0) heap[i] = x;
+        return top;
+    };
+    // issue the next `cnt` rollouts of prompt q, starting at decode step `start`
+    auto issue = [&](int q, int cnt, int64_t start) {
+        const int n = c.q_n[q];
+        int64_t mx = 0;
+        for (int j = n; j < n + cnt; ++j) {
+            const int L = c.p_len[(int64_t)q * k + j];
+            if (L < 1 || L > K.max_gen) bad = true;
+            tokens += L;
+            mx = max(mx, (int64_t)L);
+        }
+        used += cnt;
+        if (reserve) resv += k - (n + cnt);
+        const int64_t fin = start + mx - 1;  // the batch's decision step
+        if (hn < heap_cap && fin <= 0xffffffffLL) push(((uint64_t)fin << 32) | (uint32_t)q);
+        else bad = true;
+    };
+    auto draw = [&](int64_t start) {
+        while (!bad && cursor < P && hn < B - C && used + (reserve ? k : n0) + resv <= N) {
+            const int q = cursor++;
+            c.q_status[q] = ST_ACTIVE;
+            ++drawn;
+            issue(q, n0, start);
+        }
+    };
+
+    draw(0);
+    while (hn > 0 && !bad) {
+        const int64_t t = (int64_t)(heap[0] >> 32);
+        int ncont = 0;
+        const int ev = events++;
+        last = t;
+        while (hn > 0 && (int64_t)(heap[0] >> 32) == t) {  // ascending stream index within a step
+            const int q = (int)(pop() & 0xffffffffu);
+            int n = c.q_n[q], s = c.q_s[q];
+            const int cnt = n == 0 ? n0 : 1;
+            for (int j = n; j < n + cnt; ++j) s += verdict_of(K.reward_seed, q, j, c.p_thr[q]);
+            n += cnt;
+            c.q_n[q] = (uint8_t)n;
+            c.q_s[q] = (uint8_t)s;
+            if (reserve) resv -= k - n;
+            const int d = c.dec_tab[n * kTabDim + s];
+            if (d == D_COMMIT) {
+                c.q_status[q] = ST_COMMITTED;
+                c.q_round[q] = (int16_t)min(ev, 32767);
+                ++C;
+            } else if (d == D_ABANDON) {
+                c.q_status[q] = ST_ABANDONED;
+                c.q_round[q] = (int16_t)min(ev, 32767);
+            } else {
+                c.act[ncont++] = q;
+            }
+        }
+        if (stopped || C >= B) {
+            stopped = true;
+            for (int i = 0; i < ncont; ++i) c.q_status[c.act[i]] = ST_INCOMPLETE;
+            continue;
+        }
+        // continuing prompts by p_eff rank, then stream index (insertion sort: few per event)
+        for (int i = 1; i < ncont; ++i) {
+            const int q = c.act[i];
+            const int rq = c.rank_tab[c.q_n[q] * kTabDim + c.q_s[q]];
+            int j = i - 1;
+            while (j >= 0) {
+                const int p2 = c.act[j];
+                const int rp = c.rank_tab[c.q_n[p2] * kTabDim + c.q_s[p2]];
+                if (rp < rq || (rp == rq && p2 < q)) break;
+                c.act[j + 1] = p2;
+                --j;
+            }
+            c.act[j + 1] = q;
+        }
+        for (int i = 0; i < ncont; ++i) {
+            const int q = c.act[i];
+            if (used + 1 <= N) issue(q, 1, t + 1);
+            else c.q_status[q] = ST_INCOMPLETE;
+        }
+        draw(t + 1);
+    }
+    if (bad) report_error(&V.err, ERR_BOUNDS);
+    V.used = used;
+    V.gen_tokens = tokens;
+    V.drawn = drawn;
+    V.sched_steps = last + 1;
+    V.rounds_done = events;
+    V.live = 0;
+    V.done = 1;
+}
+
+}  // namespace sara

@@ -788,6 +788,9 @@ void collect_impl(sara_handle &h, const sara_prompts *pr, int64_t N, int32_t k, 
         throw SaraError(SARA_EINVAL, "prior out of range (1..8)");
     if (t->target_B < 1 || t->target_B > m.max_active) throw SaraError(SARA_EINVAL, "target_B out of range");
     if (P > 0 && (!pr->p_threshold || !pr->lengths)) throw SaraError(SARA_EINVAL, "p_threshold / lengths are NULL");
+    if (t->schedule < 0 || t->schedule > 2) throw SaraError(SARA_EINVAL, "schedule must be 0, 1 or 2");
+    if (t->schedule != 0 && h.has_model)
+        throw SaraError(SARA_EINVAL, "the asynchronous schedule runs on controller-only handles");
     if (h.has_model) {
         if (Lp < 2 || Lp > m.max_prompt_len) throw SaraError(SARA_EINVAL, "prompt_len out of range");
         if (P > 0 && !pr->tokens) throw SaraError(SARA_EINVAL, "tokens are NULL");
@@ -825,8 +828,16 @@ void collect_impl(sara_handle &h, const sara_prompts *pr, int64_t N, int32_t k, 
     }
     if (h.has_model) reset_decode_state(h, s);
     launch(s, false, dim3(1), dim3(kCtlThreads), 0, ctl_init_kernel, h.ptrs);
-    if (h.use_graph) CK(cudaGraphLaunch(h.exec, s));
-    else run_host_loop(h);
+    if (t->schedule != 0) {  // asynchronous per-prompt schedule: one event-loop kernel
+        const int cap = std::min(m.max_active, kAsyncMaxInFlight);
+        const size_t smem = (size_t)cap * sizeof(uint64_t);
+        CK(cudaFuncSetAttribute(ctl_async_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem));
+        launch(s, false, dim3(1), dim3(kCtlThreads), smem, ctl_async_kernel, h.ptrs, t->schedule == 2 ? 1 : 0, cap);
+    } else if (h.use_graph) {
+        CK(cudaGraphLaunch(h.exec, s));
+    } else {
+        run_host_loop(h);
+    }
     // results (one device -> host read per call)
     StepVars v{};
     const cudaMemcpyKind kout = out->on_device ? cudaMemcpyDeviceToDevice : cudaMemcpyDeviceToHost;

@@ -47,7 +47,7 @@ class Prompts(ctypes.Structure):
 class Thresholds(ctypes.Structure):
     _fields_ = [("tau_num", ctypes.c_int64), ("tau_den", ctypes.c_int64), ("commit_min", ctypes.c_int32),
                 ("alpha0", ctypes.c_int32), ("beta0", ctypes.c_int32), ("target_B", ctypes.c_int32),
-                ("sample_seed", ctypes.c_uint64)]
+                ("sample_seed", ctypes.c_uint64), ("schedule", ctypes.c_int32)]
 
 
 class Result(ctypes.Structure):
@@ -207,7 +207,7 @@ class Handle:
     def collect_step(self, *, thresholds, lengths, N: int, k: int, n0: int, tau, target_B: int,
                      reward_seed: int, tokens=None, prompt_len: int | None = None, commit_min: int = 0,
                      prior=(1, 1), sample_seed: int = 0, want_tokens: bool = False,
-                     outputs_on_device: bool = False) -> StepOutput:
+                     outputs_on_device: bool = False, schedule: int = 0) -> StepOutput:
         """One rollout-collection step (Algorithm 1).  Inputs are numpy arrays (host) or torch
         CUDA tensors (device); outputs are numpy arrays, or torch CUDA tensors when
         outputs_on_device."""
@@ -216,7 +216,7 @@ class Handle:
         Lp = int(tokens.shape[1]) if tokens is not None else (prompt_len or 1)
         pr = Prompts(P, Lp, _ptr(tokens), _ptr(thresholds), _ptr(lengths), 1 if on_dev else 0)
         t = tau_fraction(tau)
-        th = Thresholds(t.numerator, t.denominator, commit_min, prior[0], prior[1], target_B, sample_seed)
+        th = Thresholds(t.numerator, t.denominator, commit_min, prior[0], prior[1], target_B, sample_seed, schedule)
         if outputs_on_device:
             import torch
             status = torch.zeros(P, dtype=torch.uint8, device="cuda")

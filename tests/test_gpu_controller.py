@@ -88,3 +88,49 @@ def test_length_difficulty_workload_sara_and_ds():
             w = replace(synth.sweep_workload(8, 2, 0.45, rep, n_prompts=8192, target_B=1024), lengths=L)
             _compare(h, w)
             _compare(h, replace(w, n0=8, tau=0.0))
+
+
+def _compare_async(h, w, si, schedule):
+    from oracle import async_schedule as oa
+    ref = oa.collect_workload(w, si, reserve=schedule == 2)
+    out = h.collect_step(thresholds=si.thresholds, lengths=si.lengths, N=w.budget_N, k=w.k, n0=w.n0, tau=w.tau,
+                         target_B=w.target_B, reward_seed=w.reward_seed, prompt_len=w.prompt_len,
+                         commit_min=w.commit_floor, prior=w.prior, schedule=schedule)
+    assert np.array_equal(out.status, ref.status)
+    assert np.array_equal(out.n, ref.n) and np.array_equal(out.s, ref.s)
+    assert np.array_equal(out.decided_round.astype(np.int32), np.minimum(ref.decided_event, 32767))
+    c = ref.counters
+    for key, v in (("rollouts", c["rollouts"]), ("gen_tokens", c["gen_tokens"]), ("decode_steps", c["decode_steps"]),
+                   ("rounds", c["events"]), ("committed", c["committed"]), ("abandoned", c["abandoned"]),
+                   ("incomplete", c["incomplete"]), ("prompts_drawn", c["prompts_drawn"]),
+                   ("prefill_tokens", c["prefill_tokens"])):
+        assert out.counters[key] == v, (key, out.counters[key], v)
+
+
+def test_async_schedule_bit_exact():
+    # the asynchronous per-prompt schedule (with and without the budget reservation) against
+    # its oracle: random pools, then the 1.5B- and oversampled-shaped schedules
+    import paper_2607_26253_gb300 as pkg
+    cfg = pkg.model_cfg(None, max_prompts=2048, max_active=512, max_seqs=1, max_prompt_len=1, max_gen_len=8192,
+                        max_k=16)
+    rng = np.random.default_rng(21)
+    with pkg.Handle(cfg) as h:
+        for it in range(30):
+            k = int(rng.integers(2, 17))
+            n0 = int(rng.integers(1, k + 1))
+            P = int(rng.integers(1, 2049))
+            B = int(rng.integers(1, min(P, 512) + 1))
+            w = synth.Workload("async", None, n_prompts=P, prompt_len=int(rng.integers(1, 5)), target_B=B, k=k,
+                               n0=n0, tau=float(rng.choice([0.0, 0.3, 0.45, 0.6, 1.0])),
+                               budget_N=int(rng.integers(0, 2 * P * k + 1)), commit_min=int(rng.integers(2, k + 1)),
+                               prior=(int(rng.integers(1, 9)), int(rng.integers(1, 9))),
+                               lengths=synth.Lengths("uniform", lo=1, hi=60), seed_latent=it,
+                               seed_lengths=it + 1, reward_seed=it + 2)
+            si = synth.step_inputs(w)
+            for schedule in (1, 2):
+                _compare_async(h, w, si, schedule)
+        for name in ("1.5b", "oversampled"):
+            w = synth.WORKLOADS[name]
+            si = synth.step_inputs(w)
+            for schedule in (1, 2):
+                _compare_async(h, w, si, schedule)

@@ -44,6 +44,7 @@ def test_equal_lengths_reproduce_the_round_synchronous_oracle():
         dec = sync.decided_round >= 0
         assert np.array_equal(asy.decided_step >= 0, dec)
         assert np.array_equal(asy.decided_step[dec], (sync.decided_round[dec].astype(np.int64) + 1) * Lc - 1)
+        assert np.array_equal(asy.decided_event, sync.decided_round.astype(np.int32))
         for key in ("rollouts", "gen_tokens", "prefill_tokens", "committed", "abandoned", "incomplete",
                     "prompts_drawn"):
             assert asy.counters[key] == sync.counters[key], (it, key)
