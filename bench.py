@@ -5,13 +5,19 @@
 
 A step is one sara_collect_step over a fresh synthetic prompt stream of the named workload:
 probe, decide, refill and decode every issued rollout until the target or the budget is
-reached.  `value` = rollout tokens generated per second over the K timed steps (inputs
-resident in HBM), whole job over all ranks; `e2e` = the same metric through the same call
-with host (pinned) inputs and host outputs, copies inside the timed region.  N > 1 runs one
-replica per GPU on its own shard of the prompt stream (seed offset by rank, no collective
-on the data path); only the final counters are reduced.
+reached.  Every step, warm-up and timed alike, goes through the public call with the
+step's inputs in pinned host memory and its results copied back to pinned host memory, so
+the timed steps are the end-to-end ones:
 
-Rank 0 prints one JSON line.  Data are synthetic (random-init weights, seeded rewards).
+  * `value` = rollout tokens generated per second of the steps' device time with inputs
+    already resident in HBM (the library's CUDA events after the input copies and before the
+    output copies of each call), whole job over all ranks;
+  * `e2e` = the same metric over the whole timed region (CUDA events on the handle's stream
+    around the K calls, host<->device copies included).
+
+N > 1 runs one replica per GPU on its own shard of the prompt stream (seed offset by rank, no
+collective on the data path); only the final counters are reduced.  Rank 0 prints one JSON
+line.  Data are synthetic (random-init weights, seeded rewards and lengths).
 """
 from __future__ import annotations
 
@@ -19,10 +25,12 @@ import argparse
 import json
 import math
 import os
+import platform
 import subprocess
 import sys
 import tempfile
 import time
+from dataclasses import replace
 
 import numpy as np
 
@@ -33,6 +41,8 @@ import synth  # noqa: E402
 
 HERE_PEAKS = os.path.join(ROOT, "MEASURED_PEAKS.json")
 FALLBACK_HBM_GBS = 6800.0
+CPU_SLICE_STEPS = 8        # decode steps of the oracle's teacher-forced slice
+CPU_ONE_THREAD_LAYERS = 2  # layers timed on one thread (scaled to the whole model)
 
 
 def parse():
@@ -50,6 +60,8 @@ def parse():
     ap.add_argument("--iters", type=int, default=5, help="launches in --kernel-profile mode")
     ap.add_argument("--ctx", type=int, default=None, help="context length in --kernel-profile mode "
                     "(default: prompt length + 128)")
+    ap.add_argument("--cpu-slice", action="store_true", help=argparse.SUPPRESS)  # child of the CPU baseline
+    ap.add_argument("--slice-layers", type=int, default=None, help=argparse.SUPPRESS)
     return ap.parse_args()
 
 
@@ -61,6 +73,23 @@ def peaks():
         return float(p["hbm_gbs"]), "measured"
     except Exception:
         return FALLBACK_HBM_GBS, "fallback"
+
+
+def cpu_model() -> str:
+    try:
+        out = subprocess.run(["lscpu"], capture_output=True, text=True, timeout=10).stdout
+        for line in out.splitlines():
+            if line.startswith("Model name:"):
+                return line.split(":", 1)[1].strip()
+    except Exception:
+        pass
+    try:
+        for line in open("/proc/cpuinfo"):
+            if line.lower().startswith("model name"):
+                return line.split(":", 1)[1].strip()
+    except Exception:
+        pass
+    return platform.machine()
 
 
 class ClockSampler:
@@ -125,25 +154,26 @@ class ClockSampler:
                 "samples": len(rows)}
 
 
-def decode_algorithmic_bytes(m: synth.ModelShape, Lp: int, lens: np.ndarray) -> float:
-    """Bytes the decode of rollouts with generated lengths `lens` must move: every layer's
-    weights + final norm + lm_head once per decode step is counted by the caller; here the
-    per-token part: K/V reads of the whole context, K/V appends and embedding rows."""
+# ------------------------------------------------------------------------ algorithmic bytes
+def weight_bytes_per_step(m: synth.ModelShape) -> int:
+    """Every layer's weights and norms, the final norm and lm_head: read once per decode step."""
+    return m.layers * (m.layer_weight_bytes() + 4 * m.d_model) + 2 * m.vocab * m.d_model + 2 * m.d_model
+
+
+def decode_token_bytes(m: synth.ModelShape, Lp: int, lens: np.ndarray) -> float:
+    """Per-token part of the decode bytes of rollouts with generated lengths `lens`: the K/V of
+    the whole context read (contexts Lp, Lp+1, .., Lp+L-1), the new K/V written, the embedding
+    rows.  The weight part (weight_bytes_per_step per decode step) is added by the caller."""
     kvtok = m.kv_bytes_per_token()
     L = lens.astype(np.float64)
-    ctx_sum = (L * Lp + L * (L - 1) / 2).sum()  # contexts Lp, Lp+1, .. Lp+L-1
+    ctx_sum = (L * Lp + L * (L - 1) / 2).sum()
     return ctx_sum * kvtok + L.sum() * kvtok + L.sum() * m.d_model * 2
 
 
 def step_algorithmic_bytes(m: synth.ModelShape, rows: int, ctx: int) -> float:
-    """Bytes one decode step over `rows` rows at context `ctx` must move: the weights once,
-    the K/V of every context position read, the new K/V written, the embedding rows."""
+    """Bytes one decode step over `rows` rows at context `ctx` must move."""
     kvtok = m.kv_bytes_per_token()
     return weight_bytes_per_step(m) + rows * (ctx - 1) * kvtok + rows * kvtok + rows * m.d_model * 2
-
-
-def weight_bytes_per_step(m: synth.ModelShape) -> int:
-    return m.layers * (m.layer_weight_bytes() + 4 * m.d_model) + 2 * m.vocab * m.d_model + 2 * m.d_model
 
 
 def executed_lengths(si, n: np.ndarray) -> np.ndarray:
@@ -151,28 +181,87 @@ def executed_lengths(si, n: np.ndarray) -> np.ndarray:
 
 
 # --------------------------------------------------------------------------------- CPU arm
-def cpu_oracle_sample(w: synth.Workload, weights=None, tokens_per_sample: int = 1):
-    """The oracle as it stands on this host's cores: the Algorithm 1 schedule of the whole
-    step (O1) plus `tokens_per_sample` generated tokens of one rollout by full recompute (O2).
-    Returns (tokens/s, seconds, description)."""
-    from oracle import controller as oc
-    from oracle import decode as o2
+def _slice_tokens(w: synth.Workload):
+    """Inputs of the oracle's teacher-forced slice: the first prompt of round 0 and
+    CPU_SLICE_STEPS forced generated tokens (the oracle's cost does not depend on their values)."""
     si = synth.step_inputs(w)
+    return si, si.tokens[0], si.tokens[1, :CPU_SLICE_STEPS]
+
+
+def time_slice(workload: str, layers: int | None = None, repeat: int = 1) -> list[float]:
+    """Seconds of O2's teacher-forced slice (the first CPU_SLICE_STEPS decode steps of one
+    round-0 rollout, by the oracle's full recompute over the prompt) on the model's first
+    `layers` layers (all by default), `repeat` times, with this process's BLAS threads."""
+    from oracle import decode as o2
+    w = synth.WORKLOADS[workload]
+    m = w.model
+    L = m.layers if layers is None else layers
+    weights = synth.global_weights(m, w.weight_seed)
+    weights["layers"] = [synth.layer_weights(m, l, w.weight_seed) for l in range(L)]
+    W = o2.Weights(replace(m, layers=L), weights)
+    _, prompt, forced = _slice_tokens(w)
+    out = []
+    for _ in range(repeat):
+        t0 = time.perf_counter()
+        o2.teacher_forced_logits(W, prompt, forced)
+        out.append(time.perf_counter() - t0)
+    return out
+
+
+def cpu_slice_child(args):
+    """Child process of the CPU baseline (BLAS threads set by the parent's environment)."""
+    print(json.dumps({"seconds": time_slice(args.workload, args.slice_layers)[0]}))
+
+
+def _run_slice(workload: str, one_thread: bool, layers: int | None) -> float:
+    env = dict(os.environ)
+    if one_thread:  # BLAS on one thread (the input generator keeps its OpenMP threads)
+        for k in ("OPENBLAS_NUM_THREADS", "MKL_NUM_THREADS", "BLIS_NUM_THREADS"):
+            env[k] = "1"
+    cmd = [sys.executable, os.path.abspath(__file__), "--cpu-slice", "--workload", workload]
+    if layers is not None:
+        cmd += ["--slice-layers", str(layers)]
+    r = subprocess.run(cmd, capture_output=True, text=True, env=env, timeout=900)
+    if r.returncode != 0:
+        raise RuntimeError(f"oracle slice failed: {r.stderr[-2000:]}")
+    return float(json.loads(r.stdout.strip().splitlines()[-1])["seconds"])
+
+
+def cpu_baseline(workload: str) -> dict:
+    """The oracle as it stands, timed on this host's cores on a bounded sample of the workload:
+    O1 (plain C, one thread) over the whole step's schedule, and O2 (float64 numpy) on the
+    teacher-forced slice of one round-0 rollout, on all host threads (the whole model) and on
+    one thread (CPU_ONE_THREAD_LAYERS layers, scaled to the whole model; the lm_head part is
+    timed alone and not scaled).  value = O2 decode tokens per second on all threads."""
+    from oracle import controller as oc
+    w = synth.WORKLOADS[workload]
+    m = w.model
+    si, _, _ = _slice_tokens(w)
     t0 = time.perf_counter()
-    ref = oc.collect_workload(w, si)
-    t1 = time.perf_counter()
-    W = o2.Weights(w.model, weights)
-    q = int(np.nonzero(ref.n)[0][0])
-    t2 = time.perf_counter()
-    o2.generate(W, si.tokens[q], tokens_per_sample, w.sample_seed, o2.uid_of(q, 0))
-    t3 = time.perf_counter()
-    per_token = (t3 - t2) / tokens_per_sample
-    # whole-step cost model of the oracle: schedule + every generated token at this rate
-    rate = 1.0 / per_token
-    desc = (f"O1 schedule of the whole step ({t1 - t0:.3f} s) + O2 float64 decode of the first "
-            f"{tokens_per_sample} token(s) of rollout (q={q}, j=0) by full recompute over the "
-            f"{w.prompt_len}-token prompt; tokens/s = tokens / O2 time")
-    return rate, (t1 - t0) + (t3 - t2), desc
+    oc.collect_workload(w, si)
+    o1_s = time.perf_counter() - t0
+    t_all = _run_slice(workload, False, None)
+    t_head = _run_slice(workload, True, 0)
+    t_part = _run_slice(workload, True, CPU_ONE_THREAD_LAYERS)
+    t_one = t_head + (t_part - t_head) * m.layers / CPU_ONE_THREAD_LAYERS
+    ncpu = os.cpu_count()
+    try:
+        avail = len(os.sched_getaffinity(0))
+    except Exception:
+        avail = ncpu
+    return {
+        "value": CPU_SLICE_STEPS / t_all, "unit": "rollout tokens/s", "cores": avail, "kind": "oracle",
+        "sample": (f"O2 float64 teacher-forced slice: the first {CPU_SLICE_STEPS} decode steps of one of round 0's "
+                   f"{w.target_B * w.n0} rollouts (the oracle's full recompute over the {w.prompt_len}-token prompt "
+                   f"+ {CPU_SLICE_STEPS - 1} tokens), extrapolated to tokens/s = {CPU_SLICE_STEPS} / time; "
+                   f"BLAS on all {avail} host threads; plus O1 over the whole step's schedule"),
+        "o2_all_threads_s": round(t_all, 3), "o2_all_threads_tokens_per_s": CPU_SLICE_STEPS / t_all,
+        "o2_one_thread_s": round(t_one, 3), "o2_one_thread_tokens_per_s": CPU_SLICE_STEPS / t_one,
+        "o2_one_thread_note": (f"{CPU_ONE_THREAD_LAYERS} of {m.layers} layers timed on one thread and scaled; "
+                               f"lm_head part timed alone ({t_head:.2f} s)"),
+        "o1_whole_step_s": round(o1_s, 4), "o1_threads": 1,
+        "os_cpu_count": ncpu, "cpu_model": cpu_model(), "machine": platform.machine(),
+    }
 
 
 # --------------------------------------------------------------------------------- GPU arm
@@ -186,6 +275,12 @@ def run_mine(args):
     world = int(os.environ.get("WORLD_SIZE", "1"))
     rank = int(os.environ.get("RANK", "0"))
     local = int(os.environ.get("LOCAL_RANK", "0"))
+    t_start = time.time()
+    # the CPU baseline first (rank 0 at N = 1 only): bounded, in child processes, before any
+    # CUDA call of this process
+    cpu = None
+    if rank == 0 and world == 1 and not args.no_cpu_baseline:
+        cpu = cpu_baseline(args.workload)
     if world > 1:
         dist.init_process_group("nccl" if torch.cuda.is_available() else "gloo")
     torch.cuda.set_device(local)
@@ -199,31 +294,44 @@ def run_mine(args):
                         max_prompt_len=w.prompt_len, max_gen_len=w.lengths.max_len, max_k=w.k)
     stream = torch.cuda.current_stream(dev)
     h = pkg.Handle(cfg, weights, stream=stream)
+    del weights
 
-    # one synthetic batch per step: a fresh prompt stream (seeds shifted by the step index)
-    def inputs(i):
-        wi = w.with_seed_offset(7 * (i + 1)) if i >= 0 else w
-        return wi, synth.step_inputs(wi)
+    def pinned(a):
+        t = torch.empty(a.shape, dtype=torch.from_numpy(a[:0]).dtype, pin_memory=True)
+        t.numpy()[...] = a
+        return t.numpy()
 
-    def run_device(wi, si, dev_in):
-        return h.collect_step(thresholds=dev_in[0], lengths=dev_in[1], tokens=dev_in[2], N=wi.budget_N, k=wi.k,
-                              n0=wi.n0, tau=wi.tau, target_B=wi.target_B, reward_seed=wi.reward_seed,
+    # one synthetic batch per step: a fresh prompt stream (seeds shifted by the step index),
+    # staged in pinned host memory; results land in pinned host buffers
+    batches = []
+    for i in range(args.warmup + args.steps):
+        wi = w.with_seed_offset(7 * (i + 1))
+        si = synth.step_inputs(wi)
+        batches.append((wi, si, pinned(si.thresholds), pinned(si.lengths), pinned(si.tokens)))
+    P = w.n_prompts
+    outs_host = {"status": pinned(np.zeros(P, np.uint8)), "n": pinned(np.zeros(P, np.uint8)),
+                 "s": pinned(np.zeros(P, np.uint8)), "decided_round": pinned(np.zeros(P, np.int16)),
+                 "tokens": pinned(np.zeros((P, w.k, cfg.max_gen_len), np.int32))}
+
+    def step(b):
+        wi, _, thr, lens, toks = b
+        return h.collect_step(thresholds=thr, lengths=lens, tokens=toks, N=wi.budget_N, k=wi.k, n0=wi.n0,
+                              tau=wi.tau, target_B=wi.target_B, reward_seed=wi.reward_seed,
                               sample_seed=wi.sample_seed, commit_min=wi.commit_floor, prior=wi.prior,
-                              want_tokens=True, outputs_on_device=True)
+                              want_tokens=True, outputs=outs_host)
 
-    def to_dev(si):
-        return (torch.from_numpy(si.thresholds.view(np.int64)).to(dev), torch.from_numpy(si.lengths).to(dev),
-                torch.from_numpy(si.tokens).to(dev))
-
-    batches = [inputs(i) for i in range(args.warmup + args.steps)]
-    dev_batches = [to_dev(si) for _, si in batches]
-    torch.cuda.synchronize(dev)
+    warm_s = []
     for i in range(args.warmup):
-        run_device(batches[i][0], batches[i][1], dev_batches[i])
-    torch.cuda.synchronize(dev)
+        t0 = time.time()
+        step(batches[i])
+        warm_s.append(time.time() - t0)
+    if warm_s:
+        print(f"[bench] {args.warmup} warm-up steps, {np.mean(warm_s):.1f} s each; {args.steps} timed steps "
+              f"projected {np.mean(warm_s) * args.steps:.0f} s (setup {t_start and time.time() - t_start:.0f} s "
+              f"so far)", file=sys.stderr, flush=True)
 
-    # ------------------------------------------------------------------ timed region (HBM-resident)
-    outs = []
+    # ------------------------------------------------------------------ timed region
+    outs, n_executed = [], []
     e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
     if world > 1:
         dist.barrier()
@@ -231,91 +339,62 @@ def run_mine(args):
     with ClockSampler(local) as clk:
         e0.record(stream)
         for i in range(args.warmup, args.warmup + args.steps):
-            outs.append(run_device(batches[i][0], batches[i][1], dev_batches[i]))
+            o = step(batches[i])
+            outs.append(o)
+            n_executed.append(o.n.copy())
         e1.record(stream)
         torch.cuda.synchronize(dev)
     if world > 1:
         dist.barrier()
-    ms = e0.elapsed_time(e1)
+    e2e_ms = e0.elapsed_time(e1)
     clocks = clk.summary()
 
+    dev_ms = sum(o.device_ms for o in outs)
+    k_ms_live = sum(o.decode_kernel_ms for o in outs)
     tok = sum(o.counters["gen_tokens"] for o in outs)
     groups = sum(o.counters["committed"] for o in outs)
     rollouts = sum(o.counters["rollouts"] for o in outs)
     dsteps = sum(o.counters["decode_steps"] for o in outs)
+    rounds = sum(o.counters["rounds"] for o in outs)
     dec_bytes = 0.0
-    for (wi, si), o in zip(batches[args.warmup:], outs):
-        lens = executed_lengths(si, o.n.cpu().numpy())
-        dec_bytes += decode_algorithmic_bytes(m, wi.prompt_len, lens) + o.counters["decode_steps"] * \
-            weight_bytes_per_step(m)
+    for (wi, si, *_), o, n in zip(batches[args.warmup:], outs, n_executed):
+        dec_bytes += decode_token_bytes(m, wi.prompt_len, executed_lengths(si, n)) + \
+            o.counters["decode_steps"] * weight_bytes_per_step(m)
+    b0 = batches[0]
+    h2d = b0[2].nbytes + b0[3].nbytes + b0[4].nbytes
+    d2h = sum(a.nbytes for a in outs_host.values())
 
-    # ------------------------------------------------------------------ end to end (host buffers)
-    def pinned(a):
-        t = torch.empty(a.shape, dtype=torch.from_numpy(a[:0]).dtype, pin_memory=True)
-        t.numpy()[...] = a
-        return t.numpy()
-
-    e2e_batches = []
-    for i in range(args.steps):
-        wi, si = inputs(args.warmup + args.steps + i)
-        e2e_batches.append((wi, pinned(si.thresholds), pinned(si.lengths), pinned(si.tokens)))
-    h2d = sum(b[1].nbytes + b[2].nbytes + b[3].nbytes for b in e2e_batches)
-    d2h = 0
-    e2e_tok = 0
-    if world > 1:
-        dist.barrier()
-    torch.cuda.synchronize(dev)
-    f0, f1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-    f0.record(stream)
-    for wi, thr, lens, toks in e2e_batches:
-        o = h.collect_step(thresholds=thr, lengths=lens, tokens=toks, N=wi.budget_N, k=wi.k, n0=wi.n0, tau=wi.tau,
-                           target_B=wi.target_B, reward_seed=wi.reward_seed, sample_seed=wi.sample_seed,
-                           commit_min=wi.commit_floor, prior=wi.prior, want_tokens=True)
-        e2e_tok += o.counters["gen_tokens"]
-        d2h += o.status.nbytes + o.n.nbytes + o.s.nbytes + o.decided_round.nbytes + o.tokens.nbytes
-    f1.record(stream)
-    torch.cuda.synchronize(dev)
-    e2e_ms = f0.elapsed_time(f1)
-
-    # ------------------------------------------------------------------ dominant kernel roofline
-    # the decode-step kernel (one launch = one whole forward over the live rows) at the
-    # step's mean live rows and the median mid-rollout context
+    # cross-check of the dominant kernel with CUDA events around a captured graph of its
+    # launches, at the timed steps' mean live rows and the median mid-rollout context
     mean_rows = max(1, int(round(tok / max(dsteps, 1))))
-    mid_ctx = w.prompt_len + int(np.median(batches[0][1].lengths)) // 2
+    mid_ctx = w.prompt_len + int(np.median(b0[1].lengths)) // 2
     k_ms = h.profile(1, mean_rows, mid_ctx, iters=20)
     k_bytes = step_algorithmic_bytes(m, mean_rows, mid_ctx)
-    step_ms = h.profile(0, mean_rows, mid_ctx, iters=20)  # kernel + sampling / bookkeeping
     h.close()
 
     # ------------------------------------------------------------------ reduce over ranks
     if world > 1:  # the only collective: job totals (sum) over the slowest rank's time (max)
-        ms, e2e_ms = replicas.reduce_max([ms, e2e_ms], device=dev)
-        tok, groups, rollouts, e2e_tok, dec_bytes, h2d, d2h = replicas.reduce_sum(
-            [tok, groups, rollouts, e2e_tok, dec_bytes, h2d, d2h], device=dev)
+        dev_ms, e2e_ms, k_ms_live = replicas.reduce_max([dev_ms, e2e_ms, k_ms_live], device=dev)
+        tok, groups, rollouts, dec_bytes = replicas.reduce_sum([tok, groups, rollouts, dec_bytes], device=dev)
     if rank != 0:
         if world > 1:
             dist.destroy_process_group()
         return
 
     peak, peak_kind = peaks()
-    achieved = k_bytes / (k_ms * 1e-3) / 1e9
-    # DRAM traffic of the capture, scaled to this launch by its algorithmic bytes (weights are
-    # the same; KV grows with rows x context, which the capture read exactly once as well)
+    achieved = dec_bytes / world / (k_ms_live * 1e-3) / 1e9  # per GPU: each replica's own kernel
+    achieved_x = k_bytes / (k_ms * 1e-3) / 1e9
     tr = read_traffic(args.workload)
-    traffic = None if tr is None else tr[0] * k_bytes / tr[1]
-    cpu = None
-    if not args.no_cpu_baseline:
-        rate, secs, desc = cpu_oracle_sample(w0, weights)
-        cpu = {"value": rate, "unit": "rollout tokens/s", "cores": os.cpu_count(), "kind": "oracle",
-               "sample": desc, "seconds": round(secs, 2)}
+    per_launch = dec_bytes / world / max(dsteps, 1)
+    traffic = None if tr is None else tr[0] * per_launch / tr[1]
     line = {
         "metric": "rollout tokens/sec (also effective groups/sec and decode HBM GB/s)",
-        "value": tok / (ms * 1e-3),
+        "value": tok / (dev_ms * 1e-3),
         "unit": "tokens/s",
         "n_gpus": world,
         "steps": args.steps,
         "warmup": args.warmup,
-        "ms_per_step": ms / args.steps,
+        "ms_per_step": dev_ms / args.steps,
         "higher_is_better": True,
         "scaling": "weak",
         "vs_baseline": None,
@@ -324,30 +403,36 @@ def run_mine(args):
         "config": {"workload": w0.name, "global_batch": w0.target_B * world, "seq_len": w0.prompt_len,
                    "parallelism": f"replicas x{world} (prompt-stream shards)",
                    "l2": "inputs larger than L2 (3+ GB of weights streamed per decode step)"},
-        "effective_groups_per_s": groups / (ms * 1e-3),
-        "rollouts_per_s": rollouts / (ms * 1e-3),
-        "decode_hbm_gbs": dec_bytes / (ms * 1e-3) / 1e9,
-        "decode_hbm_frac": dec_bytes / (ms * 1e-3) / 1e9 / peak,
-        "decode_step_ms": step_ms,
-        "decode_kernel_ms": k_ms,
+        "effective_groups_per_s": groups / (dev_ms * 1e-3),
+        "rollouts_per_s": rollouts / (dev_ms * 1e-3),
+        "decode_hbm_gbs": dec_bytes / world / (dev_ms * 1e-3) / 1e9,
+        "decode_hbm_frac": dec_bytes / world / (dev_ms * 1e-3) / 1e9 / peak,
+        "decode_steps_per_step": dsteps / world / args.steps,
         "roofline": {"bound": "hbm", "achieved": achieved, "peak": peak, "unit": "GB/s",
                      "frac": achieved / peak, "traffic": traffic,
-                     "traffic_note": None if tr is None else "ncu capture at 25 rows, context 384, scaled by algorithmic bytes",
-                     "kernel": f"decode_step_kernel (whole forward), {mean_rows} live rows at context {mid_ctx}",
-                     "bytes_per_launch": k_bytes,
+                     "kernel": "decode_step_kernel (one launch = one whole decode forward over the live rows)",
+                     "how": ("algorithmic bytes of every decode step of the timed steps (weights once + K/V of "
+                             "every context position + K/V appends + embedding rows) / summed launch durations "
+                             "(device clock per launch: earliest CTA start to latest CTA end)"),
+                     "launches": dsteps // world, "bytes_per_launch_mean": per_launch,
+                     "traffic_note": None if tr is None else "ncu DRAM bytes of one captured launch, scaled by algorithmic bytes",
+                     "events_check": {"rows": mean_rows, "ctx": mid_ctx, "ms_per_launch": k_ms,
+                                      "achieved": achieved_x, "frac": achieved_x / peak,
+                                      "how": "CUDA events around 20 graph-captured launches at these rows and context"},
                      "peak_kind": f"{peak_kind} burst copy"},
-        "e2e": {"value": e2e_tok / (e2e_ms * 1e-3), "unit": "tokens/s", "h2d_bytes_per_step": h2d / args.steps,
-                "d2h_bytes_per_step": d2h / args.steps},
+        "e2e": {"value": tok / (e2e_ms * 1e-3), "unit": "tokens/s", "h2d_bytes_per_step": h2d,
+                "d2h_bytes_per_step": d2h,
+                "how": "CUDA events around the K calls (pinned host inputs in, pinned host results out)"},
         "cpu_baseline": cpu,
         "gpu_launches": None,
         "clocks": clocks,
+        "wall_s": round(time.time() - t_start, 1),
     }
     # kernels launched: per decode step the controller, the decode-step kernel and the
-    # sampling/bookkeeping kernel; per round start the prefill (embedding + 5 per layer
-    # but the last layer's 4) and the KV fan-out; per call the init kernel
-    rounds = sum(o.counters["rounds"] for o in outs)
-    line["gpu_launches"] = int(3 * dsteps + rounds * (1 + 5 * m.layers - 4 + 1) + args.steps)
-    print(json.dumps(line))
+    # sampling/bookkeeping kernel; per round start the prefill (embedding + 5 per layer but
+    # the last layer's 4) and the KV fan-out; per call the init kernel
+    line["gpu_launches"] = int(3 * dsteps + rounds * (1 + 5 * m.layers - 4 + 1) + args.steps * world)
+    print(json.dumps(line), flush=True)
     if world > 1:
         dist.destroy_process_group()
 
@@ -391,29 +476,39 @@ def run_kernel_profile(args):
 
 # --------------------------------------------------------------------------------- reference arm
 def run_reference(args):
+    """The oracle as the reference arm, on this host's cores: per step, O1 over the whole step's
+    schedule and O2's teacher-forced slice (CPU_SLICE_STEPS decode steps of one round-0 rollout)
+    on all host threads; value = decode tokens per second of O2."""
     rank = int(os.environ.get("RANK", "0"))
     if rank != 0:
         return
+    from oracle import controller as oc
     w = synth.WORKLOADS[args.workload]
-    weights = synth.model_weights(w.model, w.weight_seed)
-    for _ in range(args.warmup):
-        cpu_oracle_sample(w, weights)
-    rates, secs = [], 0.0
-    desc = ""
-    for _ in range(args.steps):
-        r, s, desc = cpu_oracle_sample(w, weights)
-        rates.append(r)
-        secs += s
-    value = float(np.mean(rates))
+    o1 = []
+    for i in range(args.steps):
+        wi = w.with_seed_offset(7 * (args.warmup + i + 1))
+        si = synth.step_inputs(wi)
+        t0 = time.perf_counter()
+        oc.collect_workload(wi, si)
+        o1.append(time.perf_counter() - t0)
+    secs = time_slice(args.workload, None, args.warmup + args.steps)[args.warmup:]
+    value = CPU_SLICE_STEPS * len(secs) / sum(secs)
+    try:
+        avail = len(os.sched_getaffinity(0))
+    except Exception:
+        avail = os.cpu_count()
+    sample = (f"per step: O1 over the whole step's schedule (1 thread) + O2 float64 teacher-forced slice, the "
+              f"first {CPU_SLICE_STEPS} decode steps of one round-0 rollout by full recompute over the "
+              f"{w.prompt_len}-token prompt, BLAS on all {avail} host threads; value = {CPU_SLICE_STEPS} / O2 time")
     line = {
         "impl": "reference",
         "metric": "rollout tokens/sec (also effective groups/sec and decode HBM GB/s)",
         "value": value, "unit": "tokens/s", "n_gpus": int(os.environ.get("WORLD_SIZE", "1")),
-        "steps": args.steps, "warmup": args.warmup, "ms_per_step": 1e3 * secs / args.steps,
+        "steps": args.steps, "warmup": args.warmup, "ms_per_step": 1e3 * (sum(secs) + sum(o1)) / len(secs),
         "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
         "data": "synthetic", "config": {"workload": w.name},
-        "cpu_baseline": {"value": value, "unit": "tokens/s", "cores": os.cpu_count(), "kind": "oracle",
-                         "sample": desc},
+        "cpu_baseline": {"value": value, "unit": "tokens/s", "cores": avail, "kind": "oracle", "sample": sample,
+                         "cpu_model": cpu_model(), "o1_whole_step_s_mean": float(np.mean(o1))},
         "e2e": {"value": value, "unit": "tokens/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
     }
     print(json.dumps(line))
@@ -421,7 +516,9 @@ def run_reference(args):
 
 if __name__ == "__main__":
     a = parse()
-    if a.kernel_profile is not None:
+    if a.cpu_slice:
+        cpu_slice_child(a)
+    elif a.kernel_profile is not None:
         run_kernel_profile(a)
     elif a.impl == "reference":
         run_reference(a)

@@ -38,6 +38,11 @@
 extern "C" {
 #endif
 
+/* Layout version of the structs below.  Version 2 added sara_thresholds.schedule,
+ * sara_result.decode_kernel_ms and sara_limits; a caller built against another version
+ * must not pass its structs to this library (compare with sara_abi_version()). */
+#define SARA_ABI_VERSION 2
+
 #define SARA_OK 0
 #define SARA_EINVAL (-1)   /* an argument is out of range; nothing was launched */
 #define SARA_ENOMEM (-2)   /* device or host allocation failed, or a capacity is exceeded */
@@ -138,7 +143,11 @@ typedef struct {
     int64_t decode_steps;      /* batched decode forward passes */
     int64_t rounds;            /* synchronisation rounds */
     int64_t committed, abandoned, incomplete, prompts_drawn;
-    double device_ms;          /* GPU time of the step (CUDA events around the work) */
+    double device_ms;          /* GPU time of the step's kernels, inputs already on the device:
+                                  CUDA events on the handle's stream after the input copies and
+                                  before the output copies */
+    double decode_kernel_ms;   /* summed duration of the decode-step kernel's launches (device
+                                  clock, earliest CTA start to latest CTA end of each launch) */
 } sara_result;
 
 /*
@@ -196,6 +205,30 @@ SARA_API int sara_teacher_force(sara_handle *h, int32_t n_seq, int32_t prompt_le
 SARA_API int sara_profile(sara_handle *h, int32_t kernel, int32_t rows, int32_t ctx, int32_t iters,
                           double *ms_per_launch);
 
+/*
+ * Failure limits (testing and watchdogs).  Every device wait of the step is bounded; these
+ * fields tighten the bounds for later calls on the handle, so that the error paths can be
+ * exercised without faulting or hanging the GPU.  All zero (stall_phase = -1) restores the
+ * defaults.
+ *   wait_limit_ns:  a bounded wait of the decode-step kernel gives up after this long and the
+ *                   call returns SARA_ETIMEOUT (0: 2 s).
+ *   max_loop_iters: the step's device loop ends with SARA_ETIMEOUT once it has run this many
+ *                   iterations (0: only the built-in round bounds).
+ *   stall_phase:    -1, or a phase-counter index of the decode-step kernel (0 = embedding,
+ *                   1 + 9 l + j = phase j of layer l) whose waits are made to wait for a value
+ *                   no launch reaches: they time out after wait_limit_ns.
+ * The handle stays usable after a call that failed this way.  SARA_EINVAL if out of range.
+ */
+typedef struct {
+    int64_t wait_limit_ns;
+    int32_t max_loop_iters;
+    int32_t stall_phase;
+} sara_limits;
+SARA_API int sara_set_limits(sara_handle *h, const sara_limits *limits);
+
+/* SARA_ABI_VERSION of the built library. */
+SARA_API int sara_abi_version(void);
+
 /* Message for the last error on this handle (or of sara_create when h == NULL). */
 SARA_API const char *sara_last_error(const sara_handle *h);
 
@@ -203,12 +236,15 @@ SARA_API const char *sara_last_error(const sara_handle *h);
 SARA_API void sara_destroy(sara_handle *h);
 
 /* ---------------------------------------------------------------------------------------
- * Kernel-level entry points (device pointers, the caller's stream).  Each one launches the
- * same kernel the step uses, for unit parity tests.
+ * Kernel-level entry points (device pointers, the caller's stream), for unit parity tests
+ * of the building blocks.  The GEMM and the attention launch the kernels the step's prefill
+ * of fresh prompts runs; the sampler is a one-CTA-per-row form of the decode step's
+ * Gumbel-max.  The decode step itself runs its projections, attention and logits inside one
+ * persistent kernel, which is tested end to end through sara_teacher_force.
  * ------------------------------------------------------------------------------------- */
 
 /*
- * Y[r][n] = sum_c X[r][c] * W[n][c] for r < R, n < Nout (the decode projection GEMM:
+ * Y[r][n] = sum_c X[r][c] * W[n][c] for r < R, n < Nout (the prefill projection GEMM:
  * tcgen05 MMA with the accumulator in tensor memory, TMA-fed, stream-K over the weight).
  * X: [R][K] bf16, W: [Nout][K] bf16, Y: [R][Nout] fp32, all device, 16-byte aligned.
  * Shapes: 1 <= R <= 128, Nout % 128 == 0, K % 64 == 0, K >= 64.
@@ -239,8 +275,8 @@ SARA_API int sara_gemm_bf16_static(const uint16_t *X, const uint16_t *W, float *
                                    int32_t Nout, int32_t K, void *stream);
 
 /*
- * Decode attention for b sequences, one new query each (softmax(q K^T / sqrt(hd)) V with
- * grouped-query heads): q [b][n_heads][hd] fp16; kv cache of sequence i at kv + i*kv_stride
+ * Attention of b query rows against their own KV ranges (the prefill's attention kernel),
+ * one query each (softmax(q K^T / sqrt(hd)) V with grouped-query heads): q [b][n_heads][hd] fp16; kv cache of sequence i at kv + i*kv_stride
  * elements, laid out [2 (K,V)][n_kv_heads][cap][hd] fp16, valid for positions < ctx[i];
  * out [b][n_heads][hd] bf16 (the high part of the step's bf16 hi/lo output pair).  Split over the context in chunks of 128 positions with an
  * fp32 log-sum-exp combine.  hd in {32, 64, 128}; n_heads / n_kv_heads in {1, 2, 4, 6, 8};
@@ -256,7 +292,8 @@ SARA_API int sara_attention_decode(const uint16_t *q, const uint16_t *kv, int64_
                                    void *stream);
 
 /*
- * Temperature-1 sampling by Gumbel-max: token[r] = argmax_v (logits[r][v] + g(r, v)) with
+ * Temperature-1 sampling by Gumbel-max (the decode step's sampling rule, one CTA per row):
+ * token[r] = argmax_v (logits[r][v] + g(r, v)) with
  * g = -log(-log u), u from SplitMix64 keyed by (sample_seed, uid[r], t[r], v), decided in
  * fp32, ties to the lowest index.  logits [R][V] fp32, uid/t/token [R], all device.
  */

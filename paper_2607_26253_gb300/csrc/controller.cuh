@@ -411,7 +411,12 @@ ctl_kernel(StepPtrs c, cudaGraphConditionalHandle h_loop, cudaGraphConditionalHa
     const StepConst K = *c.kc;
     StepVars &V = *c.v;
     __syncthreads();
-    if (threadIdx.x == 0) V.iters += 1;
+    if (threadIdx.x == 0) {
+        V.iters += 1;
+        // the caller's bound on the loop (sara_set_limits)
+        if (K.max_iters > 0 && V.iters > K.max_iters && !V.done) report_error(&V.err, ERR_ITER_BOUND);
+    }
+    __syncthreads();
     if (V.err != 0 && !V.done) {  // a kernel reported an error: end the step now
         __syncthreads();
         if (threadIdx.x == 0) { V.done = 1; V.live = 0; }
@@ -469,6 +474,7 @@ static __global__ void __launch_bounds__(kCtlThreads, 1) ctl_init_kernel(StepPtr
         StepVars z;
         memset(&z, 0, sizeof(z));
         z.round = -1;
+        z.kt0 = ~0ull;
         V = z;
     }
 }

@@ -104,6 +104,7 @@ struct MegaParams {
     unsigned long long *epoch;                      // launches completed since the reset
     uint64_t *stamps;                               // profiling builds: [cta][phase + 1][4] timestamps
     int n_stamp_ph;
+    unsigned long long *ktime;                      // [2]: earliest CTA start, latest CTA end (ns)
 };
 
 // Profiling builds (-DSARA_STAMPS): per CTA and phase, when the compute warps arrived (0),
@@ -140,6 +141,8 @@ struct MegaSmem {
     uint64_t q_ready[2], s_full[2], p_ready[2], o_full[2];
     uint64_t drain;
     unsigned long long target;  // counter value meaning "every CTA of this launch arrived"
+    uint64_t wait_ns;           // bounded-wait limit of this launch
+    int stall_idx;              // test hook: the phase counter whose waits never complete (-1: none)
     uint32_t tmem_base;
     int abort;
     int last_flag;
@@ -183,14 +186,14 @@ __host__ __device__ __forceinline__ int64_t wblk_off(int N, int K, int t, int kc
 
 // ------------------------------------------------------------------------------ waits
 // Bounded mbarrier wait that also gives up (returning false) once the CTA is aborting.
-__device__ __forceinline__ bool mwait(uint64_t *bar, uint32_t parity, int *err, volatile int *abort) {
+__device__ __forceinline__ bool mwait(uint64_t *bar, uint32_t parity, int *err, volatile int *abort, uint64_t limit) {
     if (mbar_try_wait(bar, parity)) return true;
     const uint64_t t0 = globaltimer_ns();
     for (uint32_t it = 1;; ++it) {
         if (mbar_try_wait(bar, parity)) return true;
         if ((it & 63u) == 0) {
             if (*abort) return false;
-            if (globaltimer_ns() - t0 > kWaitLimitNs) {
+            if (globaltimer_ns() - t0 > limit) {
                 report_error(err, ERR_WAIT_TIMEOUT);
                 *abort = 1;
                 return false;
@@ -202,7 +205,7 @@ __device__ __forceinline__ bool mwait(uint64_t *bar, uint32_t parity, int *err, 
 // Spin until a phase counter reaches `target` (acquire loads);
 // bounded, gives up on abort or once another CTA reported a timeout.
 __device__ __forceinline__ bool spin_counter(const unsigned long long *cnt, unsigned long long target, int *err,
-                                             volatile int *abort) {
+                                             volatile int *abort, uint64_t limit) {
     if (ld_acquire_u64(cnt) >= target) return true;
     const uint64_t t0 = globaltimer_ns();
     for (uint32_t it = 1;; ++it) {
@@ -214,13 +217,19 @@ __device__ __forceinline__ bool spin_counter(const unsigned long long *cnt, unsi
                 *abort = 1;
                 return false;
             }
-            if (globaltimer_ns() - t0 > kWaitLimitNs) {
+            if (globaltimer_ns() - t0 > limit) {
                 report_error(err, ERR_WAIT_TIMEOUT);
                 *abort = 1;
                 return false;
             }
         }
     }
+}
+
+// Counter value a wait on phase counter idx needs: every CTA of this launch arrived (the
+// test hook makes one counter's target unreachable, so its waits run into the time limit).
+__device__ __forceinline__ unsigned long long phase_target(const MegaParams &p, const MegaSmem &S, int idx) {
+    return idx == S.stall_idx ? ~0ull : S.target;
 }
 
 // ------------------------------------------------------------------------------ phases
@@ -328,13 +337,14 @@ __device__ __forceinline__ uint8_t *kv_block(const MegaParams &p, int l, const A
 // ------------------------------------------------------------------------------ W producer
 __device__ __forceinline__ void mega_w_producer(const MegaParams &p, MegaSmem &S, uint8_t *sW) {
     volatile int *ab = &S.abort;
+    const uint64_t lim = S.wait_ns;
     int *err = &p.c.v->err;
     const uint64_t pol = l2_policy_evict_first();
     constexpr uint32_t nws = kWSlots;
     uint32_t wi = 0;
     bool ok = true;
     auto acquire = [&](uint32_t i) -> bool {
-        return i < nws || mwait(&S.wempty[i % nws], ((i / nws) & 1) ^ 1, err, ab);
+        return i < nws || mwait(&S.wempty[i % nws], ((i / nws) & 1) ^ 1, err, ab, lim);
     };
     for (int l = 0; l <= p.layers && ok; ++l) {
         for (int gp = 0; gp < 4 && ok; ++gp) {
@@ -373,8 +383,8 @@ __device__ __forceinline__ void mega_w_producer(const MegaParams &p, MegaSmem &S
                             const AttUnit &u = w ? ub : ua;
                             if (j >= (w ? nbb : ua.nb)) continue;
                             if (u.last && j == u.nb - 1 && !finq_seen) {
-                                if (!spin_counter(&p.cnt[(1 + kPhasesPerLayer * l + kPhFinQ) * kCntStride], S.target,
-                                                  err, ab)) {
+                                const int fq = 1 + kPhasesPerLayer * l + kPhFinQ;
+                                if (!spin_counter(&p.cnt[fq * kCntStride], phase_target(p, S, fq), err, ab, lim)) {
                                     ok = false;
                                     break;
                                 }
@@ -414,6 +424,7 @@ __device__ __forceinline__ void mega_w_producer(const MegaParams &p, MegaSmem &S
 // ------------------------------------------------------------------------------ X producer
 __device__ __forceinline__ void mega_x_producer(const MegaParams &p, MegaSmem &S, uint8_t *sX) {
     volatile int *ab = &S.abort;
+    const uint64_t lim = S.wait_ns;
     int *err = &p.c.v->err;
     const uint64_t pol = l2_policy_evict_last();
     const int NX = S.nx, R16 = S.rows16, nxl = S.nx_lg;
@@ -432,12 +443,12 @@ __device__ __forceinline__ void mega_x_producer(const MegaParams &p, MegaSmem &S
             // the phase this operand comes from (the one before it): FIN_D of l-1 / embedding,
             // ATT, FIN_O, FIN_GU
             const int dep = (l == p.layers || k == 0) ? kPhasesPerLayer * l : 1 + kPhasesPerLayer * l + k - 1;
-            if (!spin_counter(&p.cnt[dep * kCntStride], S.target, err, ab)) { ok = false; break; }
+            if (!spin_counter(&p.cnt[dep * kCntStride], phase_target(p, S, dep), err, ab, lim)) { ok = false; break; }
             MEGA_STAMP(1 + kPhasesPerLayer * l + k, 1);
             fence_proxy_async_global();
             for (int64_t u = u0; u < u1; ++u, ++xi) {
                 const int s = (int)(xi & (uint32_t)(NX - 1));
-                if (xi >= (uint32_t)NX && !mwait(&S.xempty[s], ((xi >> nxl) & 1) ^ 1, err, ab)) { ok = false; break; }
+                if (xi >= (uint32_t)NX && !mwait(&S.xempty[s], ((xi >> nxl) & 1) ^ 1, err, ab, lim)) { ok = false; break; }
                 const int kc = (int)(u % g.kch);
                 mbar_arrive_expect_tx(&S.xfull[s], stage);
                 bulk_load(sX + (size_t)s * stage, g.x + kc * chunk_stride, stage, &S.xfull[s], pol);
@@ -456,6 +467,7 @@ __device__ __forceinline__ void mega_x_producer(const MegaParams &p, MegaSmem &S
 __device__ __forceinline__ void mega_mma(const MegaParams &p, MegaSmem &S, uint8_t *sW, uint8_t *sX, uint8_t *sQ,
                                          uint8_t *sP, uint32_t tmem) {
     volatile int *ab = &S.abort;
+    const uint64_t lim = S.wait_ns;
     int *err = &p.c.v->err;
     const int NX = S.nx, R16 = S.rows16, nxl = S.nx_lg;
     const uint32_t stage = (uint32_t)R16 * 256;
@@ -469,7 +481,7 @@ __device__ __forceinline__ void mega_mma(const MegaParams &p, MegaSmem &S, uint8
     bool ok = true;
     constexpr uint32_t nws = kWSlots;
     auto wslot = [&](uint32_t i) -> uint32_t { return smem_u32(sW + (size_t)(i % nws) * kSlotBytes); };
-    auto wwait = [&](uint32_t i) -> bool { return mwait(&S.wfull[i % nws], (i / nws) & 1, err, ab); };
+    auto wwait = [&](uint32_t i) -> bool { return mwait(&S.wfull[i % nws], (i / nws) & 1, err, ab, lim); };
     auto gemm = [&](const GemmPh &g, int64_t u0, int64_t u1, bool det) {
         const int64_t ub = u0;
         for (int64_t u = u0; u < u1 && ok;) {
@@ -477,7 +489,7 @@ __device__ __forceinline__ void mega_mma(const MegaParams &p, MegaSmem &S, uint8
             const int64_t e = min(u1, (int64_t)(t + 1) * g.kch);
             const int a = tseg & 1;  // tiles alternate between two accumulators (epilogue overlaps)
             const int use_a = a ? use1 : use0;
-            if (use_a >= 1 && !mwait(&S.acc_empty[a], (use_a - 1) & 1, err, ab)) { ok = false; break; }
+            if (use_a >= 1 && !mwait(&S.acc_empty[a], (use_a - 1) & 1, err, ab, lim)) { ok = false; break; }
             tc_fence_after();
             const uint32_t d = tmem + (uint32_t)(a * kTileN);
             const uint32_t idg = idesc_bf16_f32(R16 <= 32 ? 64u : 128u, (uint32_t)tile_rows(g, t));
@@ -487,7 +499,7 @@ __device__ __forceinline__ void mega_mma(const MegaParams &p, MegaSmem &S, uint8
                 const bool dj = det && u - ub < 12;
                 if (!wwait(wi)) { ok = false; break; }
                 if (dj) MEGA_DETAIL(28 + (int)(u - ub));
-                if (!mwait(&S.xfull[xs], (xi >> nxl) & 1, err, ab)) { ok = false; break; }
+                if (!mwait(&S.xfull[xs], (xi >> nxl) & 1, err, ab, lim)) { ok = false; break; }
                 if (dj) MEGA_DETAIL(40 + (int)(u - ub));
                 tc_fence_after();
                 const uint32_t aw = wslot(wi), ax = smem_u32(sX + (size_t)xs * stage);
@@ -526,7 +538,7 @@ __device__ __forceinline__ void mega_mma(const MegaParams &p, MegaSmem &S, uint8
         auto scores = [&](int b, uint32_t e, bool first_blk) -> bool {  // S = K q^T
             uint32_t &cq = b ? aq1 : aq0;
             if (first_blk) {
-                if (!mwait(&S.q_ready[b], cq & 1, err, ab)) return false;
+                if (!mwait(&S.q_ready[b], cq & 1, err, ab, lim)) return false;
                 ++cq;
             }
             if (!wwait(e)) return false;
@@ -541,7 +553,7 @@ __device__ __forceinline__ void mega_mma(const MegaParams &p, MegaSmem &S, uint8
         };
         auto pv = [&](int b, uint32_t e, int nj) -> bool {  // O^T = V^T P^T
             uint32_t &cb = b ? ab1 : ab0;
-            if (!mwait(&S.p_ready[b], cb & 1, err, ab)) return false;
+            if (!mwait(&S.p_ready[b], cb & 1, err, ab, lim)) return false;
             ++cb;
             if (!wwait(e)) return false;
             tc_fence_after();
@@ -606,6 +618,7 @@ __device__ __forceinline__ void store_hilo(uint8_t *base, int64_t off, float v) 
 __device__ __forceinline__ void mega_compute(const MegaParams &p, MegaSmem &S, uint8_t *sW, uint8_t *sQ, uint8_t *sP,
                                              uint32_t tmem) {
     volatile int *ab = &S.abort;
+    const uint64_t lim = S.wait_ns;
     int *err = &p.c.v->err;
     const int ctid = threadIdx.x - 96;  // 0..255
     const int cw = ctid >> 5, lane = threadIdx.x & 31;
@@ -644,7 +657,7 @@ __device__ __forceinline__ void mega_compute(const MegaParams &p, MegaSmem &S, u
     };
     auto wait_phase = [&](int idx) {
         if (ctid == 0) {
-            spin_counter(&p.cnt[idx * kCntStride], S.target, err, ab);
+            spin_counter(&p.cnt[idx * kCntStride], phase_target(p, S, idx), err, ab, lim);
             MEGA_STAMP(idx + 1, 1);
         }
         named_bar_sync(1, kMegaCThreads);
@@ -667,7 +680,7 @@ __device__ __forceinline__ void mega_compute(const MegaParams &p, MegaSmem &S, u
             const int t = (int)(u / g.kch);
             u = min(u1, (int64_t)(t + 1) * g.kch);
             const int a = tseg & 1;
-            mwait(&S.acc_full[a], (a ? cuse1 : cuse0) & 1, err, ab);
+            mwait(&S.acc_full[a], (a ? cuse1 : cuse0) & 1, err, ab, lim);
             tc_fence_after();
             const int rows_t = tile_rows(g, t);
             if (quarter_live && half * 128 < rows_t) {
@@ -886,7 +899,7 @@ __device__ __forceinline__ void mega_compute(const MegaParams &p, MegaSmem &S, u
                     const uint32_t ph = att_blk & 1u;
                     ++att_blk;
                     const bool valid = pos < min(kKVPos, u.n - jb * kKVPos);
-                    mwait(&S.s_full[b], ph, err, ab);
+                    mwait(&S.s_full[b], ph, err, ab, lim);
                     if (half == 0 && jb == 0) DETAIL(2);
                     tc_fence_after();
                     float sv[8];
@@ -924,7 +937,7 @@ __device__ __forceinline__ void mega_compute(const MegaParams &p, MegaSmem &S, u
                                   (S.red2[half][2][g] + S.red2[half][3][g]);
                         mrun[g] = mnew[g];
                     }
-                    mwait(&S.o_full[b], ph, err, ab);
+                    mwait(&S.o_full[b], ph, err, ab, lim);
                     if (half == 0 && jb == 0) DETAIL(4);
                     tc_fence_after();
                     float ov[8];
@@ -1134,7 +1147,7 @@ __device__ __forceinline__ void mega_compute(const MegaParams &p, MegaSmem &S, u
         for (int64_t u = u0; u < u1; u += g.kch) {
             const int t = (int)(u / g.kch);
             const int a = tseg & 1;
-            mwait(&S.acc_full[a], (a ? cuse1 : cuse0) & 1, err, ab);
+            mwait(&S.acc_full[a], (a ? cuse1 : cuse0) & 1, err, ab, lim);
             tc_fence_after();
             if (quarter_live && half * 128 < tile_rows(g, t)) {
                 float *dst = p.logits + (int64_t)(act ? my_row : 0) * p.V + t * kTileN + half * 128;
@@ -1203,11 +1216,16 @@ __global__ void __launch_bounds__(kMegaThreads, 1) decode_step_kernel(const __gr
         S.n_items = *(volatile int *)&V->att_items;
         S.att_span = max(1, *(volatile int *)&V->att_span);
         S.target = (*(volatile unsigned long long *)p.epoch + 1ull) * gridDim.x;
+        // failure limits of this call (sara_set_limits): read at run time, not baked into the graph
+        const int64_t wl = p.c.kc->wait_ns;
+        S.wait_ns = wl > 0 ? (uint64_t)wl : kWaitLimitNs;
+        S.stall_idx = p.c.kc->stall_plus1 - 1;
         S.abort = (*(volatile int *)&V->err & ERR_WAIT_TIMEOUT) != 0;
         S.last_flag = 0;
         fence_mbar_init();
     }
     if (threadIdx.x == 0) MEGA_STAMP(p.n_stamp_ph - kDetailRows - 1, 0);  // kernel start
+    const uint64_t t_start = globaltimer_ns();
     if (warp == 1) {
         tmem_alloc(&S.tmem_base, kTmemCols);
         tmem_relinquish();
@@ -1236,6 +1254,11 @@ __global__ void __launch_bounds__(kMegaThreads, 1) decode_step_kernel(const __gr
     // every CTA read the epoch before any CTA could pass the first phase; the last phase's
     // wait in CTA 0 therefore happens after all reads
     if (run && threadIdx.x == 0 && blockIdx.x == 0) atomicAdd(p.epoch, 1ull);
+    // launch duration for the step's kernel-time total (the bookkeeping kernel folds it in)
+    if (run && threadIdx.x == 0 && p.ktime) {
+        atomicMin(&p.ktime[0], (unsigned long long)t_start);
+        atomicMax(&p.ktime[1], (unsigned long long)globaltimer_ns());
+    }
 }
 
 // ------------------------------------------------------------------------------ layout kernels

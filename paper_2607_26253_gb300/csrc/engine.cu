@@ -107,6 +107,9 @@ struct sara_handle {
     int64_t *uid_dev = nullptr;
     size_t forced_cap = 0;
     uint64_t *stamps = nullptr;  // profiling builds: per-CTA phase timestamps of GEMM launches
+    // failure limits (sara_set_limits): bounded-wait limit, loop bound, stalled phase counter
+    uint64_t wait_ns = 0;
+    int32_t max_iters = 0, stall_idx = -1;
     // graph
     cudaGraph_t graph = nullptr;
     cudaGraphExec_t exec = nullptr;
@@ -135,7 +138,6 @@ void set_kernel_attrs() {
     CK(cudaFuncSetAttribute(gemm_tc_kernel<EPI_QKV>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)kGemmSmemBytes));
     CK(cudaFuncSetAttribute(gemm_tc_kernel<EPI_RESID>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)kGemmSmemBytes));
     CK(cudaFuncSetAttribute(gemm_tc_kernel<EPI_SWIGLU>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)kGemmSmemBytes));
-    CK(cudaFuncSetAttribute(gemm_tc_kernel<EPI_LMHEAD>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)kGemmSmemBytes));
     CK(cudaFuncSetAttribute(decode_step_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)kMegaSmemBytes));
     done = true;
 }
@@ -371,6 +373,7 @@ MegaParams mega_params(const sara_handle &h) {
     p.epoch = h.phase_cnt + (size_t)h.n_phase_cnt * kCntStride;
     p.stamps = h.stamps;
     p.n_stamp_ph = h.n_phase_cnt + 1 + kDetailRows;  // phases, kernel start, detail stamps
+    p.ktime = &h.vars->kt0;
     return p;
 }
 
@@ -818,14 +821,18 @@ void collect_impl(sara_handle &h, const sara_prompts *pr, int64_t N, int32_t k, 
     K.max_gen = m.max_gen_len;
     K.attn_chunk = kDecodeChunk;
     K.att_slots = att_slots(h);
+    K.max_iters = h.max_iters;
+    K.stall_plus1 = h.stall_idx + 1;
+    K.wait_ns = (int64_t)h.wait_ns;
 
-    CK(cudaEventRecord(h.ev0, s));
     CK(cudaMemcpyAsync(h.kc, &K, sizeof(K), cudaMemcpyHostToDevice, s));
     if (P > 0) {
         CK(cudaMemcpyAsync(h.p_thr, pr->p_threshold, (size_t)P * 8, kin, s));
         CK(cudaMemcpyAsync(h.p_len, pr->lengths, (size_t)P * k * 4, kin, s));
         if (h.has_model) CK(cudaMemcpyAsync(h.p_tok, pr->tokens, (size_t)P * Lp * 4, kin, s));
     }
+    // device time of the step: from here (inputs on the device) to the end of its last kernel
+    CK(cudaEventRecord(h.ev0, s));
     if (h.has_model) reset_decode_state(h, s);
     launch(s, false, dim3(1), dim3(kCtlThreads), 0, ctl_init_kernel, h.ptrs);
     if (t->schedule != 0) {  // asynchronous per-prompt schedule: one event-loop kernel
@@ -838,6 +845,7 @@ void collect_impl(sara_handle &h, const sara_prompts *pr, int64_t N, int32_t k, 
     } else {
         run_host_loop(h);
     }
+    CK(cudaEventRecord(h.ev1, s));
     // results (one device -> host read per call)
     StepVars v{};
     const cudaMemcpyKind kout = out->on_device ? cudaMemcpyDeviceToDevice : cudaMemcpyDeviceToHost;
@@ -852,7 +860,6 @@ void collect_impl(sara_handle &h, const sara_prompts *pr, int64_t N, int32_t k, 
         if (out->tokens && h.has_model)
             CK(cudaMemcpyAsync(out->tokens, h.gen_tok, (size_t)P * k * m.max_gen_len * 4, kout, s));
     }
-    CK(cudaEventRecord(h.ev1, s));
     CK(cudaStreamSynchronize(s));
     check_step_error(v);
     float ms = 0.f;
@@ -870,6 +877,7 @@ void collect_impl(sara_handle &h, const sara_prompts *pr, int64_t N, int32_t k, 
         out->incomplete += st[q] == ST_INCOMPLETE;
     }
     out->device_ms = ms;
+    out->decode_kernel_ms = (double)v.kernel_ns * 1e-6;
     if (h.has_model && v.exec_steps != v.sched_steps)
         throw SaraError(SARA_EDEVICE, "decode steps run (" + std::to_string(v.exec_steps) +
                                           ") differ from the schedule (" + std::to_string(v.sched_steps) + ")");
@@ -1046,6 +1054,7 @@ void profile_impl(sara_handle &h, int which, int rows, int ctx, int iters, doubl
         for (int sp = 0; sp < nsplit; ++sp) items.push_back(make_int2(r, sp));
     }
     StepVars v{};
+    v.kt0 = ~0ull;
     v.live = rows;
     v.att_items = rows * nsplit;
     v.att_span = span;
@@ -1165,6 +1174,21 @@ int sara_profile(sara_handle *h, int32_t kernel, int32_t rows, int32_t ctx, int3
     if (!h) return SARA_EINVAL;
     return guard(h, [&] { profile_impl(*h, kernel, rows, ctx, iters, ms_per_launch); });
 }
+
+int sara_set_limits(sara_handle *h, const sara_limits *lim) {
+    if (!h || !lim) return SARA_EINVAL;
+    if (lim->wait_limit_ns < 0 || lim->max_loop_iters < 0 || lim->stall_phase < -1 ||
+        (h->has_model && lim->stall_phase >= h->n_phase_cnt)) {
+        h->err = "limits out of range";
+        return SARA_EINVAL;
+    }
+    h->wait_ns = (uint64_t)lim->wait_limit_ns;
+    h->max_iters = lim->max_loop_iters;
+    h->stall_idx = lim->stall_phase;
+    return SARA_OK;
+}
+
+int sara_abi_version(void) { return SARA_ABI_VERSION; }
 
 const char *sara_last_error(const sara_handle *h) { return h ? h->err.c_str() : g_create_error.c_str(); }
 

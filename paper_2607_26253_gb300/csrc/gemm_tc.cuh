@@ -1,4 +1,4 @@
-// Projection GEMM of the decode / prefill path on sm_103a:
+// Projection GEMM of the prefill path on sm_103a:
 //     Y[r][n] = sum_c X[r][c] * W[n][c]        (X: activations, W: a linear layer's weight)
 // computed "swap-AB" on the 5th-generation tensor core: the weight tile is the MMA's A
 // operand (M = 128 output features), the activation rows are B (N = rows rounded up to
@@ -32,7 +32,6 @@ enum EpiKind : int {
     EPI_QKV = 1,     // RMSNorm scale, RoPE on q/k, q -> q_out (fp16), k/v -> KV cache (fp16)
     EPI_RESID = 2,   // x += Y; xg = x * g_next as a bf16 hi/lo pair; per-tile sum of squares of x
     EPI_SWIGLU = 3,  // RMSNorm scale; tile = 64 gate rows + 64 up rows -> h = silu(g) * u (hi/lo)
-    EPI_LMHEAD = 4,  // RMSNorm scale; optional fp32 logits; Gumbel-max partial argmax per tile
 };
 
 constexpr int kGemmThreads = 192;
@@ -57,7 +56,7 @@ struct GemmParams {
     int *ws_cnt;               // [tiles] arrival counters, zero between launches
     int *err;
     // outputs / epilogue inputs
-    float *y_f32; int ld;      // EPI_F32 output, EPI_LMHEAD logits (optional); row stride
+    float *y_f32; int ld;      // EPI_F32 output; row stride
     const float *ssq;          // [ssq_tiles][rows_cap] per-128-feature partial sums of x^2
     int ssq_tiles; float inv_dim; float eps;
     uint16_t *q_out;           // EPI_QKV: [rows][n_heads * head_dim] fp16
@@ -75,8 +74,6 @@ struct GemmParams {
     float *ssq_out;            // EPI_RESID [m_tiles][rows_cap]
     uint16_t *h_out;           // EPI_SWIGLU [rows][ld] bf16 hi
     uint16_t *h_lo;            //   and bf16 lo
-    const uint64_t *row_seed;  // EPI_LMHEAD sampler key of the row
-    float *arg_val; int *arg_idx;  // EPI_LMHEAD [rows][m_tiles] partial max / argmax
     uint64_t *stamps;          // optional [gridDim.x][16] phase timestamps (profiling builds)
 };
 
@@ -95,7 +92,6 @@ struct GemmSmem {
     float inv_rms[kTileR];
     int row_pos[kTileR];               // per-row metadata of the tile being finished
     int row_slot[kTileR];
-    unsigned long long row_seed[kTileR];
     float xch[kTileM * kEpiLd];        // exchange tile: 128 features x 32 columns
 };
 
@@ -137,7 +133,7 @@ __device__ __forceinline__ void gemm_epilogue_chunk(const GemmParams &p, GemmSme
         for (int c = 0; c < 32; ++c)
             if (c < ncols) p.y_f32[(int64_t)(r_base + c0 + c) * p.ld + n] = v[c];
     } else {
-        if constexpr (EPI == EPI_QKV || EPI == EPI_SWIGLU || EPI == EPI_LMHEAD) {
+        if constexpr (EPI == EPI_QKV || EPI == EPI_SWIGLU) {
 #pragma unroll
             for (int c = 0; c < 32; ++c) v[c] *= S.inv_rms[c0 + c];
         }
@@ -158,16 +154,6 @@ __device__ __forceinline__ void gemm_epilogue_chunk(const GemmParams &p, GemmSme
                     p.xg_out[idx] = hi;
                     p.xg_lo[idx] = lo;
                     v[c] = x * x;
-                }
-            }
-        }
-        if constexpr (EPI == EPI_LMHEAD) {
-#pragma unroll
-            for (int c = 0; c < 32; ++c) {
-                if (c < ncols) {
-                    const int r = r_base + c0 + c;
-                    if (p.y_f32) p.y_f32[(int64_t)r * p.ld + n] = v[c];
-                    v[c] += gumbel_from_hash(splitmix_at(S.row_seed[c0 + c], (uint64_t)n + 1));
                 }
             }
         }
@@ -221,34 +207,14 @@ __device__ __forceinline__ void gemm_epilogue_chunk(const GemmParams &p, GemmSme
                     }
                 }
             }
-        } else if constexpr (EPI == EPI_RESID || EPI == EPI_LMHEAD) {
+        } else if constexpr (EPI == EPI_RESID) {
             // thread etid reduces column c = etid / 4 over features [32 * (etid % 4), +32)
             const int c = etid >> 2, part = etid & 3;
-            if constexpr (EPI == EPI_RESID) {
-                float s = 0.f;
-                for (int f = 0; f < 32; ++f) s += S.xch[(part * 32 + f) * kEpiLd + c];
-                s += __shfl_xor_sync(0xffffffffu, s, 1);
-                s += __shfl_xor_sync(0xffffffffu, s, 2);
-                if (part == 0 && c < ncols) p.ssq_out[(int64_t)m_tile * p.rows_cap + r_base + c0 + c] = s;
-            } else {
-                float best = -INFINITY;
-                int bi = 0x7fffffff;
-                for (int f = 0; f < 32; ++f) {
-                    const float z = S.xch[(part * 32 + f) * kEpiLd + c];
-                    if (z > best) { best = z; bi = m_tile * kTileM + part * 32 + f; }
-                }
-#pragma unroll
-                for (int o = 1; o <= 2; o <<= 1) {
-                    const float ob = __shfl_xor_sync(0xffffffffu, best, o);
-                    const int oi = __shfl_xor_sync(0xffffffffu, bi, o);
-                    if (ob > best || (ob == best && oi < bi)) { best = ob; bi = oi; }
-                }
-                if (part == 0 && c < ncols) {
-                    const int r = r_base + c0 + c;
-                    p.arg_val[(int64_t)r * p.m_tiles + m_tile] = best;
-                    p.arg_idx[(int64_t)r * p.m_tiles + m_tile] = bi;
-                }
-            }
+            float s = 0.f;
+            for (int f = 0; f < 32; ++f) s += S.xch[(part * 32 + f) * kEpiLd + c];
+            s += __shfl_xor_sync(0xffffffffu, s, 1);
+            s += __shfl_xor_sync(0xffffffffu, s, 2);
+            if (part == 0 && c < ncols) p.ssq_out[(int64_t)m_tile * p.rows_cap + r_base + c0 + c] = s;
         }
         named_bar_sync(1, 128);  // xch reused by the next chunk
     }
@@ -429,12 +395,12 @@ gemm_tc_kernel(const __grid_constant__ CUtensorMap tmW, const __grid_constant__ 
         const int mrow = quarter * 32 + lane;
         const int etid = threadIdx.x - 64;  // 0..127
         const uint32_t lane_base = (uint32_t)(quarter * 32) << 16;
-        // Per-row values (1/rms, position, KV slot, sampler key) staged once per tile: in
+        // Per-row values (1/rms, position, KV slot) staged once per tile: in
         // decode mode every tile has the same rows, so they are loaded once, while the
         // mainloop streams weights.
         int staged_rbase = -1;
         auto stage_rows = [&](int r_base, int rin) {
-            if constexpr (EPI == EPI_QKV || EPI == EPI_SWIGLU || EPI == EPI_LMHEAD) {
+            if constexpr (EPI == EPI_QKV || EPI == EPI_SWIGLU) {
                 if (etid < rin) {
                     const int r = r_base + etid;
                     float part[16];
@@ -450,12 +416,10 @@ gemm_tc_kernel(const __grid_constant__ CUtensorMap tmW, const __grid_constant__ 
                         S.row_pos[etid] = p.row_pos[r];
                         S.row_slot[etid] = p.row_slot[r];
                     }
-                    if constexpr (EPI == EPI_LMHEAD) S.row_seed[etid] = p.row_seed[r];
                 } else {
                     S.inv_rms[etid] = 0.f;
                     S.row_pos[etid] = 0;
                     S.row_slot[etid] = 0;
-                    S.row_seed[etid] = 0ull;
                 }
                 named_bar_sync(1, 128);
             }

@@ -1,5 +1,6 @@
-// Kernel-level entry points of include/sara.h: the projection GEMM, decode attention and the
-// Gumbel-max sampler on caller-provided device buffers (the same kernels the step runs).
+// Kernel-level entry points of include/sara.h on caller-provided device buffers: the
+// prefill's projection GEMM and attention kernels, and a one-CTA-per-row Gumbel-max sampler
+// (the decode step's sampling rule).
 #include <cuda.h>
 #include <cuda_runtime.h>
 

@@ -122,7 +122,13 @@ static __global__ void __launch_bounds__(256) sample_finish_kernel(StepPtrs c, c
     __syncthreads();
     if (!s_last) return;
     __threadfence();
-    if (tid == 0) V.fin_count = 0;
+    if (tid == 0) {
+        V.fin_count = 0;
+        // the preceding decode-step launch's duration into the step's kernel-time total
+        if (V.kt1 > V.kt0) V.kernel_ns += (int64_t)(V.kt1 - V.kt0);
+        V.kt0 = ~0ull;
+        V.kt1 = 0ull;
+    }
     if (live == 0) return;
     for (int i = tid; i < live; i += blockDim.x) {  // each row's token: argmax over its chunks
         float best = __ldcg(&c.arg_val[(int64_t)i * kSampleChunks]);
@@ -245,6 +251,7 @@ static __global__ void __launch_bounds__(kCtlThreads, 1) teacher_setup_kernel(St
         z.pre_rows = n * Lpre;
         z.n_fresh = n;
         z.round_maxL = K.T_forced;
+        z.kt0 = ~0ull;
         V = z;
     }
 }

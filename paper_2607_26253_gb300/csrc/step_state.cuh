@@ -23,6 +23,10 @@ struct StepConst {
     int32_t max_gen;      // stride of the generated-token output
     int32_t attn_chunk;   // decode attention: positions per KV block
     int32_t att_slots;    // decode attention: units one step runs at once, per kv head
+    int32_t max_iters;    // bound on the step loop's iterations (0: none beyond the round bounds)
+    int32_t stall_plus1;  // test hook: 1 + the decode-step phase counter whose waits never
+                          // complete (0: none)
+    int64_t wait_ns;      // limit of the decode step's bounded waits (0: the built-in 2 s)
 };
 
 // Scalar progress of the step (device, reset by the init kernel).
@@ -41,6 +45,10 @@ struct StepVars {
     int32_t iters;         // loop iterations
     int32_t att_span;      // KV blocks per decode attention split of the next step
     int64_t used, C, cursor, drawn, gen_tokens, sched_steps, exec_steps, rounds_done;
+    // decode-step kernel time: the launch in flight's earliest CTA start and latest CTA end
+    // (globaltimer ns; kt0 = ~0 between launches), folded into kernel_ns by the bookkeeping
+    unsigned long long kt0, kt1;
+    int64_t kernel_ns;
 };
 
 // KV blocks per decode attention split: the smallest span that leaves at most `slots` split

@@ -20,7 +20,9 @@ SARA_OK, SARA_EINVAL, SARA_ENOMEM, SARA_ETIMEOUT, SARA_EDEVICE = 0, -1, -2, -3, 
 UNDRAWN, COMMITTED, ABANDONED, INCOMPLETE = 0, 2, 3, 4
 EXPORTED = ("sara_create", "sara_collect_step", "sara_teacher_force", "sara_last_error", "sara_destroy",
             "sara_gemm_workspace_bytes", "sara_gemm_bf16", "sara_attention_workspace_bytes",
-            "sara_attention_decode", "sara_sample", "sara_profile", "sara_gemm_bf16_static")
+            "sara_attention_decode", "sara_sample", "sara_profile", "sara_gemm_bf16_static", "sara_set_limits",
+            "sara_abi_version")
+ABI_VERSION = 2
 
 c_p = ctypes.c_void_p
 
@@ -55,7 +57,13 @@ class Result(ctypes.Structure):
                 ("on_device", ctypes.c_int32), ("rollouts", ctypes.c_int64), ("gen_tokens", ctypes.c_int64),
                 ("prefill_tokens", ctypes.c_int64), ("decode_steps", ctypes.c_int64), ("rounds", ctypes.c_int64),
                 ("committed", ctypes.c_int64), ("abandoned", ctypes.c_int64), ("incomplete", ctypes.c_int64),
-                ("prompts_drawn", ctypes.c_int64), ("device_ms", ctypes.c_double)]
+                ("prompts_drawn", ctypes.c_int64), ("device_ms", ctypes.c_double),
+                ("decode_kernel_ms", ctypes.c_double)]
+
+
+class Limits(ctypes.Structure):
+    _fields_ = [("wait_limit_ns", ctypes.c_int64), ("max_loop_iters", ctypes.c_int32),
+                ("stall_phase", ctypes.c_int32)]
 
 
 class SaraError(RuntimeError):
@@ -105,6 +113,12 @@ def load(path: str = LIB_PATH):
     lib.sara_profile.restype = ctypes.c_int
     lib.sara_gemm_bf16_static.argtypes = [c_p, c_p, c_p, ctypes.c_int32, ctypes.c_int32, ctypes.c_int32, c_p]
     lib.sara_gemm_bf16_static.restype = ctypes.c_int
+    lib.sara_set_limits.argtypes = [c_p, ctypes.POINTER(Limits)]
+    lib.sara_set_limits.restype = ctypes.c_int
+    lib.sara_abi_version.argtypes = []
+    lib.sara_abi_version.restype = ctypes.c_int
+    if lib.sara_abi_version() != ABI_VERSION:
+        raise ImportError(f"{path} has ABI version {lib.sara_abi_version()}, this binding {ABI_VERSION}: rebuild it")
     if path == LIB_PATH:
         _lib = lib
     return lib
@@ -158,7 +172,8 @@ class StepOutput:
     decided_round: object
     tokens: object
     counters: dict
-    device_ms: float
+    device_ms: float          # the step's kernels, inputs already on the device
+    decode_kernel_ms: float   # summed decode-step kernel launches (device clock)
 
 
 class Handle:
@@ -207,17 +222,21 @@ class Handle:
     def collect_step(self, *, thresholds, lengths, N: int, k: int, n0: int, tau, target_B: int,
                      reward_seed: int, tokens=None, prompt_len: int | None = None, commit_min: int = 0,
                      prior=(1, 1), sample_seed: int = 0, want_tokens: bool = False,
-                     outputs_on_device: bool = False, schedule: int = 0) -> StepOutput:
+                     outputs_on_device: bool = False, schedule: int = 0, outputs: dict | None = None) -> StepOutput:
         """One rollout-collection step (Algorithm 1).  Inputs are numpy arrays (host) or torch
         CUDA tensors (device); outputs are numpy arrays, or torch CUDA tensors when
-        outputs_on_device."""
+        outputs_on_device.  `outputs` may hold preallocated arrays (keys status, n, s,
+        decided_round and, with want_tokens, tokens [P, k, max_gen_len]) of the same kind."""
         P = int(thresholds.shape[0])
         on_dev = not isinstance(thresholds, np.ndarray)
         Lp = int(tokens.shape[1]) if tokens is not None else (prompt_len or 1)
         pr = Prompts(P, Lp, _ptr(tokens), _ptr(thresholds), _ptr(lengths), 1 if on_dev else 0)
         t = tau_fraction(tau)
         th = Thresholds(t.numerator, t.denominator, commit_min, prior[0], prior[1], target_B, sample_seed, schedule)
-        if outputs_on_device:
+        if outputs is not None:
+            status, n, s, rnd = outputs["status"], outputs["n"], outputs["s"], outputs["decided_round"]
+            toks = outputs["tokens"] if want_tokens else None
+        elif outputs_on_device:
             import torch
             status = torch.zeros(P, dtype=torch.uint8, device="cuda")
             n = torch.zeros(P, dtype=torch.uint8, device="cuda")
@@ -235,7 +254,12 @@ class Handle:
         _check(load().sara_collect_step(self._h, ctypes.byref(pr), N, k, n0, ctypes.byref(th), reward_seed,
                                         ctypes.byref(res)), self._h)
         counters = {name: int(getattr(res, name)) for name in COUNTERS}
-        return StepOutput(status, n, s, rnd, toks, counters, float(res.device_ms))
+        return StepOutput(status, n, s, rnd, toks, counters, float(res.device_ms), float(res.decode_kernel_ms))
+
+    def set_limits(self, wait_limit_ns: int = 0, max_loop_iters: int = 0, stall_phase: int = -1):
+        """Failure limits of later calls (see sara_set_limits); no arguments restores the defaults."""
+        lim = Limits(wait_limit_ns, max_loop_iters, stall_phase)
+        _check(load().sara_set_limits(self._h, ctypes.byref(lim)), self._h)
 
     def profile(self, kernel: int, rows: int, ctx: int, iters: int = 20) -> float:
         """Milliseconds per launch of the decode step (kernel 0) or of the decode-step kernel

@@ -67,7 +67,11 @@ def test_tiny_step_schedule_and_tokens(tiny):
             cut = int(low[0]) if low.size else L  # from a near-tie on, the draws may legitimately differ
             assert np.array_equal(got[:cut], toks[:cut]), (q, j, got[:cut + 1], toks[:cut + 1])
             compared += cut
-    assert compared > 0.7 * out.counters["gen_tokens"]
+    # a near-tie (top-two Gumbel-max margin < 1e-2, ~60x the logit error of this shape) ends a
+    # rollout's comparison; the top-two gap of 512 Gumbel scores is near Exp(1), so about 1 % of
+    # the draws are near-ties and ~90 % of the tokens are compared on average
+    print(f"compared {compared} of {out.counters['gen_tokens']} tokens")
+    assert compared > 0.8 * out.counters["gen_tokens"]
 
 
 def test_tiny_step_is_deterministic_and_reusable(tiny):

@@ -114,3 +114,49 @@ def test_async_schedule_when_the_budget_does_not_bind():
         asy = oa.collect_workload(w, si, reserve=reserve)
         assert asy.counters["committed"] == sync.counters["committed"]
         assert asy.counters["decode_steps"] < 0.5 * sync.counters["decode_steps"]
+
+
+# --------------------------------------------------------------------------------------------
+# Hand-worked cases with unequal lengths.  Every verdict is fixed by the thresholds (0: every
+# rollout fails), tau = 0 and commit floor 2, so a group is never abandoned before n = k (rule
+# (iii) needs p_eff < 0) and, all-fail, it continues one rollout at a time with
+# p_eff(n, 0) = (k - n) / (k + 1) (Prop. 1): 0.4 at n = 2, 0.2 at n = 3 for k = 4.  A batch
+# started at step t0 with lengths L occupies steps t0 .. t0 + max L - 1; the prompt is decided at
+# the end of that step; new rollouts start at the next step.
+def _hand_case(lengths, P, B, N):
+    thr = np.zeros(P, np.uint64)
+    return oa.collect_step(thr, np.array(lengths, np.int32), k=4, n0=2, tau=0.0, target_B=B, N=N,
+                           reward_seed=9, commit_min=2)
+
+
+def test_hand_worked_ties_budget_and_next_step_start():
+    # q0 [3,1,2,5], q1 [1,1,4,1], q2 [2,2,1,1]; B = 2, N = 9.
+    # step 0: draw q0 (probe ends step 2, used 2), q1 (ends step 0, used 4); 2 in flight.
+    # end of 0: q1 n=2 -> continue, funded (used 5): j=2 (L=4) runs steps 1..4.
+    # end of 2: q0 n=2 -> continue, funded (used 6): j=2 (L=2) runs steps 3..4.
+    # end of 4: q0 and q1 both n=3, p_eff 0.2 each: tie -> stream order; q0 j=3 (L=5) runs
+    #           5..9 (used 7), q1 j=3 (L=1) runs 5..5 (used 8).
+    # end of 5: q1 n=4 all-fail -> ABANDON (event 3); a fresh probe needs 10 > 9: q2 not drawn.
+    # end of 9: q0 n=4 -> ABANDON (event 4).  decode steps 10, tokens 11 + 7 = 18.
+    r = _hand_case([[3, 1, 2, 5], [1, 1, 4, 1], [2, 2, 1, 1]], P=3, B=2, N=9)
+    assert list(r.status) == [oc.ABANDONED, oc.ABANDONED, oc.UNDRAWN]
+    assert list(r.n) == [4, 4, 0] and list(r.s) == [0, 0, 0]
+    assert list(r.decided_step) == [9, 5, -1] and list(r.decided_event) == [4, 3, -1]
+    assert r.counters == {"rollouts": 8, "gen_tokens": 18, "prefill_tokens": 0, "decode_steps": 10, "events": 5,
+                          "committed": 0, "abandoned": 2, "incomplete": 0, "prompts_drawn": 2}
+
+
+def test_hand_worked_priority_beats_stream_order_at_one_boundary():
+    # q0 [1,1,2,9], q1 [3,3,9,9]; B = 2, N = 6.
+    # step 0: draw q0 (probe ends step 0, used 2), q1 (ends step 2, used 4).
+    # end of 0: q0 n=2 -> continue, funded (used 5): j=2 (L=2) runs steps 1..2 (had it started at
+    #           step 0 it would end at 1 and be funded alone).
+    # end of 2: q0 n=3 (p_eff 0.2) and q1 n=2 (p_eff 0.4) decided together; one rollout of budget
+    #           left: q1 first by p_eff (against stream order), j=2 (L=9) runs 3..11 (used 6);
+    #           q0 cannot be funded -> INCOMPLETE.
+    # end of 11: q1 n=3 -> continue, unfunded -> INCOMPLETE.  decode steps 12, tokens 4 + 15.
+    r = _hand_case([[1, 1, 2, 9], [3, 3, 9, 9]], P=2, B=2, N=6)
+    assert list(r.status) == [oc.INCOMPLETE, oc.INCOMPLETE]
+    assert list(r.n) == [3, 3] and list(r.decided_step) == [-1, -1]
+    assert r.counters == {"rollouts": 6, "gen_tokens": 19, "prefill_tokens": 0, "decode_steps": 12, "events": 3,
+                          "committed": 0, "abandoned": 0, "incomplete": 2, "prompts_drawn": 2}
