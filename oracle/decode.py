@@ -48,11 +48,18 @@ def rope(x: np.ndarray, pos: np.ndarray, theta: float) -> np.ndarray:
 
 def causal_gqa_attention(q: np.ndarray, k: np.ndarray, v: np.ndarray) -> np.ndarray:
     """q [T, H, hd], k/v [T, KVH, hd] -> [T, H, hd]; softmax(q k^T / sqrt(hd)) v, causal."""
+    return gqa_attention_after(q, k, v, 0)
+
+
+def gqa_attention_after(q: np.ndarray, k: np.ndarray, v: np.ndarray, past: int) -> np.ndarray:
+    """Causal attention of queries at positions past .. past + T - 1: q [T, H, hd] against the
+    keys / values of positions 0 .. past + T - 1, k/v [past + T, KVH, hd] -> [T, H, hd];
+    query i sees keys 0 .. past + i."""
     T, H, hd = q.shape
     kvh = k.shape[1]
     group = H // kvh
     out = np.empty_like(q)
-    mask = np.triu(np.ones((T, T), dtype=bool), 1)
+    mask = np.triu(np.ones((T, k.shape[0]), dtype=bool), past + 1)
     for h in range(H):
         kh = h // group
         sc = (q[:, h, :] @ k[:, kh, :].T) / np.sqrt(hd)
@@ -69,11 +76,16 @@ def silu(z: np.ndarray) -> np.ndarray:
 
 
 def _f64(bits: np.ndarray) -> np.ndarray:
+    """bf16 bit patterns -> float64 (float64 arrays pass through unchanged)."""
+    if bits.dtype == np.float64:
+        return bits
     return synth.bf16_bits_to_f32(bits).astype(np.float64)
 
 
-def decoder_layer(x: np.ndarray, W: dict, m: synth.ModelShape, pos: np.ndarray) -> np.ndarray:
-    """One pre-norm decoder layer on one sequence x [T, d]."""
+def decoder_layer(x: np.ndarray, W: dict, m: synth.ModelShape, pos: np.ndarray, past=None, keep=None) -> np.ndarray:
+    """One pre-norm decoder layer on one sequence x [T, d] at positions pos.  past: the
+    (k, v) of this layer for the positions before pos[0] (a cached prefix), or None; keep: a
+    list that receives this call's (k, v) after RoPE."""
     T = x.shape[0]
     hd = m.head_dim
     h = rmsnorm(x, _f64(W["attn_norm"]), m.rms_eps)
@@ -82,7 +94,13 @@ def decoder_layer(x: np.ndarray, W: dict, m: synth.ModelShape, pos: np.ndarray) 
     v = (h @ _f64(W["wv"]).T).reshape(T, m.n_kv_heads, hd)
     q = rope(q, pos, m.rope_theta)
     k = rope(k, pos, m.rope_theta)
-    o = causal_gqa_attention(q, k, v).reshape(T, m.n_heads * hd)
+    if keep is not None:
+        keep.append((k, v))
+    if past is None:
+        o = causal_gqa_attention(q, k, v)
+    else:
+        o = gqa_attention_after(q, np.concatenate([past[0], k]), np.concatenate([past[1], v]), past[0].shape[0])
+    o = o.reshape(T, m.n_heads * hd)
     x = x + o @ _f64(W["wo"]).T
     h2 = rmsnorm(x, _f64(W["mlp_norm"]), m.rms_eps)
     a = silu(h2 @ _f64(W["wgate"]).T) * (h2 @ _f64(W["wup"]).T)
@@ -188,3 +206,39 @@ def teacher_forced_logits_batch(W: Weights, prompts: np.ndarray, forced: np.ndar
     Lp, T = prompts.shape[1], forced.shape[1]
     seqs = np.concatenate([prompts, forced[:, :-1]], axis=1)
     return forward_logits(W, seqs, logit_positions=np.arange(Lp - 1, Lp - 1 + T))
+
+
+def teacher_forced_logits_shared_prefix(W: Weights, prefix: np.ndarray, suffixes: np.ndarray,
+                                        forced: np.ndarray) -> np.ndarray:
+    """teacher_forced_logits_batch for prompts that share a long prefix: prompt i is
+    prefix + suffixes[i] ([S, Ls]); forced [S, T] -> float64 [S, T, V].  The same forward as
+    forward_logits: the prefix's keys and values of every layer are computed once and each
+    sequence's later positions attend to them as they would in the full causal forward."""
+    m = W.m
+    prefix = np.asarray(prefix, dtype=np.int64)
+    suffixes = np.atleast_2d(np.asarray(suffixes, dtype=np.int64))
+    forced = np.atleast_2d(np.asarray(forced, dtype=np.int64))
+    S, Ls = suffixes.shape
+    T = forced.shape[1]
+    Lc = prefix.size
+    embed = W.g["embed"]
+    # prefix: every layer's (k, v) after RoPE
+    cache = []
+    x = _f64(embed[prefix])
+    pos = np.arange(Lc)
+    for l in range(m.layers):
+        keep = []
+        x = decoder_layer(x, W.layer(l), m, pos, keep=keep)
+        cache.append(keep[0])
+    # each sequence's own positions Lc .. Lc + Ls + T - 2
+    seqs = np.concatenate([suffixes, forced[:, :-1]], axis=1)
+    n = seqs.shape[1]
+    pos = Lc + np.arange(n)
+    xs = [_f64(embed[seqs[i]]) for i in range(S)]
+    for l in range(m.layers):
+        Wl = {key: _f64(val) for key, val in W.layer(l).items()}  # converted once for all sequences
+        xs = [decoder_layer(x, Wl, m, pos, past=cache[l]) for x in xs]
+    gf = _f64(W.g["final_norm"])
+    lm = _f64(W.g["lm_head"])
+    sel = np.arange(Ls - 1, Ls - 1 + T)
+    return np.stack([rmsnorm(x[sel], gf, m.rms_eps) @ lm.T for x in xs])

@@ -38,7 +38,8 @@
 //   6 FIN_GU h = silu(r g) * (r u), r = 1/rms(x)  (bf16 hi/lo, blocked)
 //   7 DOWN  h W_down^T -> partials
 //   8 FIN_D x += sum; x_g = x * g_next; sum of squares
-// then lm_head over whole 256-token tiles, writing the logits of the live rows.
+// then lm_head over whole 256-token tiles fused with the Gumbel-max sampler: per (row, tile,
+// half-tile) maximum of logit + noise; the logits are stored only under teacher forcing.
 //
 // Layouts (all chosen so that bulk copies land MMA operands in shared memory in the
 // 128-byte-swizzled K-major form the tensor core reads):
@@ -99,7 +100,8 @@ struct MegaParams {
     uint16_t *qkv16;                                // [rows_cap][nqkv] fp16 q (scaled), k, v of the step
     float *part;                                    // [items][KVH][Gq][hd + 2] attention split partials
     int *att_cnt;                                   // [rows_cap][KVH] split arrival counters
-    float *logits;                                  // [rows_cap][V] fp32 (read by the sampling kernel)
+    float *logits;                                  // [rows_cap][V] fp32, written if write_logits
+    int write_logits;                               // teacher forcing: store the logits too
     unsigned long long *cnt;                        // phase arrival counters (monotonic), kCntStride apart
     unsigned long long *epoch;                      // launches completed since the reset
     uint64_t *stamps;                               // profiling builds: [cta][phase + 1][4] timestamps
@@ -1133,9 +1135,14 @@ __device__ __forceinline__ void mega_compute(const MegaParams &p, MegaSmem &S, u
         arrive(base + kPhFinD, true);
     }
 
-    // ---------------------------------------------------------------- lm_head
-    // logits = (x_g W_lm^T) / rms(x) for the live rows; the sampling kernel that follows
-    // spreads the Gumbel-max over the whole GPU
+    // ---------------------------------------------------------------- lm_head + Gumbel-max
+    // logits = (x_g W_lm^T) / rms(x) for the live rows, fused with the temperature-1 sampler:
+    // each thread scans its row's 128 columns of a tile in increasing token order, adds the
+    // Gumbel noise g(row key, token) and keeps the first maximum of logit + g; the per (row,
+    // tile, half) maxima go to the bookkeeping kernel, which takes the row's argmax (ties to
+    // the lowest token id).  Products and sums are rounded separately (no contraction), as
+    // the sampler on stored logits would do them.  The logits themselves are written only
+    // when requested (teacher forcing).
     {
         wait_phase(kPhasesPerLayer * p.layers);
         load_rstd(p.ssqA);
@@ -1144,13 +1151,19 @@ __device__ __forceinline__ void mega_compute(const MegaParams &p, MegaSmem &S, u
         gemm_range(g, u0, u1);
         const bool act = my_row < R;
         const float rs = act ? S.rstd[my_row] : 0.f;
+        const uint64_t seed = act ? __ldg(&p.c.row_seed[my_row]) : 0ull;
+        const int nparts = 2 * g.T;
+        float best = -INFINITY;  // running over this thread's tiles (its row and half)
+        int bi = 0x7fffffff;
         for (int64_t u = u0; u < u1; u += g.kch) {
             const int t = (int)(u / g.kch);
             const int a = tseg & 1;
             mwait(&S.acc_full[a], (a ? cuse1 : cuse0) & 1, err, ab, lim);
             tc_fence_after();
             if (quarter_live && half * 128 < tile_rows(g, t)) {
-                float *dst = p.logits + (int64_t)(act ? my_row : 0) * p.V + t * kTileN + half * 128;
+                const int n0 = t * kTileN + half * 128;
+                float *dst = p.logits + (int64_t)(act ? my_row : 0) * p.V + n0;
+                const float best0 = best;  // the maximum over this thread's earlier tiles
 #pragma unroll 1
                 for (int cc = 0; cc < 4; ++cc) {
                     float v[32];
@@ -1160,11 +1173,47 @@ __device__ __forceinline__ void mega_compute(const MegaParams &p, MegaSmem &S, u
                         for (int e = 0; e < 32; ++e) v[e] += __shfl_xor_sync(0xffffffffu, v[e], 8);
                     }
                     if (act) {
-                        float4 *q = reinterpret_cast<float4 *>(dst + cc * 32);
 #pragma unroll
-                        for (int e = 0; e < 8; ++e)
-                            q[e] = make_float4(v[4 * e] * rs, v[4 * e + 1] * rs, v[4 * e + 2] * rs, v[4 * e + 3] * rs);
+                        for (int e = 0; e < 32; ++e) v[e] = __fmul_rn(v[e], rs);
+                        if (p.write_logits) {
+                            float4 *q = reinterpret_cast<float4 *>(dst + cc * 32);
+#pragma unroll
+                            for (int e = 0; e < 8; ++e) q[e] = make_float4(v[4 * e], v[4 * e + 1], v[4 * e + 2], v[4 * e + 3]);
+                        }
+                        // Only tokens whose noise could lift them over the best so far are
+                        // evaluated exactly: g(u) increases with u = (top 24 hash bits + 0.5) / 2^24,
+                        // so v_e + g(u_e) > best needs u_e > exp(-exp(-(best - max_e v_e))); the
+                        // cut is taken 1e-3 lower in g and 4 codes lower in the 24-bit u, far
+                        // beyond the rounding of the float evaluation, so no candidate is lost.
+                        // `best` runs over all of this thread's tiles: a (tile, half) whose
+                        // tokens cannot beat an earlier tile's maximum reports -inf, which the
+                        // row's argmax ignores (ties go to the lower token id either way).
+                        float vmax = v[0];
+#pragma unroll
+                        for (int e = 1; e < 32; ++e) vmax = fmaxf(vmax, v[e]);
+                        const float ureq = expf(-expf(-(best - vmax - 1e-3f)));  // 0 while best = -inf
+                        const float cut = ureq * 16777216.0f - 4.0f;
+                        const uint32_t thr = cut > 0.f ? (uint32_t)cut : 0u;
+                        const int nb = n0 + cc * 32;
+                        uint32_t cand = 0;
+#pragma unroll
+                        for (int e = 0; e < 32; ++e)
+                            cand |= (uint32_t)((uint32_t)(splitmix_at(seed, (uint64_t)(nb + e) + 1) >> 40) >= thr) << e;
+                        while (cand) {  // candidates in increasing token order: the first maximum is kept
+                            const int e = __ffs(cand) - 1;
+                            cand &= cand - 1;
+                            float ve = v[0];
+#pragma unroll
+                            for (int k = 1; k < 32; ++k) ve = (k == e) ? v[k] : ve;
+                            const float z = __fadd_rn(ve, gumbel_from_hash(splitmix_at(seed, (uint64_t)(nb + e) + 1)));
+                            if (z > best) { best = z; bi = nb + e; }
+                        }
                     }
+                }
+                if (act) {  // this (tile, half)'s maximum if it beats the earlier tiles, else -inf
+                    const bool won = best > best0;
+                    p.c.arg_val[(int64_t)my_row * nparts + 2 * t + half] = won ? best : -INFINITY;
+                    p.c.arg_idx[(int64_t)my_row * nparts + 2 * t + half] = won ? bi : 0x7fffffff;
                 }
             }
             tc_fence_before();

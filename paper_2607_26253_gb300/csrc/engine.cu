@@ -369,6 +369,7 @@ MegaParams mega_params(const sara_handle &h) {
     p.part = h.attn_part;
     p.att_cnt = h.attn_cnt;
     p.logits = h.logit_buf;
+    p.write_logits = 0;
     p.cnt = h.phase_cnt;
     p.epoch = h.phase_cnt + (size_t)h.n_phase_cnt * kCntStride;
     p.stamps = h.stamps;
@@ -378,11 +379,13 @@ MegaParams mega_params(const sara_handle &h) {
 }
 
 // One decode step over the live rows: the persistent decode-step kernel (embedding, every
-// layer, lm_head logits) followed by the Gumbel-max sampling and bookkeeping kernel.
-void enqueue_decode_step(sara_handle &h, cudaStream_t s) {
-    launch_ex(s, false, true, dim3(h.sms), dim3(kMegaThreads), kMegaSmemBytes, decode_step_kernel, mega_params(h));
-    launch(s, false, dim3(h.cfg.max_seqs, kSampleChunks), dim3(256), 0, sample_finish_kernel, h.ptrs,
-           (const float *)h.logit_buf, h.cfg.vocab);
+// layer, lm_head with the fused Gumbel-max maxima) followed by the sampling finish and
+// bookkeeping kernel.  write_logits: also store the fp32 logits (teacher forcing).
+void enqueue_decode_step(sara_handle &h, cudaStream_t s, bool write_logits = false) {
+    MegaParams mp = mega_params(h);
+    mp.write_logits = write_logits ? 1 : 0;
+    launch_ex(s, false, true, dim3(h.sms), dim3(kMegaThreads), kMegaSmemBytes, decode_step_kernel, mp);
+    launch(s, false, dim3(h.cfg.max_seqs), dim3(256), 0, sample_finish_kernel, h.ptrs, h.cfg.vocab);
 }
 
 // Prefill of the fresh prompts of a round: embedding, every layer up to the last layer's
@@ -749,9 +752,10 @@ void create_impl(sara_handle &h, const sara_model_cfg *cfgp, const sara_weights 
         const int Gq = m.n_heads / KVH;
         h.attn_part = h.mem.alloc<float>((size_t)h.att_cap * KVH * Gq * (hd + 2), false);
         h.attn_cnt = h.mem.alloc<int>((size_t)S * KVH);
-        c.lm_tiles = kSampleChunks;
-        h.lm_val = h.mem.alloc<float>((size_t)S * kSampleChunks, false);
-        h.lm_idx = h.mem.alloc<int>((size_t)S * kSampleChunks, false);
+        // the lm_head epilogue's sampler maxima: [rows][2 per 256-token tile]
+        c.lm_tiles = (m.vocab + kTileN - 1) / kTileN;
+        h.lm_val = h.mem.alloc<float>((size_t)S * 2 * c.lm_tiles, false);
+        h.lm_idx = h.mem.alloc<int>((size_t)S * 2 * c.lm_tiles, false);
         h.logit_buf = h.mem.alloc<float>((size_t)S * m.vocab, false);
         c.arg_val = h.lm_val;
         c.arg_idx = h.lm_idx;
@@ -925,7 +929,7 @@ void teacher_impl(sara_handle &h, int n, int Lp, const int32_t *prompts, int T, 
         enqueue_prefill(h, s, false);
         enqueue_kv_fanout(h, s, false, c);
         for (int step = 0; step < T; ++step) {
-            enqueue_decode_step(h, s);
+            enqueue_decode_step(h, s, true);
             // rows stay in rollout order for all T steps (every rollout has length T)
             CK(cudaMemcpy2DAsync(logits + (size_t)step * m.vocab, (size_t)T * m.vocab * 4, h.logit_buf,
                                  (size_t)m.vocab * 4, (size_t)m.vocab * 4, n, kout, s));

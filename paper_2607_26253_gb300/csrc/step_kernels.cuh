@@ -63,15 +63,13 @@ __device__ __forceinline__ int scan256(int v, int &total, int *warp_tot) {
     return before + x - v;
 }
 
-constexpr int kSampleChunks = 8;  // vocabulary chunks per row (one CTA each)
-
-// Gumbel-max sampling + step bookkeeping.  CTA (r, ch), r < live, draws the Gumbel noise of
-// tokens [ch * V / 8, ..) of row r from the row's sampler key, adds it to the logits and
-// keeps the argmax (ties: lowest token id).  The last CTA to finish reduces each row's
-// chunk partials, then appends each row's token to its rollout, retires rollouts that
-// reached their length, compacts the live rows (order kept) and writes the next step's rows
-// and attention items.
-static __global__ void __launch_bounds__(256) sample_finish_kernel(StepPtrs c, const float *logits, int vocab) {
+// Sampling finish + step bookkeeping, after the decode-step kernel.  That kernel's lm_head
+// epilogue left, per live row, the first maximum of logit + Gumbel noise of every (256-token
+// tile, 128-token half) (arg_val / arg_idx [rows][2 * tiles]); CTA r reduces row r's maxima
+// to its token (ties: lowest token id).  The last CTA to finish appends each row's token to
+// its rollout, retires rollouts that reached their length, compacts the live rows (order
+// kept) and writes the next step's rows and attention items.
+static __global__ void __launch_bounds__(256) sample_finish_kernel(StepPtrs c, int vocab) {
     __shared__ float sv[8];
     __shared__ int si[8];
     __shared__ int s_last;
@@ -80,23 +78,17 @@ static __global__ void __launch_bounds__(256) sample_finish_kernel(StepPtrs c, c
     pdl_allow_dependents();
     StepVars &V = *c.v;
     const int live = V.live;
-    const int r = blockIdx.x, ch = blockIdx.y;
+    const int r = blockIdx.x;
     const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
     if (r < live) {
-        const int chunk = ((vocab + kSampleChunks - 1) / kSampleChunks + 3) & ~3;
-        const int n0 = ch * chunk, n1 = min(vocab, n0 + chunk);
-        const uint64_t seed = c.row_seed[r];
-        const float *lr = logits + (int64_t)r * vocab;
+        const int tiles = (vocab + 255) / 256, nparts = 2 * tiles;
         float best = -INFINITY;
         int bi = 0x7fffffff;
-        for (int n = n0 + 4 * tid; n < n1; n += 4 * blockDim.x) {
-            const float4 l4 = __ldcg(reinterpret_cast<const float4 *>(lr + n));
-            const float l[4] = {l4.x, l4.y, l4.z, l4.w};
-#pragma unroll
-            for (int e = 0; e < 4; ++e) {
-                const float z = l[e] + gumbel_from_hash(splitmix_at(seed, (uint64_t)(n + e) + 1));
-                if (z > best) { best = z; bi = n + e; }
-            }
+        for (int j = tid; j < nparts; j += blockDim.x) {
+            if ((j & 1) * 128 >= min(256, vocab - 256 * (j >> 1))) continue;  // a half tile past the vocabulary
+            const float v = __ldcg(&c.arg_val[(int64_t)r * nparts + j]);
+            const int id = __ldcg(&c.arg_idx[(int64_t)r * nparts + j]);
+            if (v > best || (v == best && id < bi)) { best = v; bi = id; }
         }
 #pragma unroll
         for (int o = 16; o > 0; o >>= 1) {
@@ -109,15 +101,14 @@ static __global__ void __launch_bounds__(256) sample_finish_kernel(StepPtrs c, c
         if (tid == 0) {
             for (int w = 1; w < 8; ++w)
                 if (sv[w] > best || (sv[w] == best && si[w] < bi)) { best = sv[w]; bi = si[w]; }
-            c.arg_val[(int64_t)r * kSampleChunks + ch] = best;
-            c.arg_idx[(int64_t)r * kSampleChunks + ch] = bi;
+            c.sampled[r] = bi;
         }
     }
     __threadfence();
     __syncthreads();
     if (tid == 0) {
         const int old = atomicAdd(&V.fin_count, 1);
-        s_last = (old == (int)(gridDim.x * gridDim.y) - 1);
+        s_last = (old == (int)gridDim.x - 1);
     }
     __syncthreads();
     if (!s_last) return;
@@ -130,17 +121,6 @@ static __global__ void __launch_bounds__(256) sample_finish_kernel(StepPtrs c, c
         V.kt1 = 0ull;
     }
     if (live == 0) return;
-    for (int i = tid; i < live; i += blockDim.x) {  // each row's token: argmax over its chunks
-        float best = __ldcg(&c.arg_val[(int64_t)i * kSampleChunks]);
-        int bi = __ldcg(&c.arg_idx[(int64_t)i * kSampleChunks]);
-        for (int q = 1; q < kSampleChunks; ++q) {
-            const float v = __ldcg(&c.arg_val[(int64_t)i * kSampleChunks + q]);
-            const int id = __ldcg(&c.arg_idx[(int64_t)i * kSampleChunks + q]);
-            if (v > best || (v == best && id < bi)) { best = v; bi = id; }
-        }
-        c.sampled[i] = bi;
-    }
-    __syncthreads();
     const StepConst &K = *c.kc;
     const int Lp = K.Lp;
     // bookkeeping over the live rows (several passes of 256)

@@ -158,3 +158,45 @@ def test_full_shape_step_schedule_1p5b(pkg):
         for j in range(int(out.n[q])):
             t = out.tokens[q, j, :si.lengths[q, j]]
             assert t.min() >= 0 and t.max() < w.model.vocab
+
+
+# Long contexts at the full shapes: many rows over a 2,000-token shared prefix, so that the
+# decode step runs the paths the benchmark runs -- 26 rows (one stacked hi/lo operand per
+# k-step) and 80 rows (above 64: hi and lo as separate 128-row operands), attention units of
+# several KV blocks and rows split over several units, merged by the O projection.  The
+# oracle computes the prefix once (its keys and values are shared) and then every row's own
+# positions; rows differ in their last 4 prompt tokens and in their forced tokens.
+LONG_PREFIX, LONG_SUFFIX, LONG_T, LONG_ROWS = 2000, 4, 2, 80
+
+
+@pytest.fixture(scope="module", params=["1.5b", "3b"])
+def long_case(pkg, request):
+    w = synth.WORKLOADS[request.param]
+    m = w.model
+    weights = synth.model_weights(m, w.weight_seed)
+    rng = np.random.default_rng(20)
+    prefix = rng.integers(0, m.vocab, LONG_PREFIX).astype(np.int32)
+    suffixes = rng.integers(0, m.vocab, (LONG_ROWS, LONG_SUFFIX)).astype(np.int32)
+    forced = rng.integers(0, m.vocab, (LONG_ROWS, LONG_T)).astype(np.int32)
+    want = o2.teacher_forced_logits_shared_prefix(o2.Weights(m, weights), prefix, suffixes, forced)
+    prompts = np.concatenate([np.tile(prefix, (LONG_ROWS, 1)), suffixes], axis=1)
+    cfg = pkg.model_cfg(m, max_prompts=LONG_ROWS, max_active=LONG_ROWS, max_seqs=128,
+                        max_prompt_len=prompts.shape[1], max_gen_len=8, max_k=w.k)
+    h = pkg.Handle(cfg, weights)
+    yield w, h, prompts, forced, want
+    h.close()
+
+
+@pytest.mark.parametrize("n", [26, LONG_ROWS])
+def test_full_shape_long_context_teacher_forced(long_case, n):
+    w, h, prompts, forced, want = long_case
+    uids = np.arange(n, dtype=np.int64) * 64 + 3
+    logits, sampled = h.teacher_force(prompts[:n], forced[:n], uids, w.sample_seed)
+    err, rel = logit_errors(logits, want[:n])
+    print(f"{w.model.name} rows {n} context {prompts.shape[1]}: max-abs {err:.2e} rel-L2 {rel:.2e}")
+    assert err < LOGIT_MAX_ABS and rel < LOGIT_REL_L2, (err, rel)
+    for i in range(n):
+        for t in range(LONG_T):
+            tok, margin = o2.sample_token(logits[i, t], w.sample_seed, int(uids[i]), t)
+            if margin > 1e-4:
+                assert sampled[i, t] == tok, (i, t)

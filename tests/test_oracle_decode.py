@@ -171,3 +171,28 @@ def test_gumbel_max_samples_softmax():
     big = np.zeros(100)
     big[42] = 60.0
     assert all(o2.sample_token(big, 1, u, 0)[0] == 42 for u in range(50))
+
+
+def test_attention_after_a_cached_prefix_equals_the_full_causal_attention():
+    rng = np.random.default_rng(7)
+    Tall, past, H, KVH, hd = 23, 15, 6, 2, 8
+    q = rng.standard_normal((Tall, H, hd))
+    k = rng.standard_normal((Tall, KVH, hd))
+    v = rng.standard_normal((Tall, KVH, hd))
+    full = o2.causal_gqa_attention(q, k, v)
+    tail = o2.gqa_attention_after(q[past:], k, v, past)
+    assert np.allclose(tail, full[past:], rtol=0, atol=1e-13)
+
+
+def test_shared_prefix_teacher_forcing_equals_full_recompute(tiny_weights):
+    W = tiny_weights
+    rng = np.random.default_rng(8)
+    V = W.m.vocab
+    prefix = rng.integers(0, V, 21)
+    suffixes = rng.integers(0, V, (3, 4))
+    forced = rng.integers(0, V, (3, 5))
+    got = o2.teacher_forced_logits_shared_prefix(W, prefix, suffixes, forced)
+    prompts = np.concatenate([np.tile(prefix, (3, 1)), suffixes], axis=1)
+    want = o2.teacher_forced_logits_batch(W, prompts, forced)
+    assert got.shape == want.shape == (3, 5, V)
+    assert np.abs(got - want).max() < 1e-11 * np.abs(want).max()
