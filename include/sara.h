@@ -39,7 +39,8 @@ extern "C" {
 #endif
 
 /* Layout version of the structs below.  Version 2 added sara_thresholds.schedule,
- * sara_result.decode_kernel_ms and sara_limits; a caller built against another version
+ * sara_model_cfg.kv_blocks, sara_result.decode_kernel_ms and kv_blocks_peak, and sara_limits;
+ * a caller built against another version
  * must not pass its structs to this library (compare with sara_abi_version()). */
 #define SARA_ABI_VERSION 2
 
@@ -76,6 +77,11 @@ typedef struct {
     int32_t max_gen_len;     /* largest generated length of one rollout
                                 (max_prompt_len + max_gen_len <= 12288) */
     int32_t max_k;           /* largest group size k (<= 64) */
+    int32_t kv_blocks;       /* rollouts' private KV blocks of 128 positions in the paged cache
+                                (0: enough for max_seqs rollouts of max_gen_len); a step that
+                                needs more returns SARA_ENOMEM.  The prompts' full blocks are
+                                held apart (max_active x (max_prompt_len - 1) / 128 of them) and
+                                shared by each prompt's rollouts. */
 } sara_model_cfg;
 
 /* Policy weights, bf16 bit patterns, row-major [out_features][in_features] like a linear
@@ -148,6 +154,7 @@ typedef struct {
                                   before the output copies */
     double decode_kernel_ms;   /* summed duration of the decode-step kernel's launches (device
                                   clock, earliest CTA start to latest CTA end of each launch) */
+    int64_t kv_blocks_peak;    /* most private KV blocks in use at once during the step */
 } sara_result;
 
 /*

@@ -242,6 +242,25 @@ static __device__ void ctl_round_setup(const StepConst &K, StepVars &V, const St
         maxL = max(maxL, c.seq_len[r]);
     }
     maxL = blk_max(maxL, sh);
+    // KV blocks of the round's rollouts (the previous round's were all freed as its rollouts
+    // finished): the prompt's full blocks, shared, then one private block from the free stack
+    // for the block holding position Lp - 1 (the prompt's tail is copied into it), in slot order
+    {
+        const int nsh = shared_blocks(Lp, K.attn_chunk);
+        const int top = V.blk_top;
+        __syncthreads();
+        if (R > top) { if (threadIdx.x == 0) report_error(&V.err, ERR_CAPACITY); return; }
+        for (int r = threadIdx.x; r < R; r += kCtlThreads) {
+            int32_t *bt = c.blk_tab + (int64_t)r * c.nblk_max;
+            const int ps = c.seq_pslot[r];
+            for (int j = 0; j < nsh; ++j) bt[j] = ps * c.nsh_max + j;
+            bt[nsh] = c.blk_free[top - 1 - r];
+        }
+        if (threadIdx.x == 0) {
+            V.blk_top = top - R;
+            V.blk_low = min(V.blk_low, top - R);
+        }
+    }
     // prefill rows: fresh prompt f, token t < Lp - 1, written into prompt slot fresh_pslot[f]
     const int Lpre = Lp - 1;
     const int pre_rows = n_fresh * Lpre;
@@ -470,11 +489,14 @@ static __global__ void __launch_bounds__(kCtlThreads, 1) ctl_init_kernel(StepPtr
         c.q_pslot[q] = -1;
     }
     ctl_build_tables(K, c);
+    // every private KV block free (popped from the top: ids n_shared, n_shared + 1, .. first)
+    for (int i = threadIdx.x; i < c.n_priv; i += kCtlThreads) c.blk_free[i] = c.n_shared + c.n_priv - 1 - i;
     if (threadIdx.x == 0) {
         StepVars z;
         memset(&z, 0, sizeof(z));
         z.round = -1;
         z.kt0 = ~0ull;
+        z.blk_top = z.blk_low = c.n_priv;
         V = z;
     }
 }

@@ -66,6 +66,7 @@ constexpr int kKVPos = 128;           // positions per KV block (an attention sp
 constexpr int kKVBlockBytes = 65536;  // K 2 x 16 KB + V^T 2 x 16 KB
 constexpr int kMegaMaxSplits = 96;    // splits per row a merge handles (context <= 96 blocks)
 constexpr int kPhasesPerLayer = 9;
+constexpr int kMaxCtaBlocks = 256;    // attention KV block ids a CTA keeps in shared memory
 // phases of a layer (counter index 1 + 9 l + phase)
 enum : int { kPhQKV = 0, kPhFinQ = 1, kPhAtt = 2, kPhO = 3, kPhFinO = 4, kPhGU = 5, kPhFinGU = 6, kPhDown = 7,
              kPhFinD = 8 };
@@ -85,9 +86,8 @@ struct MegaParams {
     const uint16_t *attn_norm, *mlp_norm;           // [L][d]
     const uint16_t *final_norm;                     // [d]
     const float2 *rope;                             // [positions][hd/2] (cos, sin)
-    uint8_t *kv;                                    // blocked KV cache
-    int64_t kv_layer, kv_slot;                      // bytes
-    int kv_nblk;                                    // 128-position blocks per (slot, kv head)
+    uint8_t *kv;                                    // paged KV cache: block id b of layer l, kv head h
+    int64_t kv_layer;                               // at kv + l * kv_layer + (b * KVH + h) * 64 KB
     StepPtrs c;
     int rows_cap, rows_cap16;
     int gp_qkv, gp_o;                               // CTAs taking part in the QKV / O projections
@@ -150,6 +150,12 @@ struct MegaSmem {
     int last_flag;
     int rows, rows16, nx, nx_lg, n_items, att_span;  // nx = 2^nx_lg X stages
     float rstd[128];
+    // KV block ids: of this CTA's attention blocks (unit i's block j at ablk[aoff[i] + j]), and
+    // of each row's current position (ablk_ok = 0: too many to hold, looked up in the table)
+    int ablk[kMaxCtaBlocks];
+    int aoff[32];
+    int rowblk[128];
+    int ablk_ok;
     float red[2][4][8], red2[2][4][8];  // per warp group: attention max / sum reductions
     float mw[2][8][kMegaMaxSplits];      // per warp group: split weights of a merge
     float ml[2][8];
@@ -330,10 +336,55 @@ __device__ __forceinline__ void att_range(const MegaParams &p, int n_items, int6
     a0 = v * NU / G;
     a1 = (v + 1) * NU / G;
 }
-// Block j of unit u in layer l's KV cache.
-__device__ __forceinline__ uint8_t *kv_block(const MegaParams &p, int l, const AttUnit &u, int j) {
-    return p.kv + l * p.kv_layer + (int64_t)u.slot * p.kv_slot +
-           ((int64_t)u.kvh * p.kv_nblk + u.p0 / kKVPos + j) * kKVBlockBytes;
+// Address of block id b, kv head h of layer l in the paged KV cache.
+__device__ __forceinline__ uint8_t *kv_addr(const MegaParams &p, int l, int b, int h) {
+    return p.kv + l * p.kv_layer + ((int64_t)b * p.KVH + h) * kKVBlockBytes;
+}
+// Block j of this CTA's attention unit ui (= a - a0) in layer l's KV cache.
+__device__ __forceinline__ uint8_t *kv_block(const MegaParams &p, const MegaSmem &S, int l, const AttUnit &u, int ui,
+                                             int j) {
+    const int b = S.ablk_ok ? S.ablk[S.aoff[ui] + j]
+                            : __ldg(&p.c.blk_tab[(int64_t)u.slot * p.c.nblk_max + u.p0 / kKVPos + j]);
+    return kv_addr(p, l, b, u.kvh);
+}
+
+// The KV block ids of this CTA's attention units (one warp, lane i: unit a0 + i), read once
+// per launch from the block table into shared memory for the W producer.
+__device__ __forceinline__ void fill_att_blocks(const MegaParams &p, MegaSmem &S, int lane) {
+    int64_t a0, a1;
+    att_range(p, S.n_items, a0, a1);
+    const int nu = (int)(a1 - a0);
+    bool ok = nu <= 32;
+    int nb = 0, off = 0;
+    AttUnit u{};
+    if (ok) {
+        if (lane < nu) {
+            u = att_unit(p, a0 + lane, S.att_span);
+            nb = u.nb;
+        }
+        int x = nb;  // inclusive warp scan of the block counts
+#pragma unroll
+        for (int o = 1; o < 32; o <<= 1) {
+            const int y = __shfl_up_sync(0xffffffffu, x, o);
+            if (lane >= o) x += y;
+        }
+        off = x - nb;
+        ok = __shfl_sync(0xffffffffu, x, 31) <= kMaxCtaBlocks;
+    }
+    if (ok && lane < nu) {
+        S.aoff[lane] = off;
+        const int32_t *src = p.c.blk_tab + (int64_t)u.slot * p.c.nblk_max + u.p0 / kKVPos;
+        for (int j0 = 0; j0 < nb; j0 += 8) {  // eight loads in flight
+            int v[8];
+#pragma unroll
+            for (int q = 0; q < 8; ++q) v[q] = j0 + q < nb ? __ldg(src + j0 + q) : 0;
+#pragma unroll
+            for (int q = 0; q < 8; ++q)
+                if (j0 + q < nb) S.ablk[off + j0 + q] = v[q];
+        }
+    }
+    if (lane == 0) S.ablk_ok = ok ? 1 : 0;
+    __syncwarp();
 }
 
 // ------------------------------------------------------------------------------ W producer
@@ -393,7 +444,7 @@ __device__ __forceinline__ void mega_w_producer(const MegaParams &p, MegaSmem &S
                                 fence_proxy_async_global();
                                 finq_seen = true;
                             }
-                            const uint8_t *blk = kv_block(p, l, u, j);
+                            const uint8_t *blk = kv_block(p, S, l, u, (int)(a - a0) + w, j);
                             const int nj = min(kKVPos, u.n - j * kKVPos);
                             const uint32_t kb = (uint32_t)(((nj + 7) & ~7) * 128), vb = (uint32_t)(p.hd * 128);
                             if (!acquire(wi)) { ok = false; break; }
@@ -752,6 +803,12 @@ __device__ __forceinline__ void mega_compute(const MegaParams &p, MegaSmem &S, u
         }
     };
 
+    // the KV block of each row's current position (its k, v are appended there every layer)
+    if (ctid < R) {
+        const int pos = __ldg(&p.c.row_pos[ctid]);
+        S.rowblk[ctid] = __ldg(&p.c.blk_tab[(int64_t)__ldg(&p.c.row_slot[ctid]) * p.c.nblk_max + pos / kKVPos]);
+    }
+
     // ---------------------------------------------------------------- embedding
     // (same (row, 64-feature) units and lanes as the finalisation that reads them back)
     for (int u = gw; u < R * (d / 64); u += nw) {
@@ -839,9 +896,7 @@ __device__ __forceinline__ void mega_compute(const MegaParams &p, MegaSmem &S, u
                     (uint32_t)h0 | ((uint32_t)h1 << 16);
                 if (!isq) {  // the new position's k / v into the cache (blocked layout)
                     const int kvh = head - p.H - (isk ? 0 : p.KVH);
-                    const int slot = __ldg(&p.c.row_slot[r]);
-                    uint8_t *blk = p.kv + l * p.kv_layer + (int64_t)slot * p.kv_slot +
-                                   ((int64_t)kvh * p.kv_nblk + pos / kKVPos) * kKVBlockBytes;
+                    uint8_t *blk = kv_addr(p, l, S.rowblk[r], kvh);
                     const int pp = pos % kKVPos;
                     if (isk) {
                         *reinterpret_cast<uint32_t *>(blk + kv_k_off(pp, d0)) = (uint32_t)h0 | ((uint32_t)h1 << 16);
@@ -1287,6 +1342,7 @@ __global__ void __launch_bounds__(kMegaThreads, 1) decode_step_kernel(const __gr
     const bool run = !S.abort && S.rows > 0;
     if (run) {
         if (warp == 0) {
+            fill_att_blocks(p, S, lane);
             if (lane == 0) mega_w_producer(p, S, sW);
         } else if (warp == 1) {
             if (lane == 0) mega_mma(p, S, sW, sX, sQ, sP, tmem);
@@ -1325,52 +1381,78 @@ static __global__ void block_weights_kernel(const uint16_t *src, uint8_t *dst, i
     }
 }
 
-// Copy every layer's prompt KV (positions < Lp - 1, row-major [2][n_kv][cap_p][hd] per prompt
-// slot) into rollout slot s < live in the blocked decode layout (run once at a round start).
-// One thread per K granule (8 dims of a position) or per V granule (8 positions of a dim).
-static __global__ void kv_fanout_kernel(const uint16_t *pkv, uint8_t *kv, const StepPtrs c, int layers, int n_kv,
-                                        int hd, int cap_p, int64_t kv_layer, int64_t kv_slot, int nblk,
-                                        int max_active) {
+// Round start of the paged KV cache, from the prefill's row-major prompt KV ([2][n_kv][cap_p]
+// [hd] per prompt slot and layer, positions < Lp - 1): (a) every fresh prompt's full blocks
+// (positions < nsh * 128), which its rollouts share; (b) every live rollout's private block
+// holding position Lp - 1, filled with the prompt's tail positions nsh * 128 .. Lp - 2.  One
+// thread per K granule (8 dims of a position) or V granule (8 positions of a dim).
+static __global__ void prompt_blocks_kernel(const uint16_t *pkv, uint8_t *kv, const StepPtrs c, int layers, int n_kv,
+                                            int hd, int cap_p, int64_t kv_layer, int max_active) {
     pdl_wait_prior_grids();
     pdl_allow_dependents();
-    const int live = c.v->live;
-    const int Lpre = c.kc->Lp - 1;
+    const int live = c.v->live, n_fresh = c.v->n_fresh;
+    const int Lp = c.kc->Lp, Lpre = Lp - 1;
+    const int nsh = shared_blocks(Lp, kKVPos);
     const int gk = hd / 8;
-    const int64_t nk = (int64_t)Lpre * gk;
-    const int64_t nv = (int64_t)((Lpre + 7) / 8) * hd;
-    const int64_t per = nk + nv;
-    const int64_t total = (int64_t)layers * live * n_kv * per;
+    // per (layer, kv head) plane: K granules npos * gk, then V granules ceil(npos / 8) * hd
+    const int na = nsh * kKVPos, nt = Lpre - na;  // positions of a shared plane / of a tail plane
+    const int64_t per_a = (int64_t)na * gk + (int64_t)(na / 8) * hd;
+    const int64_t per_b = (int64_t)nt * gk + (int64_t)((nt + 7) / 8) * hd;
+    const int64_t tot_a = (int64_t)n_fresh * layers * n_kv * per_a;
+    const int64_t total = tot_a + (int64_t)live * layers * n_kv * per_b;
     for (int64_t e = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; e < total; e += (int64_t)gridDim.x * blockDim.x) {
-        int64_t rem = e;
-        const int64_t per_layer = (int64_t)live * n_kv * per;
-        const int l = (int)(rem / per_layer);
-        rem -= l * per_layer;
-        const int s = (int)(rem / ((int64_t)n_kv * per));
-        rem -= (int64_t)s * n_kv * per;
+        int64_t rem;
+        int owner, npos, p0;  // owner: fresh prompt f or rollout slot s; positions [p0, p0 + npos)
+        int64_t per;
+        if (e < tot_a) {
+            rem = e;
+            per = per_a;
+            npos = na;
+            p0 = 0;
+        } else {
+            rem = e - tot_a;
+            per = per_b;
+            npos = nt;
+            p0 = na;
+        }
+        const int64_t per_owner = (int64_t)layers * n_kv * per;
+        owner = (int)(rem / per_owner);
+        rem -= (int64_t)owner * per_owner;
+        const int l = (int)(rem / ((int64_t)n_kv * per));
+        rem -= (int64_t)l * n_kv * per;
         const int kvh = (int)(rem / per);
         rem -= (int64_t)kvh * per;
-        const int ps = c.seq_pslot[s];
+        const bool shared = e < tot_a;
+        const int ps = shared ? c.fresh_pslot[owner] : c.seq_pslot[owner];
         const uint16_t *kplane = pkv + (((int64_t)l * max_active + ps) * 2 * n_kv + kvh) * cap_p * hd;
         const uint16_t *vplane = kplane + (int64_t)n_kv * cap_p * hd;
-        uint8_t *dst = kv + l * kv_layer + (int64_t)s * kv_slot + (int64_t)kvh * nblk * kKVBlockBytes;
-        if (rem < nk) {
-            const int pos = (int)(rem / gk), j = (int)(rem - (int64_t)pos * gk);
-            const uint4 v = *reinterpret_cast<const uint4 *>(kplane + (int64_t)pos * hd + j * 8);
-            *reinterpret_cast<uint4 *>(dst + (int64_t)(pos / kKVPos) * kKVBlockBytes + kv_k_off(pos % kKVPos, j * 8)) = v;
+        const int nk = npos * gk;
+        int pos, dd = 0;
+        bool isk = rem < nk;
+        if (isk) {
+            pos = p0 + (int)(rem / gk);
+            dd = (int)(rem - (int64_t)(pos - p0) * gk) * 8;
         } else {
             rem -= nk;
-            const int pg = (int)(rem / hd), dd = (int)(rem - (int64_t)pg * hd);
+            pos = p0 + (int)(rem / hd) * 8;
+            dd = (int)(rem - (int64_t)((pos - p0) / 8) * hd);
+        }
+        const int b = pos / kKVPos;
+        const int blk = shared ? ps * c.nsh_max + b : c.blk_tab[(int64_t)owner * c.nblk_max + b];
+        uint8_t *dst = kv + l * kv_layer + ((int64_t)blk * n_kv + kvh) * kKVBlockBytes;
+        if (isk) {
+            const uint4 v = *reinterpret_cast<const uint4 *>(kplane + (int64_t)pos * hd + dd);
+            *reinterpret_cast<uint4 *>(dst + kv_k_off(pos % kKVPos, dd)) = v;
+        } else {
             uint32_t w[4];
 #pragma unroll
             for (int q = 0; q < 4; ++q) {
-                const int p0 = pg * 8 + 2 * q;
-                const uint32_t a = p0 < Lpre ? vplane[(int64_t)p0 * hd + dd] : 0u;
-                const uint32_t b = p0 + 1 < Lpre ? vplane[(int64_t)(p0 + 1) * hd + dd] : 0u;
-                w[q] = a | (b << 16);
+                const int pa = pos + 2 * q;
+                const uint32_t x = pa < Lpre ? vplane[(int64_t)pa * hd + dd] : 0u;
+                const uint32_t y = pa + 1 < Lpre ? vplane[(int64_t)(pa + 1) * hd + dd] : 0u;
+                w[q] = x | (y << 16);
             }
-            const int pos = pg * 8;
-            *reinterpret_cast<uint4 *>(dst + (int64_t)(pos / kKVPos) * kKVBlockBytes + kv_v_off(pos % kKVPos, dd)) =
-                make_uint4(w[0], w[1], w[2], w[3]);
+            *reinterpret_cast<uint4 *>(dst + kv_v_off(pos % kKVPos, dd)) = make_uint4(w[0], w[1], w[2], w[3]);
         }
     }
 }

@@ -71,10 +71,10 @@ struct sara_handle {
     uint8_t *wb_qkv = nullptr, *wb_o = nullptr, *wb_gu = nullptr, *wb_down = nullptr, *wb_lm = nullptr;
     int64_t ls_qkv = 0, ls_o = 0, ls_gu = 0, ls_down = 0;
     // KV caches: rollout slots in the blocked decode layout, prompt slots row-major
-    uint8_t *kv_seq = nullptr;
+    uint8_t *kv_seq = nullptr;  // paged KV pool: [layer][block id][kv head] 64 KB blocks
     uint16_t *kv_pr = nullptr;
-    int cap_s = 0, cap_p = 0, kv_nblk = 0;
-    int64_t kv_seq_layer = 0, kv_seq_slot = 0, kv_pr_layer = 0, kv_pr_slot = 0;
+    int cap_s = 0, cap_p = 0;
+    int64_t kv_seq_layer = 0, kv_pr_layer = 0, kv_pr_slot = 0;
     float2 *rope = nullptr;
     Acts pre;
     // decode-step activations (blocked operands) and phase counters
@@ -351,8 +351,6 @@ MegaParams mega_params(const sara_handle &h) {
     p.rope = h.rope;
     p.kv = h.kv_seq;
     p.kv_layer = h.kv_seq_layer;
-    p.kv_slot = h.kv_seq_slot;
-    p.kv_nblk = h.kv_nblk;
     p.c = h.ptrs;
     p.rows_cap = m.max_seqs;
     p.rows_cap16 = h.rows_cap16;
@@ -408,15 +406,15 @@ void enqueue_prefill(sara_handle &h, cudaStream_t s, bool pdl) {
     }
 }
 
-void enqueue_kv_fanout(sara_handle &h, cudaStream_t s, bool pdl, const StepPtrs &c) {
+void enqueue_prompt_blocks(sara_handle &h, cudaStream_t s, bool pdl, const StepPtrs &c) {
     const sara_model_cfg &m = h.cfg;
-    launch(s, pdl, dim3(h.sms * 8), dim3(256), 0, kv_fanout_kernel, (const uint16_t *)h.kv_pr, h.kv_seq, c, m.layers,
-           m.n_kv_heads, m.head_dim, h.cap_p, h.kv_seq_layer, h.kv_seq_slot, h.kv_nblk, m.max_active);
+    launch(s, pdl, dim3(h.sms * 8), dim3(256), 0, prompt_blocks_kernel, (const uint16_t *)h.kv_pr, h.kv_seq, c,
+           m.layers, m.n_kv_heads, m.head_dim, h.cap_p, h.kv_seq_layer, m.max_active);
 }
 
 void enqueue_round_start(sara_handle &h, cudaStream_t s, bool pdl) {
     enqueue_prefill(h, s, pdl);
-    enqueue_kv_fanout(h, s, pdl, h.ptrs);
+    enqueue_prompt_blocks(h, s, pdl, h.ptrs);
 }
 
 // ------------------------------------------------------------------------ graph
@@ -648,6 +646,7 @@ void validate_cfg(const sara_model_cfg &m) {
     if (m.vocab % 128 || m.vocab < 128) bad("vocab must be a multiple of 128");
     if (m.max_seqs < 1 || m.max_seqs > kTileR) bad("max_seqs must be 1..128");
     if (m.max_prompt_len < 2 || m.max_gen_len < 1) bad("max_prompt_len >= 2 and max_gen_len >= 1 required");
+    if (m.kv_blocks < 0) bad("kv_blocks < 0");
     if (!(m.rms_eps > 0.f) || !(m.rope_theta > 0.f)) bad("rms_eps and rope_theta must be positive");
 }
 
@@ -724,12 +723,18 @@ void create_impl(sara_handle &h, const sara_model_cfg *cfgp, const sara_weights 
         c.max_seqs = S;
         h.gen_tok = h.mem.alloc<int32_t>((size_t)P * K * m.max_gen_len, false);
         c.gen_tok = h.gen_tok;
-        // KV caches: rollout slots [layer][slot][kv][128-position block] in the blocked decode
-        // layout (64 KB per block, zero-filled so padded head dims read as 0); prompt slots
-        // row-major [layer][pslot][2][kv][cap_p][hd]
-        h.kv_nblk = (h.cap_s + kKVPos - 1) / kKVPos;
-        h.kv_seq_slot = (int64_t)KVH * h.kv_nblk * kKVBlockBytes;
-        h.kv_seq_layer = h.kv_seq_slot * S;
+        // Paged KV cache of 128-position blocks in the decode layout (64 KB per block and kv
+        // head, zero-filled so padded head dims read as 0): the prompts' full blocks (shared by
+        // their rollouts), then the rollouts' private blocks, handed out as positions are
+        // reached and returned when a rollout finishes.  Prompt slots row-major
+        // [layer][pslot][2][kv][cap_p][hd] (the prefill's own layout).
+        c.nblk_max = (h.cap_s + kKVPos - 1) / kKVPos;
+        c.nsh_max = shared_blocks(m.max_prompt_len, kKVPos);
+        c.n_shared = Bc * c.nsh_max;
+        c.n_priv = m.kv_blocks > 0 ? m.kv_blocks : S * ((m.max_gen_len + kKVPos - 1) / kKVPos + 2);
+        c.blk_tab = h.mem.alloc<int32_t>((size_t)S * c.nblk_max);
+        c.blk_free = h.mem.alloc<int32_t>((size_t)c.n_priv);
+        h.kv_seq_layer = (int64_t)(c.n_shared + c.n_priv) * KVH * kKVBlockBytes;
         h.kv_pr_slot = 2LL * KVH * h.cap_p * hd;
         h.kv_pr_layer = h.kv_pr_slot * Bc;
         h.kv_seq = h.mem.alloc<uint8_t>((size_t)h.kv_seq_layer * m.layers);
@@ -882,6 +887,7 @@ void collect_impl(sara_handle &h, const sara_prompts *pr, int64_t N, int32_t k, 
     }
     out->device_ms = ms;
     out->decode_kernel_ms = (double)v.kernel_ns * 1e-6;
+    out->kv_blocks_peak = h.has_model ? (int64_t)(h.ptrs.n_priv - v.blk_low) : 0;
     if (h.has_model && v.exec_steps != v.sched_steps)
         throw SaraError(SARA_EDEVICE, "decode steps run (" + std::to_string(v.exec_steps) +
                                           ") differ from the schedule (" + std::to_string(v.sched_steps) + ")");
@@ -927,7 +933,7 @@ void teacher_impl(sara_handle &h, int n, int Lp, const int32_t *prompts, int T, 
         reset_decode_state(h, s);
         launch(s, false, dim3(1), dim3(kCtlThreads), 0, teacher_setup_kernel, c, n, (const int64_t *)h.uid_dev);
         enqueue_prefill(h, s, false);
-        enqueue_kv_fanout(h, s, false, c);
+        enqueue_prompt_blocks(h, s, false, c);
         for (int step = 0; step < T; ++step) {
             enqueue_decode_step(h, s, true);
             // rows stay in rollout order for all T steps (every rollout has length T)
@@ -1057,14 +1063,24 @@ void profile_impl(sara_handle &h, int which, int rows, int ctx, int iters, doubl
         uid[r] = r;
         for (int sp = 0; sp < nsplit; ++sp) items.push_back(make_int2(r, sp));
     }
+    const StepPtrs &c = h.ptrs;
+    // KV blocks: row r's blocks of positions < ctx are private ids (wrapping round the pool if
+    // it is smaller: the values read are then another row's, which only timing sees); later
+    // blocks come from a full free stack
+    std::vector<int32_t> bt((size_t)rows * c.nblk_max, c.n_shared), fr(c.n_priv);
+    for (int r = 0; r < rows; ++r)
+        for (int j = 0; j < nblk; ++j) bt[(size_t)r * c.nblk_max + j] = c.n_shared + (r * nblk + j) % c.n_priv;
+    for (int i = 0; i < c.n_priv; ++i) fr[i] = c.n_shared + c.n_priv - 1 - i;
     StepVars v{};
     v.kt0 = ~0ull;
     v.live = rows;
     v.att_items = rows * nsplit;
     v.att_span = span;
     v.round_maxL = 1 << 30;
-    const StepPtrs &c = h.ptrs;
+    v.blk_top = v.blk_low = c.n_priv;
     reset_decode_state(h, s);
+    CK(cudaMemcpyAsync(c.blk_tab, bt.data(), bt.size() * 4, cudaMemcpyHostToDevice, s));
+    CK(cudaMemcpyAsync(c.blk_free, fr.data(), fr.size() * 4, cudaMemcpyHostToDevice, s));
     CK(cudaMemcpyAsync(h.kc, &K, sizeof(K), cudaMemcpyHostToDevice, s));
     CK(cudaMemcpyAsync(h.vars, &v, sizeof(v), cudaMemcpyHostToDevice, s));
     CK(cudaMemcpyAsync(c.row_slot, slot.data(), rows * 4, cudaMemcpyHostToDevice, s));

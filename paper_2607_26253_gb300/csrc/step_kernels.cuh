@@ -122,9 +122,11 @@ static __global__ void __launch_bounds__(256) sample_finish_kernel(StepPtrs c, i
     }
     if (live == 0) return;
     const StepConst &K = *c.kc;
-    const int Lp = K.Lp;
+    const int Lp = K.Lp, B = K.attn_chunk;
+    const int nsh = shared_blocks(Lp, B);
     // bookkeeping over the live rows (several passes of 256)
     int out = 0;
+    int top = V.blk_top, low = V.blk_low;  // the KV block free stack (same value in every thread)
     for (int base = 0; base < live; base += 256) {
         const int i = base + tid;
         int keep = 0, slot = 0, gen = 0, next_tok = 0;
@@ -143,6 +145,28 @@ static __global__ void __launch_bounds__(256) sample_finish_kernel(StepPtrs c, i
             c.seq_gen[slot] = gen;
             keep = gen < c.seq_len[slot];
         }
+        // KV blocks, in row order: a finished rollout returns its private blocks (positions
+        // up to Lp - 2 + gen), then a kept one whose next position opens a block takes one
+        int32_t *bt = c.blk_tab + (int64_t)slot * c.nblk_max;
+        int nfree = 0, need = 0;
+        if (i < live) {
+            if (!keep) nfree = (Lp + gen - 2) / B - nsh + 1;
+            else need = ((Lp - 1 + gen) % B) == 0;
+        }
+        int ftot;
+        const int foff = scan256(nfree, ftot, warp_tot);
+        for (int j = 0; j < nfree; ++j) c.blk_free[top + foff + j] = bt[nsh + j];
+        top += ftot;
+        __syncthreads();
+        int atot;
+        const int aoff = scan256(need, atot, warp_tot);
+        if (need) {
+            const int at = top - 1 - aoff;
+            if (at >= 0) bt[(Lp - 1 + gen) / B] = c.blk_free[at];
+            else report_error(&V.err, ERR_CAPACITY);
+        }
+        top = max(0, top - atot);
+        low = min(low, top);
         // stable in-place compaction: a kept row lands at or before its own index
         int tot;
         const int before = scan256(keep, tot, warp_tot);
@@ -187,6 +211,8 @@ static __global__ void __launch_bounds__(256) sample_finish_kernel(StepPtrs c, i
         V.att_span = span;
         V.exec_steps += 1;
         V.round_steps += 1;
+        V.blk_top = top;
+        V.blk_low = low;
     }
 }
 
@@ -199,7 +225,14 @@ static __global__ void __launch_bounds__(kCtlThreads, 1) teacher_setup_kernel(St
     const int nblk = (Lp + K.attn_chunk - 1) / K.attn_chunk;
     const int span = att_span_for((int64_t)n * nblk, K.att_slots);
     const int nsplit = (nblk + span - 1) / span;
+    const int nsh = shared_blocks(Lp, K.attn_chunk);
+    for (int i = threadIdx.x; i < c.n_priv; i += kCtlThreads) c.blk_free[i] = c.n_shared + c.n_priv - 1 - i;
+    __syncthreads();
     for (int r = threadIdx.x; r < n; r += kCtlThreads) {
+        int32_t *bt = c.blk_tab + (int64_t)r * c.nblk_max;  // prompt r's full blocks, then a private one
+        for (int j = 0; j < nsh; ++j) bt[j] = r * c.nsh_max + j;
+        bt[nsh] = r < c.n_priv ? c.blk_free[c.n_priv - 1 - r] : c.n_shared;  // (n > n_priv: an error)
+        c.fresh_pslot[r] = r;
         c.seq_q[r] = r;
         c.seq_j[r] = 0;
         c.seq_len[r] = K.T_forced;
@@ -232,6 +265,8 @@ static __global__ void __launch_bounds__(kCtlThreads, 1) teacher_setup_kernel(St
         z.n_fresh = n;
         z.round_maxL = K.T_forced;
         z.kt0 = ~0ull;
+        z.blk_top = z.blk_low = c.n_priv - n;
+        if (n > c.n_priv) z.err |= ERR_CAPACITY;
         V = z;
     }
 }

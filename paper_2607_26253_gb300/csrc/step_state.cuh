@@ -49,6 +49,8 @@ struct StepVars {
     // (globaltimer ns; kt0 = ~0 between launches), folded into kernel_ns by the bookkeeping
     unsigned long long kt0, kt1;
     int64_t kernel_ns;
+    // paged KV cache: free private blocks on the stack, and the fewest ever free
+    int32_t blk_top, blk_low;
 };
 
 // KV blocks per decode attention split: the smallest span that leaves at most `slots` split
@@ -95,6 +97,16 @@ struct StepPtrs {
     int32_t *arg_idx;
     int32_t lm_tiles;
     int32_t max_seqs, max_active, pre_cap, att_cap;
+    // paged KV cache of 128-position blocks.  Block ids [0, n_shared) hold the prompts' full
+    // blocks (prompt slot ps owns ids ps * nsh_max ..), ids [n_shared, n_shared + n_priv) are
+    // the rollouts' private blocks, handed out from the free stack blk_free[0, blk_top).
+    int32_t *blk_tab;          // [max_seqs][nblk_max] block id of rollout slot s's block b
+    int32_t *blk_free;         // [n_priv]
+    int32_t nblk_max, nsh_max, n_shared, n_priv;
 };
+
+// Full prompt blocks (shared by a prompt's rollouts) when the prefill writes positions
+// 0 .. Lp - 2; the block holding Lp - 1, the first decode position, is each rollout's own.
+__host__ __device__ inline int shared_blocks(int Lp, int block) { return (Lp - 1) / block; }
 
 }  // namespace sara

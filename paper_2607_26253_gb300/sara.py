@@ -32,7 +32,8 @@ class ModelCfg(ctypes.Structure):
                 ("n_kv_heads", ctypes.c_int32), ("head_dim", ctypes.c_int32), ("ffn", ctypes.c_int32),
                 ("vocab", ctypes.c_int32), ("rope_theta", ctypes.c_float), ("rms_eps", ctypes.c_float),
                 ("max_prompts", ctypes.c_int32), ("max_active", ctypes.c_int32), ("max_seqs", ctypes.c_int32),
-                ("max_prompt_len", ctypes.c_int32), ("max_gen_len", ctypes.c_int32), ("max_k", ctypes.c_int32)]
+                ("max_prompt_len", ctypes.c_int32), ("max_gen_len", ctypes.c_int32), ("max_k", ctypes.c_int32),
+                ("kv_blocks", ctypes.c_int32)]
 
 
 class Weights(ctypes.Structure):
@@ -58,7 +59,7 @@ class Result(ctypes.Structure):
                 ("prefill_tokens", ctypes.c_int64), ("decode_steps", ctypes.c_int64), ("rounds", ctypes.c_int64),
                 ("committed", ctypes.c_int64), ("abandoned", ctypes.c_int64), ("incomplete", ctypes.c_int64),
                 ("prompts_drawn", ctypes.c_int64), ("device_ms", ctypes.c_double),
-                ("decode_kernel_ms", ctypes.c_double)]
+                ("decode_kernel_ms", ctypes.c_double), ("kv_blocks_peak", ctypes.c_int64)]
 
 
 class Limits(ctypes.Structure):
@@ -149,15 +150,15 @@ def tau_fraction(tau) -> Fraction:
 
 
 def model_cfg(shape, *, max_prompts: int, max_active: int, max_seqs: int, max_prompt_len: int,
-              max_gen_len: int, max_k: int = 64) -> ModelCfg:
+              max_gen_len: int, max_k: int = 64, kv_blocks: int = 0) -> ModelCfg:
     """ModelCfg from a shape with fields layers, d_model, n_heads, n_kv_heads, head_dim, ffn, vocab,
     rope_theta, rms_eps (shape=None: controller-only handle)."""
     if shape is None:
         return ModelCfg(0, 0, 0, 0, 0, 0, 0, 0.0, 0.0, max_prompts, max_active, max_seqs, max_prompt_len,
-                        max_gen_len, max_k)
+                        max_gen_len, max_k, 0)
     return ModelCfg(shape.layers, shape.d_model, shape.n_heads, shape.n_kv_heads, shape.head_dim, shape.ffn,
                     shape.vocab, shape.rope_theta, shape.rms_eps, max_prompts, max_active, max_seqs,
-                    max_prompt_len, max_gen_len, max_k)
+                    max_prompt_len, max_gen_len, max_k, kv_blocks)
 
 
 COUNTERS = ("rollouts", "gen_tokens", "prefill_tokens", "decode_steps", "rounds", "committed", "abandoned",
@@ -174,6 +175,7 @@ class StepOutput:
     counters: dict
     device_ms: float          # the step's kernels, inputs already on the device
     decode_kernel_ms: float   # summed decode-step kernel launches (device clock)
+    kv_blocks_peak: int       # most private KV blocks in use at once
 
 
 class Handle:
@@ -254,7 +256,8 @@ class Handle:
         _check(load().sara_collect_step(self._h, ctypes.byref(pr), N, k, n0, ctypes.byref(th), reward_seed,
                                         ctypes.byref(res)), self._h)
         counters = {name: int(getattr(res, name)) for name in COUNTERS}
-        return StepOutput(status, n, s, rnd, toks, counters, float(res.device_ms), float(res.decode_kernel_ms))
+        return StepOutput(status, n, s, rnd, toks, counters, float(res.device_ms), float(res.decode_kernel_ms),
+                          int(res.kv_blocks_peak))
 
     def set_limits(self, wait_limit_ns: int = 0, max_loop_iters: int = 0, stall_phase: int = -1):
         """Failure limits of later calls (see sara_set_limits); no arguments restores the defaults."""

@@ -96,3 +96,37 @@ def test_limits_out_of_range_rejected(pkg):
             with pytest.raises(pkg.SaraError) as e:
                 h.set_limits(**kw)
             assert e.value.code == pkg.SARA_EINVAL
+
+
+def test_kv_pool_exhaustion_and_exact_fit(pkg):
+    """The paged KV cache: a pool smaller than one round's rollouts returns SARA_ENOMEM (and the
+    handle stays usable); a pool of exactly the peak the step reported runs the step again with
+    the same schedule and tokens -- the cache needs blocks for live positions only."""
+    w = synth.WORKLOADS["tiny"]
+    weights = synth.model_weights(w.model, w.weight_seed)
+    si = synth.step_inputs(w)
+    with pkg.Handle(handle_cfg(w, pkg), weights) as h:
+        ref = h.collect_step(thresholds=si.thresholds, lengths=si.lengths, tokens=si.tokens, N=w.budget_N, k=w.k,
+                             n0=w.n0, tau=w.tau, target_B=w.target_B, reward_seed=w.reward_seed,
+                             sample_seed=w.sample_seed, want_tokens=True)
+    # every tiny rollout (prompt 32 + at most 32 tokens) lives in one private block: the peak is
+    # the largest round, the probe round of B x n0 rollouts
+    assert ref.kv_blocks_peak == w.target_B * w.n0
+    small = handle_cfg(w, pkg)
+    small.kv_blocks = ref.kv_blocks_peak - 1
+    with pkg.Handle(small, weights) as h:
+        with pytest.raises(pkg.SaraError) as e:
+            _step(h, w, si)
+        assert e.value.code == pkg.SARA_ENOMEM
+    exact = handle_cfg(w, pkg)
+    exact.kv_blocks = ref.kv_blocks_peak
+    with pkg.Handle(exact, weights) as h:
+        out = h.collect_step(thresholds=si.thresholds, lengths=si.lengths, tokens=si.tokens, N=w.budget_N, k=w.k,
+                             n0=w.n0, tau=w.tau, target_B=w.target_B, reward_seed=w.reward_seed,
+                             sample_seed=w.sample_seed, want_tokens=True)
+    _assert_oracle_schedule(out, w, si)
+    assert out.kv_blocks_peak == ref.kv_blocks_peak
+    for q in range(w.n_prompts):
+        for j in range(int(out.n[q])):
+            L = int(si.lengths[q, j])
+            assert np.array_equal(out.tokens[q, j, :L], ref.tokens[q, j, :L])
