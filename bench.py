@@ -439,19 +439,21 @@ def run_mine(args):
 
 def read_traffic(workload: str):
     """(DRAM bytes, algorithmic bytes) of one launch of the dominant kernel from the committed
-    ncu summary, or None."""
-    path = os.path.join(ROOT, "profiles", f"decode_step_{workload.replace('.', 'p')}_ncu.md")
-    got = {}
-    try:
-        for line in open(path):
-            for key in ("traffic_bytes_per_launch:", "algorithmic_bytes_per_launch:"):
-                if line.startswith(key):
-                    got[key] = float(line.split(":", 1)[1].split()[0])
-    except OSError:
-        return None
-    if len(got) != 2:
-        return None
-    return got["traffic_bytes_per_launch:"], got["algorithmic_bytes_per_launch:"]
+    ncu summary of the workload's model shape, or None."""
+    shape = {"1.5b": "1p5b", "oversampled": "1p5b", "3b": "3b"}.get(workload)
+    for kind in ("ncu", "dram"):
+        path = os.path.join(ROOT, "profiles", f"decode_step_{shape}_{kind}.md")
+        got = {}
+        try:
+            for line in open(path):
+                for key in ("traffic_bytes_per_launch:", "algorithmic_bytes_per_launch:"):
+                    if line.startswith(key):
+                        got[key] = float(line.split(":", 1)[1].split()[0])
+        except OSError:
+            continue
+        if len(got) == 2:
+            return got["traffic_bytes_per_launch:"], got["algorithmic_bytes_per_launch:"]
+    return None
 
 
 # --------------------------------------------------------------------------------- ncu mode

@@ -38,8 +38,9 @@
 extern "C" {
 #endif
 
-/* Layout version of the structs below.  Version 2 added sara_thresholds.schedule,
- * sara_model_cfg.kv_blocks, sara_result.decode_kernel_ms and kv_blocks_peak, and sara_limits;
+/* Layout version of the structs below.  Version 2 added sara_thresholds.schedule and decay,
+ * sara_prompts.prior_a / prior_b, sara_model_cfg.kv_blocks, sara_result.decode_kernel_ms,
+ * kv_blocks_peak and prior_a_next / prior_b_next, and sara_limits;
  * a caller built against another version
  * must not pass its structs to this library (compare with sara_abi_version()). */
 #define SARA_ABI_VERSION 2
@@ -111,6 +112,12 @@ typedef struct {
     const uint64_t *p_threshold;   /* [P] latent success rate as floor(p * 2^32); 2^32 = always */
     const int32_t *lengths;        /* [P][k] generated tokens of rollout j of prompt q, >= 1 */
     int32_t on_device;
+    const double *prior_a;         /* [P] warm-start Beta prior of each prompt (App. D: its
+                                      posterior carried from earlier steps), or NULL: every
+                                      prompt starts from the integer prior of sara_thresholds */
+    const double *prior_b;         /* [P], given together with prior_a; positive and finite.
+                                      Decisions then compare p_eff in fp64 (log-Gamma), which
+                                      agrees with exact arithmetic away from ties. */
 } sara_prompts;
 
 /* Decision-rule parameters (Eq. decide, App. D). */
@@ -130,6 +137,8 @@ typedef struct {
                                   time comes from the length table (decode_steps), rounds
                                   counts the step boundaries with decisions and decided_round
                                   holds the index of the deciding one (capped at 32767). */
+    double decay;              /* warm-start decay lambda in [0, 1] of the carried priors that
+                                  sara_result.prior_a_next / prior_b_next receive */
 } sara_thresholds;
 
 /* Results of one step.  Array pointers may be NULL (not written); they are host or device
@@ -155,6 +164,10 @@ typedef struct {
     double decode_kernel_ms;   /* summed duration of the decode-step kernel's launches (device
                                   clock, earliest CTA start to latest CTA end of each launch) */
     int64_t kv_blocks_peak;    /* most private KV blocks in use at once during the step */
+    double *prior_a_next;      /* [P] or NULL (host or device per on_device): the next step's
+                                  warm-start prior, alpha0 + decay (a - alpha0 + s) with a the
+                                  prior this step used and s the prompt's successes */
+    double *prior_b_next;      /* [P] or NULL: beta0 + decay (b - beta0 + n - s) */
 } sara_result;
 
 /*

@@ -151,6 +151,26 @@ static __device__ void ctl_build_tables(const StepConst &K, const StepPtrs &c) {
     }
 }
 
+// ------------------------------------------------------------------------------------------
+// Warm-start (App. D): a prompt's prior Beta(a, b) is real, carried from earlier steps, so the
+// predictor of Prop. 1 / Eq. (peff) is evaluated in fp64 through log-Gamma and Eq. (decide)
+// compares it with tau_low in fp64 (decisions agree with exact arithmetic away from ties).
+__device__ __forceinline__ double log_beta(double x, double y) { return lgamma(x) + lgamma(y) - lgamma(x + y); }
+__device__ __forceinline__ double peff_real(int n, int s, int k, double a, double b) {
+    if (s > 0 && s < n) return 1.0;
+    const double ap = a + s, bp = b + (n - s);
+    const int r = k - n;
+    double out = 1.0;
+    if (s == 0) out -= exp(log_beta(ap, bp + r) - log_beta(ap, bp));  // the rest all fail
+    if (s == n) out -= exp(log_beta(ap + r, bp) - log_beta(ap, bp));  // the rest all succeed
+    return out;
+}
+__device__ __forceinline__ int decide_real(int n, int s, const StepConst &K, double a, double b) {
+    if (s > 0 && s < n && n >= K.commit_min) return D_COMMIT;
+    if (n == K.k) return D_ABANDON;
+    return peff_real(n, s, K.k, a, b) < K.tau_f ? D_ABANDON : D_CONTINUE;
+}
+
 __device__ __forceinline__ int verdict_of(uint64_t seed, int64_t q, int j, uint64_t thr) {
     return (splitmix_at(seed, (uint64_t)q * 64u + (uint64_t)j + 1u) >> 32) < thr ? 1 : 0;
 }
@@ -159,12 +179,20 @@ __device__ __forceinline__ uint64_t sampler_row_seed(uint64_t sample_seed, int64
     return splitmix_at(sample_seed, (uint64_t)uid * (1ull << 20) + (uint64_t)t + 1u);
 }
 
-// use_handles: bit 0 = the loop handle exists, bit 1 = the round-start handle exists.
-__device__ __forceinline__ void set_conds(cudaGraphConditionalHandle h_loop, cudaGraphConditionalHandle h_round,
-                                          int loop, int round_start, int use_handles) {
+// The step graph's conditions: h[0] loop, h[1] rollouts join (their KV set-up runs), h[2] fresh
+// prompts are prefilled first (-1: whenever rollouts join).  use_handles: bit 0 = h[0] exists,
+// bit 1 = h[1] and h[2] exist.
+struct CondHandles {
+    cudaGraphConditionalHandle h[3];
+};
+__device__ __forceinline__ void set_conds(const CondHandles &hs, int loop, int round_start, int use_handles,
+                                          int prefill = -1) {
     if (threadIdx.x == 0) {
-        if (use_handles & 1) cudaGraphSetConditional(h_loop, loop ? 1u : 0u);
-        if (use_handles & 2) cudaGraphSetConditional(h_round, round_start ? 1u : 0u);
+        if (use_handles & 1) cudaGraphSetConditional(hs.h[0], loop ? 1u : 0u);
+        if (use_handles & 2) {
+            cudaGraphSetConditional(hs.h[1], round_start ? 1u : 0u);
+            cudaGraphSetConditional(hs.h[2], (prefill < 0 ? round_start : prefill) ? 1u : 0u);
+        }
     }
 }
 
@@ -255,10 +283,12 @@ static __device__ void ctl_round_setup(const StepConst &K, StepVars &V, const St
             const int ps = c.seq_pslot[r];
             for (int j = 0; j < nsh; ++j) bt[j] = ps * c.nsh_max + j;
             bt[nsh] = c.blk_free[top - 1 - r];
+            c.new_slots[r] = r;
         }
         if (threadIdx.x == 0) {
             V.blk_top = top - R;
             V.blk_low = min(V.blk_low, top - R);
+            V.n_new = R;
         }
     }
     // prefill rows: fresh prompt f, token t < Lp - 1, written into prompt slot fresh_pslot[f]
@@ -321,7 +351,8 @@ static __device__ void ctl_round(const StepConst &K, StepVars &V, const StepPtrs
         long long commits = 0;
         for (int i = tid; i < n_act; i += kCtlThreads) {
             const int q = c.act[i];
-            const int d = c.dec_tab[c.q_n[q] * kTabDim + c.q_s[q]];
+            const int d = K.warm ? decide_real(c.q_n[q], c.q_s[q], K, c.q_pa[q], c.q_pb[q])
+                                 : c.dec_tab[c.q_n[q] * kTabDim + c.q_s[q]];
             if (d == D_COMMIT) { c.q_status[q] = ST_COMMITTED; c.q_round[q] = (int16_t)V.round; ++commits; }
             else if (d == D_ABANDON) { c.q_status[q] = ST_ABANDONED; c.q_round[q] = (int16_t)V.round; }
         }
@@ -347,7 +378,40 @@ static __device__ void ctl_round(const StepConst &K, StepVars &V, const StepPtrs
     // ---- 3. fund continuing prompts by p_eff priority while the budget allows
     const long long budget = K.N - V.used;
     int n_funded = n_cont;
-    if ((long long)n_cont > budget) {
+    if ((long long)n_cont > budget && K.warm) {
+        // warm-start priors: p_eff is real, so each continuing prompt counts the prompts ahead
+        // of it (higher p_eff, or equal p_eff and lower stream index) over tiles of the keys
+        const int take = (int)max(0ll, budget);
+        for (int i = tid; i < n_cont; i += kCtlThreads) {
+            const int q = c.act[i];
+            c.q_key[i] = peff_real(c.q_n[q], c.q_s[q], k, c.q_pa[q], c.q_pb[q]);
+        }
+        __syncthreads();
+        __shared__ double tkey[kCtlThreads];
+        __shared__ int tq[kCtlThreads];
+        for (int base = 0; base < n_cont; base += kCtlThreads) {
+            const int i = base + tid;
+            const double ki = i < n_cont ? c.q_key[i] : 0.0;
+            const int qi = i < n_cont ? c.act[i] : 0;
+            int ahead = 0;
+            for (int t0 = 0; t0 < n_cont; t0 += kCtlThreads) {
+                __syncthreads();
+                if (t0 + tid < n_cont) {
+                    tkey[tid] = c.q_key[t0 + tid];
+                    tq[tid] = c.act[t0 + tid];
+                }
+                __syncthreads();
+                const int m = min(kCtlThreads, n_cont - t0);
+                for (int j = 0; j < m; ++j) ahead += (tkey[j] > ki) || (tkey[j] == ki && tq[j] < qi);
+            }
+            if (i < n_cont && ahead >= take) c.q_status[qi] = ST_INCOMPLETE;
+        }
+        __syncthreads();
+        n_funded = blk_compact(c.act, n_cont, c.act_tmp,
+                               [&](int i) { return c.q_status[c.act[i]] == ST_ACTIVE; }, sh);
+        for (int i = tid; i < n_funded; i += kCtlThreads) c.act[i] = c.act_tmp[i];
+        __syncthreads();
+    } else if ((long long)n_cont > budget) {
         const int take = (int)max(0ll, budget);
         for (int b = tid; b < 2 * kMaxK + 2; b += kCtlThreads) sh.hist[b] = 0;
         __syncthreads();
@@ -422,9 +486,259 @@ static __device__ void ctl_round(const StepConst &K, StepVars &V, const StepPtrs
     __syncthreads();
 }
 
+// ------------------------------------------------------------------------------------------
+// Asynchronous per-prompt schedule on the decode engine (Discussion, Limitations (ii): no round
+// barrier).  At every decode-step boundary the prompts whose batch in flight finished in the
+// step just run (dec_list, from the bookkeeping kernel) are decided as one event: verdicts of
+// the batch, DECIDE (Eq. decide) in stream order; after |C| >= B nothing is issued and
+// continuing prompts end INCOMPLETE (rollouts in flight still finish and are decided);
+// otherwise continuing prompts are funded one rollout each by p_eff rank (ties: stream index)
+// while the budget allows, then fresh prompts are drawn in stream order while fewer than
+// B - |C| prompts are in flight and a whole n0-probe fits the budget (reserve: also every prompt
+// in flight running to k).  New rollouts decode from the next step on; fresh prompts are
+// prefilled in between.  The event logic is serial (thread 0): an event holds few prompts.
+static __device__ void ctl_async_events(const StepConst &K, StepVars &V, const StepPtrs &c) {
+    const int k = K.k, n0 = K.n0, B = K.B, P = K.P;
+    const int reserve = K.schedule == 2;
+    int ni = 0;
+    int64_t used = V.used, resv = V.resv, tokens = V.gen_tokens, C = V.C, cursor = V.cursor, drawn = V.drawn;
+    int inflight = V.in_flight, ptop = V.pslot_top;
+    bool bad = false, cap = false;
+    auto issue = [&](int q, int cnt) {
+        const int n = c.q_n[q];
+        for (int j = n; j < n + cnt; ++j) {
+            const int L = c.p_len[(int64_t)q * k + j];
+            if (L < 1 || L > K.max_gen) bad = true;
+            tokens += L;
+        }
+        used += cnt;
+        if (reserve) resv += k - (n + cnt);
+        c.q_inflight[q] = cnt;
+        c.iss_q[ni] = q;
+        c.iss_c[ni] = cnt;
+        ++ni;
+        ++inflight;
+    };
+    auto free_pslot = [&](int q) { c.pslot_free[ptop++] = c.q_pslot[q]; };
+    auto draw = [&]() {
+        while (cursor < P && inflight < B - C && used + (reserve ? k : n0) + resv <= K.N) {
+            if (ptop <= 0 || ni >= c.max_active) { cap = true; break; }
+            const int q = (int)cursor++;
+            c.q_status[q] = ST_ACTIVE;
+            c.q_pslot[q] = c.pslot_free[--ptop];
+            ++drawn;
+            issue(q, n0);
+        }
+    };
+    auto key_before = [&](int p2, int q) {  // p2 funded before q: higher p_eff, then lower index
+        if (K.warm) {
+            const double a = peff_real(c.q_n[p2], c.q_s[p2], k, c.q_pa[p2], c.q_pb[p2]);
+            const double b = peff_real(c.q_n[q], c.q_s[q], k, c.q_pa[q], c.q_pb[q]);
+            return a > b || (a == b && p2 < q);
+        }
+        const int rp = c.rank_tab[c.q_n[p2] * kTabDim + c.q_s[p2]], rq = c.rank_tab[c.q_n[q] * kTabDim + c.q_s[q]];
+        return rp < rq || (rp == rq && p2 < q);
+    };
+    if (V.round < 0) {  // the first probes
+        V.round = 0;
+        draw();
+    } else if (V.n_dec > 0) {
+        const int nd = V.n_dec;
+        for (int i = 1; i < nd; ++i) {  // stream order
+            const int q = c.dec_list[i];
+            int j = i - 1;
+            while (j >= 0 && c.dec_list[j] > q) { c.dec_list[j + 1] = c.dec_list[j]; --j; }
+            c.dec_list[j + 1] = q;
+        }
+        const int ev = V.events++;
+        int ncont = 0;
+        for (int i = 0; i < nd; ++i) {
+            const int q = c.dec_list[i];
+            --inflight;
+            int n = c.q_n[q], sc = c.q_s[q];
+            const int cnt = n == 0 ? n0 : 1;
+            for (int j = n; j < n + cnt; ++j) sc += verdict_of(K.reward_seed, q, j, c.p_thr[q]);
+            n += cnt;
+            c.q_n[q] = (uint8_t)n;
+            c.q_s[q] = (uint8_t)sc;
+            if (reserve) resv -= k - n;
+            const int d = K.warm ? decide_real(n, sc, K, c.q_pa[q], c.q_pb[q]) : c.dec_tab[n * kTabDim + sc];
+            if (d == D_COMMIT) {
+                c.q_status[q] = ST_COMMITTED;
+                c.q_round[q] = (int16_t)min(ev, 32767);
+                ++C;
+                free_pslot(q);
+            } else if (d == D_ABANDON) {
+                c.q_status[q] = ST_ABANDONED;
+                c.q_round[q] = (int16_t)min(ev, 32767);
+                free_pslot(q);
+            } else {
+                c.act[ncont++] = q;
+            }
+        }
+        if (V.stopped || C >= B) {
+            V.stopped = 1;
+            for (int i = 0; i < ncont; ++i) {
+                c.q_status[c.act[i]] = ST_INCOMPLETE;
+                free_pslot(c.act[i]);
+            }
+        } else {
+            for (int i = 1; i < ncont; ++i) {  // priority order (insertion sort: few per event)
+                const int q = c.act[i];
+                int j = i - 1;
+                while (j >= 0 && !key_before(c.act[j], q)) { c.act[j + 1] = c.act[j]; --j; }
+                c.act[j + 1] = q;
+            }
+            for (int i = 0; i < ncont; ++i) {
+                const int q = c.act[i];
+                if (used + 1 <= K.N) {
+                    issue(q, 1);
+                } else {
+                    c.q_status[q] = ST_INCOMPLETE;
+                    free_pslot(q);
+                }
+            }
+            draw();
+        }
+    }
+    if (bad) report_error(&V.err, ERR_BOUNDS);
+    if (cap) report_error(&V.err, ERR_CAPACITY);
+    V.n_dec = 0;
+    V.n_iss = ni;
+    V.used = used;
+    V.resv = resv;
+    V.gen_tokens = tokens;
+    V.C = C;
+    V.cursor = cursor;
+    V.drawn = drawn;
+    V.in_flight = inflight;
+    V.pslot_top = ptop;
+}
+
+// The rollouts issued at this boundary join the live rows (all threads): rollout slots and a
+// private KV block from the free stacks, rows appended after the live ones, prefill rows of the
+// fresh prompts, then the attention items of every live row.
+static __device__ void ctl_async_join(const StepConst &K, StepVars &V, const StepPtrs &c, CtlShared &sh) {
+    const int tid = threadIdx.x;
+    const int Lp = K.Lp, Lpre = Lp - 1, nsh = shared_blocks(Lp, K.attn_chunk);
+    const int n_iss = V.n_iss, live0 = V.live, stop = V.slot_top, btop = V.blk_top;
+    int R = 0, nf = 0;
+    for (int base = 0; base < n_iss; base += kCtlThreads) {
+        const int e = base + tid;
+        const int cnt = e < n_iss ? c.iss_c[e] : 0;
+        const int q = e < n_iss ? c.iss_q[e] : 0;
+        const int fresh = (e < n_iss && c.q_n[q] == 0) ? 1 : 0;
+        int tot, ftot;
+        const int off = blk_excl_scan(cnt, tot, sh);
+        const int foff = blk_excl_scan(fresh, ftot, sh);
+        if (e < n_iss) {
+            const int ps = c.q_pslot[q];
+            for (int t = 0; t < cnt; ++t) {
+                const int r = R + off + t;  // new rollout index
+                if (r >= stop || r >= btop || live0 + r >= c.max_seqs) continue;  // capacity: reported below
+                const int slot = c.slot_free[stop - 1 - r];
+                const int j = c.q_n[q] + t;
+                c.seq_q[slot] = q;
+                c.seq_j[slot] = j;
+                c.seq_len[slot] = c.p_len[(int64_t)q * K.k + j];
+                c.seq_gen[slot] = 0;
+                c.seq_pslot[slot] = ps;
+                c.seq_uid[slot] = (int64_t)q * 64 + j;
+                int32_t *bt = c.blk_tab + (int64_t)slot * c.nblk_max;
+                for (int b = 0; b < nsh; ++b) bt[b] = ps * c.nsh_max + b;
+                bt[nsh] = c.blk_free[btop - 1 - r];
+                c.new_slots[r] = slot;
+                const int row = live0 + r;
+                c.row_slot[row] = slot;
+                c.row_pos[row] = Lp - 1;
+                c.row_tok[row] = c.p_tok[(int64_t)q * Lp + Lp - 1];
+                c.row_seed[row] = sampler_row_seed(K.sample_seed, c.seq_uid[slot], 0);
+            }
+            if (fresh) {
+                c.fresh_pslot[nf + foff] = ps;
+                c.act_tmp[nf + foff] = q;
+            }
+        }
+        R += tot;
+        nf += ftot;
+    }
+    __syncthreads();
+    if (R > stop || R > btop || live0 + R > c.max_seqs) {
+        if (tid == 0) report_error(&V.err, ERR_CAPACITY);
+        return;
+    }
+    // prefill rows of the fresh prompts (in the issue order of fresh_pslot)
+    const int pre_rows = nf * Lpre;
+    if (pre_rows > c.pre_cap) { if (tid == 0) report_error(&V.err, ERR_CAPACITY); return; }
+    for (int r = tid; r < pre_rows; r += kCtlThreads) {  // fresh prompt f = act_tmp[f], token t
+        const int f = r / Lpre, t = r - f * Lpre;
+        c.pre_slot[r] = c.fresh_pslot[f];
+        c.pre_pos[r] = t;
+        c.pre_tok[r] = c.p_tok[(int64_t)c.act_tmp[f] * Lp + t];
+        c.pre_items[r] = make_int2(r, 0);
+        c.pre_item0[r] = r;
+    }
+    __syncthreads();
+    const int live = live0 + R;
+    // attention items of every live row: splits of `span` KV blocks
+    int blocks = 0;
+    for (int base = 0; base < live; base += kCtlThreads) {
+        const int i = base + tid;
+        int tot;
+        blk_excl_scan(i < live ? (c.row_pos[i] + K.attn_chunk) / K.attn_chunk : 0, tot, sh);
+        blocks += tot;
+    }
+    const int span = att_span_for(blocks, K.att_slots);
+    int items = 0;
+    for (int base = 0; base < live; base += kCtlThreads) {
+        const int i = base + tid;
+        const int ns = (i < live) ? ((c.row_pos[i] + K.attn_chunk) / K.attn_chunk + span - 1) / span : 0;
+        int tot;
+        const int before = blk_excl_scan(ns, tot, sh);
+        if (i < live) {
+            const int i0 = items + before;
+            c.row_item0[i] = i0;
+            for (int sp = 0; sp < ns; ++sp) {
+                if (i0 + sp < c.att_cap) c.att_items[i0 + sp] = make_int2(i, sp);
+                else report_error(&V.err, ERR_CAPACITY);
+            }
+        }
+        items += tot;
+    }
+    __syncthreads();
+    if (tid == 0) {
+        V.slot_top = stop - R;
+        V.blk_top = btop - R;
+        V.blk_low = min(V.blk_low, btop - R);
+        V.n_new = R;
+        V.live = live;
+        V.att_items = min(items, c.att_cap);
+        V.att_span = span;
+        V.pre_rows = pre_rows;
+        V.n_fresh = nf;
+    }
+}
+
+static __device__ void ctl_async_step(const StepConst &K, StepVars &V, const StepPtrs &c, CtlShared &sh,
+                                      const CondHandles &hs, int use_handles) {
+    if (threadIdx.x == 0) ctl_async_events(K, V, c);
+    __syncthreads();
+    if (V.err == 0) ctl_async_join(K, V, c, sh);
+    __syncthreads();
+    const int done = V.err != 0 || V.live == 0;
+    if (done && threadIdx.x == 0) {  // nothing in flight and nothing issued: the step is over
+        V.done = 1;
+        V.live = 0;
+        V.rounds_done = V.events;
+        V.sched_steps = V.exec_steps;
+    }
+    __syncthreads();
+    set_conds(hs, !done, !done && V.n_new > 0, use_handles, !done && V.n_fresh > 0);
+}
+
 // Per-iteration controller kernel of the step graph.
 static __global__ void __launch_bounds__(kCtlThreads, 1)
-ctl_kernel(StepPtrs c, cudaGraphConditionalHandle h_loop, cudaGraphConditionalHandle h_round, int use_handles) {
+ctl_kernel(StepPtrs c, CondHandles hs, int use_handles) {
     __shared__ CtlShared sh;
     pdl_wait_prior_grids();
     const StepConst K = *c.kc;
@@ -439,26 +753,35 @@ ctl_kernel(StepPtrs c, cudaGraphConditionalHandle h_loop, cudaGraphConditionalHa
     if (V.err != 0 && !V.done) {  // a kernel reported an error: end the step now
         __syncthreads();
         if (threadIdx.x == 0) { V.done = 1; V.live = 0; }
-        set_conds(h_loop, h_round, 0, 0, use_handles);
+        set_conds(hs, 0, 0, use_handles);
         return;
     }
-    if (V.done) { set_conds(h_loop, h_round, 0, 0, use_handles); return; }
+    if (V.done) { set_conds(hs, 0, 0, use_handles); return; }
+    if (K.schedule != 0 && K.decode) {  // asynchronous: an event boundary after every decode step
+        if (V.exec_steps > (int64_t)K.N * K.max_gen + 1) {  // bound: every rollout at full length in turn
+            if (threadIdx.x == 0) { report_error(&V.err, ERR_ITER_BOUND); V.done = 1; V.live = 0; }
+            set_conds(hs, 0, 0, use_handles);
+            return;
+        }
+        ctl_async_step(K, V, c, sh, hs, use_handles);
+        return;
+    }
     if (V.live > 0) {
         // mid-round: the round may run at most round_maxL decode steps
         const int stop = V.round_steps > V.round_maxL;
         if (stop && threadIdx.x == 0) { report_error(&V.err, ERR_ITER_BOUND); V.done = 1; }
-        set_conds(h_loop, h_round, !stop, 0, use_handles);
+        set_conds(hs, !stop, 0, use_handles);
         return;
     }
     if (K.teacher) {  // teacher forcing runs one prepared round
         if (threadIdx.x == 0) V.done = 1;
-        set_conds(h_loop, h_round, 0, 0, use_handles);
+        set_conds(hs, 0, 0, use_handles);
         return;
     }
     // a round boundary: bound the number of rounds (each issues >= 1 rollout)
     if (V.rounds_done > K.N + 1) {
         if (threadIdx.x == 0) { report_error(&V.err, ERR_ITER_BOUND); V.done = 1; }
-        set_conds(h_loop, h_round, 0, 0, use_handles);
+        set_conds(hs, 0, 0, use_handles);
         return;
     }
     ctl_round(K, V, c, sh);
@@ -473,7 +796,22 @@ ctl_kernel(StepPtrs c, cudaGraphConditionalHandle h_loop, cudaGraphConditionalHa
             if (c.q_status[c.act[i]] == ST_ACTIVE) c.q_status[c.act[i]] = ST_INCOMPLETE;
         if (threadIdx.x == 0) { V.live = 0; V.n_act = 0; }
     }
-    set_conds(h_loop, h_round, !done, !done && K.decode, use_handles);
+    set_conds(hs, !done, !done && K.decode, use_handles, !done && K.decode && V.n_fresh > 0);
+}
+
+// The next step's priors (warm-start carry, App. D): decayed evidence on top of the base
+// prior, a' = alpha0 + lambda (a - alpha0 + s), b' = beta0 + lambda (b - beta0 + n - s), with
+// (a, b) the prior this step used (the base prior unless warm).
+static __global__ void carry_prior_kernel(const StepPtrs c, double lambda, double *a_next, double *b_next) {
+    const StepConst &K = *c.kc;
+    for (int q = blockIdx.x * blockDim.x + threadIdx.x; q < K.P; q += gridDim.x * blockDim.x) {
+        const double a0 = K.a0, b0 = K.b0;
+        const double a = K.warm ? c.q_pa[q] : a0, b = K.warm ? c.q_pb[q] : b0;
+        const int n = c.q_n[q], s = c.q_s[q];
+        // rounded operation by operation (no contraction), as the formula reads
+        a_next[q] = __dadd_rn(a0, __dmul_rn(lambda, __dadd_rn(__dsub_rn(a, a0), (double)s)));
+        b_next[q] = __dadd_rn(b0, __dmul_rn(lambda, __dadd_rn(__dsub_rn(b, b0), (double)(n - s))));
+    }
 }
 
 // Reset the step state and build the decision tables (one CTA).
@@ -491,12 +829,19 @@ static __global__ void __launch_bounds__(kCtlThreads, 1) ctl_init_kernel(StepPtr
     ctl_build_tables(K, c);
     // every private KV block free (popped from the top: ids n_shared, n_shared + 1, .. first)
     for (int i = threadIdx.x; i < c.n_priv; i += kCtlThreads) c.blk_free[i] = c.n_shared + c.n_priv - 1 - i;
+    if (K.decode) {  // the asynchronous schedule's free rollout and prompt slots, batches in flight
+        for (int i = threadIdx.x; i < c.max_seqs; i += kCtlThreads) c.slot_free[i] = c.max_seqs - 1 - i;
+        for (int i = threadIdx.x; i < c.max_active; i += kCtlThreads) c.pslot_free[i] = c.max_active - 1 - i;
+        for (int q = threadIdx.x; q < K.P; q += kCtlThreads) c.q_inflight[q] = 0;
+    }
     if (threadIdx.x == 0) {
         StepVars z;
         memset(&z, 0, sizeof(z));
         z.round = -1;
         z.kt0 = ~0ull;
         z.blk_top = z.blk_low = c.n_priv;
+        z.slot_top = c.max_seqs;
+        z.pslot_top = c.max_active;
         V = z;
     }
 }

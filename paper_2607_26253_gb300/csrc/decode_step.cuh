@@ -1381,16 +1381,17 @@ static __global__ void block_weights_kernel(const uint16_t *src, uint8_t *dst, i
     }
 }
 
-// Round start of the paged KV cache, from the prefill's row-major prompt KV ([2][n_kv][cap_p]
+// KV set-up of the rollouts that join, from the prefill's row-major prompt KV ([2][n_kv][cap_p]
 // [hd] per prompt slot and layer, positions < Lp - 1): (a) every fresh prompt's full blocks
-// (positions < nsh * 128), which its rollouts share; (b) every live rollout's private block
-// holding position Lp - 1, filled with the prompt's tail positions nsh * 128 .. Lp - 2.  One
-// thread per K granule (8 dims of a position) or V granule (8 positions of a dim).
+// (positions < nsh * 128), which its rollouts share; (b) every new rollout's private block
+// holding position Lp - 1 (slots new_slots[0 .. n_new)), filled with the prompt's tail positions
+// nsh * 128 .. Lp - 2.  One thread per K granule (8 dims of a position) or V granule (8
+// positions of a dim).
 static __global__ void prompt_blocks_kernel(const uint16_t *pkv, uint8_t *kv, const StepPtrs c, int layers, int n_kv,
                                             int hd, int cap_p, int64_t kv_layer, int max_active) {
     pdl_wait_prior_grids();
     pdl_allow_dependents();
-    const int live = c.v->live, n_fresh = c.v->n_fresh;
+    const int n_new = c.v->n_new, n_fresh = c.v->n_fresh;
     const int Lp = c.kc->Lp, Lpre = Lp - 1;
     const int nsh = shared_blocks(Lp, kKVPos);
     const int gk = hd / 8;
@@ -1399,7 +1400,7 @@ static __global__ void prompt_blocks_kernel(const uint16_t *pkv, uint8_t *kv, co
     const int64_t per_a = (int64_t)na * gk + (int64_t)(na / 8) * hd;
     const int64_t per_b = (int64_t)nt * gk + (int64_t)((nt + 7) / 8) * hd;
     const int64_t tot_a = (int64_t)n_fresh * layers * n_kv * per_a;
-    const int64_t total = tot_a + (int64_t)live * layers * n_kv * per_b;
+    const int64_t total = tot_a + (int64_t)n_new * layers * n_kv * per_b;
     for (int64_t e = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; e < total; e += (int64_t)gridDim.x * blockDim.x) {
         int64_t rem;
         int owner, npos, p0;  // owner: fresh prompt f or rollout slot s; positions [p0, p0 + npos)
@@ -1423,7 +1424,8 @@ static __global__ void prompt_blocks_kernel(const uint16_t *pkv, uint8_t *kv, co
         const int kvh = (int)(rem / per);
         rem -= (int64_t)kvh * per;
         const bool shared = e < tot_a;
-        const int ps = shared ? c.fresh_pslot[owner] : c.seq_pslot[owner];
+        const int slot = shared ? 0 : c.new_slots[owner];
+        const int ps = shared ? c.fresh_pslot[owner] : c.seq_pslot[slot];
         const uint16_t *kplane = pkv + (((int64_t)l * max_active + ps) * 2 * n_kv + kvh) * cap_p * hd;
         const uint16_t *vplane = kplane + (int64_t)n_kv * cap_p * hd;
         const int nk = npos * gk;
@@ -1438,7 +1440,7 @@ static __global__ void prompt_blocks_kernel(const uint16_t *pkv, uint8_t *kv, co
             dd = (int)(rem - (int64_t)((pos - p0) / 8) * hd);
         }
         const int b = pos / kKVPos;
-        const int blk = shared ? ps * c.nsh_max + b : c.blk_tab[(int64_t)owner * c.nblk_max + b];
+        const int blk = shared ? ps * c.nsh_max + b : c.blk_tab[(int64_t)slot * c.nblk_max + b];
         uint8_t *dst = kv + l * kv_layer + ((int64_t)blk * n_kv + kvh) * kKVBlockBytes;
         if (isk) {
             const uint4 v = *reinterpret_cast<const uint4 *>(kplane + (int64_t)pos * hd + dd);

@@ -107,6 +107,7 @@ struct sara_handle {
     int64_t *uid_dev = nullptr;
     size_t forced_cap = 0;
     uint64_t *stamps = nullptr;  // profiling builds: per-CTA phase timestamps of GEMM launches
+    double *prior_next = nullptr;  // [2][max_prompts] warm-start priors of the next step
     // failure limits (sara_set_limits): bounded-wait limit, loop bound, stalled phase counter
     uint64_t wait_ns = 0;
     int32_t max_iters = 0, stall_idx = -1;
@@ -412,51 +413,53 @@ void enqueue_prompt_blocks(sara_handle &h, cudaStream_t s, bool pdl, const StepP
            m.layers, m.n_kv_heads, m.head_dim, h.cap_p, h.kv_seq_layer, m.max_active);
 }
 
-void enqueue_round_start(sara_handle &h, cudaStream_t s, bool pdl) {
-    enqueue_prefill(h, s, pdl);
-    enqueue_prompt_blocks(h, s, pdl, h.ptrs);
-}
 
 // ------------------------------------------------------------------------ graph
 void build_graph(sara_handle &h) {
     const bool pdl = h.use_pdl;
     CK(cudaGraphCreate(&h.graph, 0));
-    cudaGraphConditionalHandle h_loop;
-    CK(cudaGraphConditionalHandleCreate(&h_loop, h.graph, 1, cudaGraphCondAssignDefault));
+    CondHandles hs{};
+    CK(cudaGraphConditionalHandleCreate(&hs.h[0], h.graph, 1, cudaGraphCondAssignDefault));
     cudaGraphNodeParams wp{};
     wp.type = cudaGraphNodeTypeConditional;
-    wp.conditional.handle = h_loop;
+    wp.conditional.handle = hs.h[0];
     wp.conditional.type = cudaGraphCondTypeWhile;
     wp.conditional.size = 1;
     cudaGraphNode_t wnode;
     CK(cudaGraphAddNode(&wnode, h.graph, nullptr, nullptr, 0, &wp));
     cudaGraph_t body = wp.conditional.phGraph_out[0];
-    cudaGraphConditionalHandle h_round = 0;
-    if (h.has_model) CK(cudaGraphConditionalHandleCreate(&h_round, body, 0, cudaGraphCondAssignDefault));
-
+    if (h.has_model) {
+        CK(cudaGraphConditionalHandleCreate(&hs.h[1], body, 0, cudaGraphCondAssignDefault));
+        CK(cudaGraphConditionalHandleCreate(&hs.h[2], body, 0, cudaGraphCondAssignDefault));
+    }
     cudaStream_t cs = h.cap_stream;
     CK(cudaStreamBeginCaptureToGraph(cs, body, nullptr, nullptr, 0, cudaStreamCaptureModeRelaxed));
-    launch(cs, false, dim3(1), dim3(kCtlThreads), 0, ctl_kernel, h.ptrs, h_loop, h_round, h.has_model ? 3 : 1);
+    launch(cs, false, dim3(1), dim3(kCtlThreads), 0, ctl_kernel, h.ptrs, hs, h.has_model ? 3 : 1);
     if (h.has_model) {
-        cudaStreamCaptureStatus st;
-        cudaGraph_t capg;
-        const cudaGraphNode_t *deps = nullptr;
-        size_t ndeps = 0;
-        CK(cudaStreamGetCaptureInfo(cs, &st, nullptr, &capg, &deps, nullptr, &ndeps));
-        std::vector<cudaGraphNode_t> dv(deps, deps + ndeps);
-        cudaGraphNodeParams ip{};
-        ip.type = cudaGraphNodeTypeConditional;
-        ip.conditional.handle = h_round;
-        ip.conditional.type = cudaGraphCondTypeIf;
-        ip.conditional.size = 1;
-        cudaGraphNode_t inode;
-        CK(cudaGraphAddNode(&inode, capg, dv.data(), nullptr, dv.size(), &ip));
-        CK(cudaStreamUpdateCaptureDependencies(cs, &inode, nullptr, 1, cudaStreamSetCaptureDependencies));
-        cudaGraph_t ibody = ip.conditional.phGraph_out[0];
-        CK(cudaStreamBeginCaptureToGraph(h.cap_stream2, ibody, nullptr, nullptr, 0, cudaStreamCaptureModeRelaxed));
-        enqueue_round_start(h, h.cap_stream2, pdl);
-        cudaGraph_t ib2;
-        CK(cudaStreamEndCapture(h.cap_stream2, &ib2));
+        // IF(fresh prompts) { prefill }, then IF(new rollouts) { KV blocks of the new rollouts }
+        auto add_if = [&](cudaGraphConditionalHandle hc, const std::function<void(cudaStream_t)> &fill) {
+            cudaStreamCaptureStatus st;
+            cudaGraph_t capg;
+            const cudaGraphNode_t *deps = nullptr;
+            size_t ndeps = 0;
+            CK(cudaStreamGetCaptureInfo(cs, &st, nullptr, &capg, &deps, nullptr, &ndeps));
+            std::vector<cudaGraphNode_t> dv(deps, deps + ndeps);
+            cudaGraphNodeParams ip{};
+            ip.type = cudaGraphNodeTypeConditional;
+            ip.conditional.handle = hc;
+            ip.conditional.type = cudaGraphCondTypeIf;
+            ip.conditional.size = 1;
+            cudaGraphNode_t inode;
+            CK(cudaGraphAddNode(&inode, capg, dv.data(), nullptr, dv.size(), &ip));
+            CK(cudaStreamUpdateCaptureDependencies(cs, &inode, nullptr, 1, cudaStreamSetCaptureDependencies));
+            cudaGraph_t ibody = ip.conditional.phGraph_out[0];
+            CK(cudaStreamBeginCaptureToGraph(h.cap_stream2, ibody, nullptr, nullptr, 0, cudaStreamCaptureModeRelaxed));
+            fill(h.cap_stream2);
+            cudaGraph_t ib2;
+            CK(cudaStreamEndCapture(h.cap_stream2, &ib2));
+        };
+        add_if(hs.h[2], [&](cudaStream_t st) { enqueue_prefill(h, st, pdl); });
+        add_if(hs.h[1], [&](cudaStream_t st) { enqueue_prompt_blocks(h, st, pdl, h.ptrs); });
         enqueue_decode_step(h, cs);
     }
     cudaGraph_t b2;
@@ -466,17 +469,20 @@ void build_graph(sara_handle &h) {
 
 // Host-driven loop (debugging, SARA_GRAPH=0): the same kernels as the graph body, one
 // iteration at a time, with the round-start branch decided on the host.
-void run_host_loop(sara_handle &h) {
+void run_host_loop(sara_handle &h, int schedule) {
     cudaStream_t s = h.stream;
     StepVars v{};
     for (;;) {
-        launch(s, false, dim3(1), dim3(kCtlThreads), 0, ctl_kernel, h.ptrs, (cudaGraphConditionalHandle)0,
-               (cudaGraphConditionalHandle)0, 0);
+        launch(s, false, dim3(1), dim3(kCtlThreads), 0, ctl_kernel, h.ptrs, CondHandles{}, 0);
         CK(cudaMemcpyAsync(&v, h.vars, sizeof(v), cudaMemcpyDeviceToHost, s));
         CK(cudaStreamSynchronize(s));
         if (v.done || v.err) break;
         if (!h.has_model) continue;
-        if (v.round_steps == 0 && v.live > 0) enqueue_round_start(h, s, h.use_pdl);
+        const bool joins = schedule != 0 ? v.n_new > 0 : (v.round_steps == 0 && v.live > 0);
+        if (joins) {
+            if (v.n_fresh > 0) enqueue_prefill(h, s, h.use_pdl);
+            enqueue_prompt_blocks(h, s, h.use_pdl, h.ptrs);
+        }
         enqueue_decode_step(h, s);
     }
 }
@@ -681,6 +687,10 @@ void create_impl(sara_handle &h, const sara_model_cfg *cfgp, const sara_weights 
     c.p_len = h.p_len;
     c.q_status = h.mem.alloc<uint8_t>(P);
     c.q_n = h.mem.alloc<uint8_t>(P);
+    c.q_pa = h.mem.alloc<double>(P);
+    c.q_pb = h.mem.alloc<double>(P);
+    c.q_key = h.mem.alloc<double>((size_t)Bc + 1);
+    h.prior_next = h.mem.alloc<double>((size_t)2 * P);
     c.q_s = h.mem.alloc<uint8_t>(P);
     c.q_round = h.mem.alloc<int16_t>(P);
     c.q_pslot = h.mem.alloc<int32_t>(P);
@@ -734,6 +744,11 @@ void create_impl(sara_handle &h, const sara_model_cfg *cfgp, const sara_weights 
         c.n_priv = m.kv_blocks > 0 ? m.kv_blocks : S * ((m.max_gen_len + kKVPos - 1) / kKVPos + 2);
         c.blk_tab = h.mem.alloc<int32_t>((size_t)S * c.nblk_max);
         c.blk_free = h.mem.alloc<int32_t>((size_t)c.n_priv);
+        c.new_slots = h.mem.alloc<int32_t>((size_t)S);
+        c.q_inflight = h.mem.alloc<int32_t>((size_t)P);
+        c.dec_list = h.mem.alloc<int32_t>((size_t)std::max(Bc, S) + 1);
+        c.slot_free = h.mem.alloc<int32_t>((size_t)S);
+        c.pslot_free = h.mem.alloc<int32_t>((size_t)Bc);
         h.kv_seq_layer = (int64_t)(c.n_shared + c.n_priv) * KVH * kKVBlockBytes;
         h.kv_pr_slot = 2LL * KVH * h.cap_p * hd;
         h.kv_pr_layer = h.kv_pr_slot * Bc;
@@ -801,8 +816,15 @@ void collect_impl(sara_handle &h, const sara_prompts *pr, int64_t N, int32_t k, 
     if (t->target_B < 1 || t->target_B > m.max_active) throw SaraError(SARA_EINVAL, "target_B out of range");
     if (P > 0 && (!pr->p_threshold || !pr->lengths)) throw SaraError(SARA_EINVAL, "p_threshold / lengths are NULL");
     if (t->schedule < 0 || t->schedule > 2) throw SaraError(SARA_EINVAL, "schedule must be 0, 1 or 2");
-    if (t->schedule != 0 && h.has_model)
-        throw SaraError(SARA_EINVAL, "the asynchronous schedule runs on controller-only handles");
+    const bool warm = pr->prior_a != nullptr || pr->prior_b != nullptr;
+    if (warm && (!pr->prior_a || !pr->prior_b)) throw SaraError(SARA_EINVAL, "prior_a and prior_b go together");
+    if (warm && t->schedule != 0) throw SaraError(SARA_EINVAL, "warm-start priors run with the round schedule");
+    if (!(t->decay >= 0.0 && t->decay <= 1.0)) throw SaraError(SARA_EINVAL, "decay must be in [0, 1]");
+    if (warm && !pr->on_device) {
+        for (int q = 0; q < P; ++q)
+            if (!(pr->prior_a[q] > 0.0 && pr->prior_b[q] > 0.0 && pr->prior_a[q] < 1e12 && pr->prior_b[q] < 1e12))
+                throw SaraError(SARA_EINVAL, "warm-start priors must be positive and finite");
+    }
     if (h.has_model) {
         if (Lp < 2 || Lp > m.max_prompt_len) throw SaraError(SARA_EINVAL, "prompt_len out of range");
         if (P > 0 && !pr->tokens) throw SaraError(SARA_EINVAL, "tokens are NULL");
@@ -833,18 +855,25 @@ void collect_impl(sara_handle &h, const sara_prompts *pr, int64_t N, int32_t k, 
     K.max_iters = h.max_iters;
     K.stall_plus1 = h.stall_idx + 1;
     K.wait_ns = (int64_t)h.wait_ns;
+    K.tau_f = (double)t->tau_num / (double)t->tau_den;
+    K.warm = warm ? 1 : 0;
+    K.schedule = t->schedule;
 
     CK(cudaMemcpyAsync(h.kc, &K, sizeof(K), cudaMemcpyHostToDevice, s));
     if (P > 0) {
         CK(cudaMemcpyAsync(h.p_thr, pr->p_threshold, (size_t)P * 8, kin, s));
         CK(cudaMemcpyAsync(h.p_len, pr->lengths, (size_t)P * k * 4, kin, s));
         if (h.has_model) CK(cudaMemcpyAsync(h.p_tok, pr->tokens, (size_t)P * Lp * 4, kin, s));
+        if (warm) {
+            CK(cudaMemcpyAsync(h.ptrs.q_pa, pr->prior_a, (size_t)P * 8, kin, s));
+            CK(cudaMemcpyAsync(h.ptrs.q_pb, pr->prior_b, (size_t)P * 8, kin, s));
+        }
     }
     // device time of the step: from here (inputs on the device) to the end of its last kernel
     CK(cudaEventRecord(h.ev0, s));
     if (h.has_model) reset_decode_state(h, s);
     launch(s, false, dim3(1), dim3(kCtlThreads), 0, ctl_init_kernel, h.ptrs);
-    if (t->schedule != 0) {  // asynchronous per-prompt schedule: one event-loop kernel
+    if (t->schedule != 0 && !h.has_model) {  // asynchronous schedule without decode: one event-loop kernel
         const int cap = std::min(m.max_active, kAsyncMaxInFlight);
         const size_t smem = (size_t)cap * sizeof(uint64_t);
         CK(cudaFuncSetAttribute(ctl_async_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem));
@@ -852,8 +881,11 @@ void collect_impl(sara_handle &h, const sara_prompts *pr, int64_t N, int32_t k, 
     } else if (h.use_graph) {
         CK(cudaGraphLaunch(h.exec, s));
     } else {
-        run_host_loop(h);
+        run_host_loop(h, t->schedule);
     }
+    if (P > 0 && (out->prior_a_next || out->prior_b_next))
+        launch(s, false, dim3((P + 255) / 256), dim3(256), 0, carry_prior_kernel, h.ptrs, t->decay, h.prior_next,
+               h.prior_next + P);
     CK(cudaEventRecord(h.ev1, s));
     // results (one device -> host read per call)
     StepVars v{};
@@ -866,6 +898,8 @@ void collect_impl(sara_handle &h, const sara_prompts *pr, int64_t N, int32_t k, 
         if (out->n) CK(cudaMemcpyAsync(out->n, h.ptrs.q_n, P, kout, s));
         if (out->s) CK(cudaMemcpyAsync(out->s, h.ptrs.q_s, P, kout, s));
         if (out->decided_round) CK(cudaMemcpyAsync(out->decided_round, h.ptrs.q_round, (size_t)P * 2, kout, s));
+        if (out->prior_a_next) CK(cudaMemcpyAsync(out->prior_a_next, h.prior_next, (size_t)P * 8, kout, s));
+        if (out->prior_b_next) CK(cudaMemcpyAsync(out->prior_b_next, h.prior_next + P, (size_t)P * 8, kout, s));
         if (out->tokens && h.has_model)
             CK(cudaMemcpyAsync(out->tokens, h.gen_tok, (size_t)P * k * m.max_gen_len * 4, kout, s));
     }

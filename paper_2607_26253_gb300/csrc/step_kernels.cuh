@@ -127,6 +127,7 @@ static __global__ void __launch_bounds__(256) sample_finish_kernel(StepPtrs c, i
     // bookkeeping over the live rows (several passes of 256)
     int out = 0;
     int top = V.blk_top, low = V.blk_low;  // the KV block free stack (same value in every thread)
+    int stop = V.slot_top;                 // the free rollout slots (asynchronous schedule)
     for (int base = 0; base < live; base += 256) {
         const int i = base + tid;
         int keep = 0, slot = 0, gen = 0, next_tok = 0;
@@ -167,6 +168,19 @@ static __global__ void __launch_bounds__(256) sample_finish_kernel(StepPtrs c, i
         }
         top = max(0, top - atot);
         low = min(low, top);
+        if (K.schedule != 0) {
+            // asynchronous schedule: a finished rollout returns its slot, and the prompt whose
+            // batch it completes is listed for the decisions at this step boundary
+            const int fin = (i < live && !keep) ? 1 : 0;
+            int stot;
+            const int soff = scan256(fin, stot, warp_tot);
+            if (fin) {
+                c.slot_free[stop + soff] = slot;
+                const int q = c.seq_q[slot];
+                if (atomicSub(&c.q_inflight[q], 1) == 1) c.dec_list[atomicAdd(&V.n_dec, 1)] = q;
+            }
+            stop += stot;
+        }
         // stable in-place compaction: a kept row lands at or before its own index
         int tot;
         const int before = scan256(keep, tot, warp_tot);
@@ -213,6 +227,7 @@ static __global__ void __launch_bounds__(256) sample_finish_kernel(StepPtrs c, i
         V.round_steps += 1;
         V.blk_top = top;
         V.blk_low = low;
+        V.slot_top = stop;
     }
 }
 
@@ -233,6 +248,7 @@ static __global__ void __launch_bounds__(kCtlThreads, 1) teacher_setup_kernel(St
         for (int j = 0; j < nsh; ++j) bt[j] = r * c.nsh_max + j;
         bt[nsh] = r < c.n_priv ? c.blk_free[c.n_priv - 1 - r] : c.n_shared;  // (n > n_priv: an error)
         c.fresh_pslot[r] = r;
+        c.new_slots[r] = r;
         c.seq_q[r] = r;
         c.seq_j[r] = 0;
         c.seq_len[r] = K.T_forced;
@@ -266,6 +282,7 @@ static __global__ void __launch_bounds__(kCtlThreads, 1) teacher_setup_kernel(St
         z.round_maxL = K.T_forced;
         z.kt0 = ~0ull;
         z.blk_top = z.blk_low = c.n_priv - n;
+        z.n_new = n;
         if (n > c.n_priv) z.err |= ERR_CAPACITY;
         V = z;
     }

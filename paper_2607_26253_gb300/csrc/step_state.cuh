@@ -27,6 +27,10 @@ struct StepConst {
     int32_t stall_plus1;  // test hook: 1 + the decode-step phase counter whose waits never
                           // complete (0: none)
     int64_t wait_ns;      // limit of the decode step's bounded waits (0: the built-in 2 s)
+    double tau_f;         // tau_num / tau_den (the warm-start predictor compares in fp64)
+    int32_t warm;         // 1: per-prompt real priors q_pa / q_pb (warm-start) decide
+    int32_t schedule;     // 0: synchronised rounds; 1 / 2: asynchronous per prompt (2: with the
+                          // budget reserve), decided and refilled at every decode step
 };
 
 // Scalar progress of the step (device, reset by the init kernel).
@@ -51,6 +55,13 @@ struct StepVars {
     int64_t kernel_ns;
     // paged KV cache: free private blocks on the stack, and the fewest ever free
     int32_t blk_top, blk_low;
+    // new rollouts of this loop iteration (their slots in new_slots), for the KV set-up
+    int32_t n_new;
+    // asynchronous schedule: prompts whose batch finished in the last decode step (dec_list),
+    // decision events so far, prompts with a batch in flight, the stop flag, free rollout slots
+    // and prompt slots on their stacks, the budget held back for prompts in flight (reserve)
+    int32_t n_dec, events, in_flight, stopped, slot_top, pslot_top;
+    int64_t resv;
 };
 
 // KV blocks per decode attention split: the smallest span that leaves at most `slots` split
@@ -76,6 +87,11 @@ struct StepPtrs {
     int32_t *act, *act_tmp, *iss_q, *iss_c, *fresh_pslot;
     // exact decision / priority tables
     uint8_t *dec_tab, *rank_tab;
+    // warm-start: per-prompt real Beta prior (used when StepConst::warm, else every prompt has
+    // the integer prior of StepConst and the exact tables decide); p_eff keys of the continuing
+    // prompts
+    double *q_pa, *q_pb;
+    double *q_key;
     // sequences (slots)
     int32_t *seq_q, *seq_j, *seq_len, *seq_gen, *seq_pslot;
     int64_t *seq_uid;
@@ -103,6 +119,12 @@ struct StepPtrs {
     int32_t *blk_tab;          // [max_seqs][nblk_max] block id of rollout slot s's block b
     int32_t *blk_free;         // [n_priv]
     int32_t nblk_max, nsh_max, n_shared, n_priv;
+    int32_t *new_slots;        // [max_seqs] slots of the rollouts that start at the next step
+    // asynchronous schedule
+    int32_t *q_inflight;       // [P] rollouts of the prompt's batch still decoding
+    int32_t *dec_list;         // [max_active] prompts to decide at this step boundary
+    int32_t *slot_free;        // [max_seqs] free rollout slots
+    int32_t *pslot_free;       // [max_active] free prompt slots
 };
 
 // Full prompt blocks (shared by a prompt's rollouts) when the prefill writes positions

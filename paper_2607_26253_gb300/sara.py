@@ -44,13 +44,14 @@ class Weights(ctypes.Structure):
 
 class Prompts(ctypes.Structure):
     _fields_ = [("n_prompts", ctypes.c_int32), ("prompt_len", ctypes.c_int32), ("tokens", c_p),
-                ("p_threshold", c_p), ("lengths", c_p), ("on_device", ctypes.c_int32)]
+                ("p_threshold", c_p), ("lengths", c_p), ("on_device", ctypes.c_int32), ("prior_a", c_p),
+                ("prior_b", c_p)]
 
 
 class Thresholds(ctypes.Structure):
     _fields_ = [("tau_num", ctypes.c_int64), ("tau_den", ctypes.c_int64), ("commit_min", ctypes.c_int32),
                 ("alpha0", ctypes.c_int32), ("beta0", ctypes.c_int32), ("target_B", ctypes.c_int32),
-                ("sample_seed", ctypes.c_uint64), ("schedule", ctypes.c_int32)]
+                ("sample_seed", ctypes.c_uint64), ("schedule", ctypes.c_int32), ("decay", ctypes.c_double)]
 
 
 class Result(ctypes.Structure):
@@ -59,7 +60,8 @@ class Result(ctypes.Structure):
                 ("prefill_tokens", ctypes.c_int64), ("decode_steps", ctypes.c_int64), ("rounds", ctypes.c_int64),
                 ("committed", ctypes.c_int64), ("abandoned", ctypes.c_int64), ("incomplete", ctypes.c_int64),
                 ("prompts_drawn", ctypes.c_int64), ("device_ms", ctypes.c_double),
-                ("decode_kernel_ms", ctypes.c_double), ("kv_blocks_peak", ctypes.c_int64)]
+                ("decode_kernel_ms", ctypes.c_double), ("kv_blocks_peak", ctypes.c_int64),
+                ("prior_a_next", c_p), ("prior_b_next", c_p)]
 
 
 class Limits(ctypes.Structure):
@@ -176,6 +178,7 @@ class StepOutput:
     device_ms: float          # the step's kernels, inputs already on the device
     decode_kernel_ms: float   # summed decode-step kernel launches (device clock)
     kv_blocks_peak: int       # most private KV blocks in use at once
+    prior_next: tuple | None = None  # (a, b) warm-start priors of the next step, if requested
 
 
 class Handle:
@@ -224,17 +227,22 @@ class Handle:
     def collect_step(self, *, thresholds, lengths, N: int, k: int, n0: int, tau, target_B: int,
                      reward_seed: int, tokens=None, prompt_len: int | None = None, commit_min: int = 0,
                      prior=(1, 1), sample_seed: int = 0, want_tokens: bool = False,
-                     outputs_on_device: bool = False, schedule: int = 0, outputs: dict | None = None) -> StepOutput:
+                     outputs_on_device: bool = False, schedule: int = 0, outputs: dict | None = None,
+                     prior_a=None, prior_b=None, decay: float = 0.0, want_next_prior: bool = False) -> StepOutput:
         """One rollout-collection step (Algorithm 1).  Inputs are numpy arrays (host) or torch
         CUDA tensors (device); outputs are numpy arrays, or torch CUDA tensors when
         outputs_on_device.  `outputs` may hold preallocated arrays (keys status, n, s,
-        decided_round and, with want_tokens, tokens [P, k, max_gen_len]) of the same kind."""
+        decided_round and, with want_tokens, tokens [P, k, max_gen_len]) of the same kind.
+        prior_a / prior_b: per-prompt warm-start priors (float64 [P], same kind as the inputs);
+        want_next_prior: also return the next step's priors carried with `decay`."""
         P = int(thresholds.shape[0])
         on_dev = not isinstance(thresholds, np.ndarray)
         Lp = int(tokens.shape[1]) if tokens is not None else (prompt_len or 1)
-        pr = Prompts(P, Lp, _ptr(tokens), _ptr(thresholds), _ptr(lengths), 1 if on_dev else 0)
+        pr = Prompts(P, Lp, _ptr(tokens), _ptr(thresholds), _ptr(lengths), 1 if on_dev else 0, _ptr(prior_a),
+                     _ptr(prior_b))
         t = tau_fraction(tau)
-        th = Thresholds(t.numerator, t.denominator, commit_min, prior[0], prior[1], target_B, sample_seed, schedule)
+        th = Thresholds(t.numerator, t.denominator, commit_min, prior[0], prior[1], target_B, sample_seed, schedule,
+                        float(decay))
         if outputs is not None:
             status, n, s, rnd = outputs["status"], outputs["n"], outputs["s"], outputs["decided_round"]
             toks = outputs["tokens"] if want_tokens else None
@@ -252,12 +260,21 @@ class Handle:
             s = np.zeros(P, np.uint8)
             rnd = np.zeros(P, np.int16)
             toks = np.empty((P, k, self.cfg.max_gen_len), np.int32) if want_tokens else None
+        pan = pbn = None
+        if want_next_prior:
+            if outputs_on_device:
+                import torch
+                pan = torch.empty(P, dtype=torch.float64, device="cuda")
+                pbn = torch.empty(P, dtype=torch.float64, device="cuda")
+            else:
+                pan, pbn = np.empty(P, np.float64), np.empty(P, np.float64)
         res = Result(_ptr(status), _ptr(n), _ptr(s), _ptr(rnd), _ptr(toks), 1 if outputs_on_device else 0)
+        res.prior_a_next, res.prior_b_next = _ptr(pan), _ptr(pbn)
         _check(load().sara_collect_step(self._h, ctypes.byref(pr), N, k, n0, ctypes.byref(th), reward_seed,
                                         ctypes.byref(res)), self._h)
         counters = {name: int(getattr(res, name)) for name in COUNTERS}
         return StepOutput(status, n, s, rnd, toks, counters, float(res.device_ms), float(res.decode_kernel_ms),
-                          int(res.kv_blocks_peak))
+                          int(res.kv_blocks_peak), (pan, pbn) if want_next_prior else None)
 
     def set_limits(self, wait_limit_ns: int = 0, max_loop_iters: int = 0, stall_phase: int = -1):
         """Failure limits of later calls (see sara_set_limits); no arguments restores the defaults."""

@@ -200,3 +200,68 @@ def test_full_shape_long_context_teacher_forced(long_case, n):
             tok, margin = o2.sample_token(logits[i, t], w.sample_seed, int(uids[i]), t)
             if margin > 1e-4:
                 assert sampled[i, t] == tok, (i, t)
+
+
+# The asynchronous per-prompt schedule on the decode engine (no round barrier): every prompt is
+# decided at the end of the decode step in which its batch finishes, and the rollouts it issues
+# join the live rows at the next step.  The schedule must equal the asynchronous oracle's bit
+# for bit (decision events in place of rounds) and every decoded token the float64 oracle's
+# Gumbel-max draw up to the first near-tie.
+def _assert_async_schedule(out, ref):
+    assert np.array_equal(out.status, ref.status)
+    assert np.array_equal(out.n, ref.n) and np.array_equal(out.s, ref.s)
+    assert np.array_equal(out.decided_round.astype(np.int32), np.minimum(ref.decided_event, 32767))
+    c = ref.counters
+    for key, v in (("rollouts", c["rollouts"]), ("gen_tokens", c["gen_tokens"]), ("decode_steps", c["decode_steps"]),
+                   ("rounds", c["events"]), ("committed", c["committed"]), ("abandoned", c["abandoned"]),
+                   ("incomplete", c["incomplete"]), ("prompts_drawn", c["prompts_drawn"]),
+                   ("prefill_tokens", c["prefill_tokens"])):
+        assert out.counters[key] == v, (key, out.counters[key], v)
+
+
+@pytest.mark.parametrize("schedule", [1, 2])
+def test_tiny_async_schedule_and_tokens(tiny, schedule):
+    from oracle import async_schedule as oa
+    w, weights, h = tiny
+    si = synth.step_inputs(w)
+    out = _run_step(h, w, si, want_tokens=True, schedule=schedule)
+    ref = oa.collect_workload(w, si, reserve=schedule == 2)
+    _assert_async_schedule(out, ref)
+    W = o2.Weights(w.model, weights)
+    compared = 0
+    for q in np.nonzero(ref.n)[0]:
+        for j in range(int(ref.n[q])):
+            L = int(si.lengths[q, j])
+            toks, margins, _ = o2.generate(W, si.tokens[q], L, w.sample_seed, o2.uid_of(int(q), j))
+            low = np.nonzero(margins < 1e-2)[0]
+            cut = int(low[0]) if low.size else L
+            assert np.array_equal(out.tokens[q, j, :cut], toks[:cut]), (q, j)
+            compared += cut
+    assert compared > 0.8 * out.counters["gen_tokens"]
+
+
+def test_tiny_async_other_seeds_and_the_round_schedule_after(tiny):
+    from oracle import async_schedule as oa
+    w0, _, h = tiny
+    for off in (100, 200):
+        for kw in ({}, {"commit_min": 4}, {"budget_N": 90}):
+            w = replace(w0.with_seed_offset(off), **kw)
+            si = synth.step_inputs(w)
+            for schedule in (1, 2):
+                _assert_async_schedule(_run_step(h, w, si, schedule=schedule),
+                                       oa.collect_workload(w, si, reserve=schedule == 2))
+            _assert_schedule(_run_step(h, w, si), oc.collect_workload(w, si))  # the same handle, rounds again
+
+
+def test_full_shape_async_step_1p5b(pkg):
+    from oracle import async_schedule as oa
+    w = synth.WORKLOADS["1.5b"]
+    weights = synth.model_weights(w.model, w.weight_seed)
+    si = synth.step_inputs(w)
+    with pkg.Handle(handle_cfg(w, pkg), weights) as h:
+        out = _run_step(h, w, si, want_tokens=True, schedule=2)
+    _assert_async_schedule(out, oa.collect_workload(w, si, reserve=True))
+    for q in np.nonzero(out.n)[0][:8]:
+        for j in range(int(out.n[q])):
+            t = out.tokens[q, j, :si.lengths[q, j]]
+            assert t.min() >= 0 and t.max() < w.model.vocab
