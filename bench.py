@@ -52,6 +52,9 @@ def parse():
     ap.add_argument("--warmup", type=int, default=3)
     ap.add_argument("--impl", default="mine", choices=["mine", "reference"])
     ap.add_argument("--workload", default="1.5b", choices=sorted(synth.WORKLOADS))
+    ap.add_argument("--schedule", type=int, default=0, choices=[0, 1, 2],
+                    help="0: Algorithm 1's synchronised rounds (the paper's method, the default); 1 / 2: the "
+                         "asynchronous per-prompt schedule without / with the budget reserve")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--kernel-profile", type=int, default=None, metavar="KERNEL",
                     help="profiling mode for ncu: launch one decode kernel (sara_profile ids; 0 = whole "
@@ -60,6 +63,9 @@ def parse():
     ap.add_argument("--iters", type=int, default=5, help="launches in --kernel-profile mode")
     ap.add_argument("--ctx", type=int, default=None, help="context length in --kernel-profile mode "
                     "(default: prompt length + 128)")
+    ap.add_argument("--controller", action="store_true",
+                    help="time the on-device controller alone (controller-only handles) over the sweep grid "
+                         "k x n0 x tau at P = 65,536: microseconds per round and decisions per second")
     ap.add_argument("--cpu-slice", action="store_true", help=argparse.SUPPRESS)  # child of the CPU baseline
     ap.add_argument("--slice-layers", type=int, default=None, help=argparse.SUPPRESS)
     return ap.parse_args()
@@ -318,7 +324,7 @@ def run_mine(args):
         return h.collect_step(thresholds=thr, lengths=lens, tokens=toks, N=wi.budget_N, k=wi.k, n0=wi.n0,
                               tau=wi.tau, target_B=wi.target_B, reward_seed=wi.reward_seed,
                               sample_seed=wi.sample_seed, commit_min=wi.commit_floor, prior=wi.prior,
-                              want_tokens=True, outputs=outs_host)
+                              want_tokens=True, outputs=outs_host, schedule=args.schedule)
 
     warm_s = []
     for i in range(args.warmup):
@@ -400,7 +406,9 @@ def run_mine(args):
         "vs_baseline": None,
         "dtype": "bf16",
         "data": "synthetic (random-init weights N(0,0.02), seeded prompts, rewards and lengths)",
-        "config": {"workload": w0.name, "global_batch": w0.target_B * world, "seq_len": w0.prompt_len,
+        "config": {"workload": w0.name + ("" if args.schedule == 0 else
+                                          f" [asynchronous schedule{' + reserve' if args.schedule == 2 else ''}]"),
+                   "global_batch": w0.target_B * world, "seq_len": w0.prompt_len,
                    "parallelism": f"replicas x{world} (prompt-stream shards)",
                    "l2": "inputs larger than L2 (3+ GB of weights streamed per decode step)"},
         "effective_groups_per_s": groups / (dev_ms * 1e-3),
@@ -429,9 +437,12 @@ def run_mine(args):
         "wall_s": round(time.time() - t_start, 1),
     }
     # kernels launched: per decode step the controller, the decode-step kernel and the
-    # sampling/bookkeeping kernel; per round start the prefill (embedding + 5 per layer but
-    # the last layer's 4) and the KV fan-out; per call the init kernel
+    # sampling/bookkeeping kernel; per round start (or, asynchronous, per decision event) at most
+    # the prefill (embedding + 5 per layer but the last layer's 4) and the KV set-up; per call
+    # the init kernel
     line["gpu_launches"] = int(3 * dsteps + rounds * (1 + 5 * m.layers - 4 + 1) + args.steps * world)
+    line["committed_per_step"] = groups / world / args.steps
+    line["kv_blocks_peak"] = max(o.kv_blocks_peak for o in outs)
     print(json.dumps(line), flush=True)
     if world > 1:
         dist.destroy_process_group()
@@ -474,6 +485,45 @@ def run_kernel_profile(args):
     with pkg.Handle(cfg, weights, stream=torch.cuda.current_stream()) as h:
         ms = h.profile(args.kernel_profile, args.rows, ctx, iters=args.iters)
     print(json.dumps({"kernel": args.kernel_profile, "rows": args.rows, "ctx": ctx, "ms_per_launch": ms}))
+
+
+# --------------------------------------------------------------------------------- controller
+def run_controller(args):
+    """The SARA controller kernel alone (Algorithm 1's rounds without decode) on the 63-point
+    sweep grid at P = 65,536, B = 8,192, N = 4P: per point the device time of the step (CUDA
+    events of the call, inputs in HBM), rounds, and decisions (one DECIDE per active prompt per
+    round: n_q - n0 + 1 for every drawn prompt)."""
+    import torch
+
+    import paper_2607_26253_gb300 as pkg
+    torch.cuda.set_device(0)
+    P, B = 65536, 8192
+    cfg = pkg.model_cfg(None, max_prompts=P, max_active=B, max_seqs=1, max_prompt_len=1, max_gen_len=1, max_k=16)
+    rows = []
+    with pkg.Handle(cfg, stream=torch.cuda.current_stream()) as h:
+        for k in synth.SWEEP_K:
+            for n0 in synth.SWEEP_N0:
+                for tau in synth.SWEEP_TAU:
+                    w = synth.sweep_workload(k, n0, tau)
+                    si = synth.step_inputs(w)
+                    thr = torch.from_numpy(si.thresholds.view(np.int64)).cuda()
+                    lens = torch.from_numpy(si.lengths).cuda()
+                    kw = dict(thresholds=thr, lengths=lens, N=w.budget_N, k=k, n0=n0, tau=tau, target_B=B,
+                              reward_seed=w.reward_seed)
+                    h.collect_step(**kw)  # warm-up
+                    o = h.collect_step(**kw)
+                    n = o.n.astype(np.int64)
+                    dec = int((n[n > 0] - n0 + 1).sum())
+                    rows.append((k, n0, tau, o.device_ms, o.counters["rounds"], dec))
+    ms = np.array([r[3] for r in rows])
+    rounds = np.array([r[4] for r in rows])
+    dec = np.array([r[5] for r in rows])
+    print(json.dumps({"metric": "controller microseconds per round / decisions per second (sweep, P = 65,536)",
+                      "points": len(rows), "us_per_round_median": float(np.median(1e3 * ms / rounds)),
+                      "us_per_round_max": float(np.max(1e3 * ms / rounds)),
+                      "decisions_per_s_median": float(np.median(dec / (ms * 1e-3))),
+                      "k8_n0_2_tau045": next({"ms": r[3], "rounds": r[4], "decisions": r[5]} for r in rows
+                                            if r[0] == 8 and r[1] == 2 and abs(r[2] - 0.45) < 1e-9)}))
 
 
 # --------------------------------------------------------------------------------- reference arm
@@ -522,6 +572,8 @@ if __name__ == "__main__":
         cpu_slice_child(a)
     elif a.kernel_profile is not None:
         run_kernel_profile(a)
+    elif a.controller:
+        run_controller(a)
     elif a.impl == "reference":
         run_reference(a)
     else:
