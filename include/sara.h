@@ -40,10 +40,11 @@ extern "C" {
 
 /* Layout version of the structs below.  Version 2 added sara_thresholds.schedule and decay,
  * sara_prompts.prior_a / prior_b, sara_model_cfg.kv_blocks, sara_result.decode_kernel_ms,
- * kv_blocks_peak and prior_a_next / prior_b_next, and sara_limits;
+ * kv_blocks_peak and prior_a_next / prior_b_next, and sara_limits; version 3
+ * sara_limits.eager_softmax;
  * a caller built against another version
  * must not pass its structs to this library (compare with sara_abi_version()). */
-#define SARA_ABI_VERSION 2
+#define SARA_ABI_VERSION 3
 
 #define SARA_OK 0
 #define SARA_EINVAL (-1)   /* an argument is out of range; nothing was launched */
@@ -237,12 +238,21 @@ SARA_API int sara_profile(sara_handle *h, int32_t kernel, int32_t rows, int32_t 
  *   stall_phase:    -1, or a phase-counter index of the decode-step kernel (0 = embedding,
  *                   1 + 9 l + j = phase j of layer l) whose waits are made to wait for a value
  *                   no launch reaches: they time out after wait_limit_ns.
+ *   eager_softmax:  the decode attention's online softmax (Sec. 2's rollout model: causal
+ *                   attention over the KV cache) takes each KV block's probabilities against
+ *                   a running maximum.  0 (default): the maximum is re-based only when a score
+ *                   exceeds it by more than 2^8, so probabilities stay <= 256 and most blocks
+ *                   skip the block maximum and the output rescale.  1: re-based at every block
+ *                   that raises it (probabilities <= 1).  The same softmax up to rounding; the
+ *                   switch exists to test the rescale path.
  * The handle stays usable after a call that failed this way.  SARA_EINVAL if out of range.
  */
 typedef struct {
     int64_t wait_limit_ns;
     int32_t max_loop_iters;
     int32_t stall_phase;
+    int32_t eager_softmax;
+    int32_t reserved;        /* must be 0 */
 } sara_limits;
 SARA_API int sara_set_limits(sara_handle *h, const sara_limits *limits);
 

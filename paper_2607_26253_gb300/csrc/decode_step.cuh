@@ -21,7 +21,8 @@
 //
 // Warp roles (352 threads, 11 warps):
 //   warp 0   W producer: bulk copies of pre-swizzled weight tiles and KV blocks
-//   warp 1   tcgen05 issuer and tensor-memory owner
+//   warp 1   tcgen05 issuer and tensor-memory owner; hands the attention phase's KV tiles
+//            to the compute warp group that runs their unit
 //   warp 2   X producer: activation chunks, after the phase they come from has completed
 //   warps 3..10  compute: GEMM epilogues, attention softmax / merge, residual + RMSNorm +
 //                SwiGLU finalisation, embedding, logits
@@ -30,8 +31,10 @@
 //   0 QKV   x_g W_qkv^T -> partials        (a subset of the CTAs: few tiles)
 //   1 FIN_Q q, k, v = RMSNorm scale + RoPE of the summed partials, fp16, once per row; the
 //           new k, v appended to the KV cache
-//   2 ATT   softmax(q K^T) V on the tensor cores, 128-position KV blocks, online softmax
-//           over a split's blocks; the last split of a row to finish merges the splits
+//   2 ATT   softmax(q K^T) V, 128-position KV blocks, online softmax over a split's blocks
+//           with warp-level MMAs (mma.sync: N = 8 heads, operands and accumulators in
+//           registers; the tcgen05 path's issue / commit / tensor-memory round trips cost more
+//           than these products); the last split of a row to finish merges the splits
 //   3 O     att W_o^T -> partials           (a subset of the CTAs)
 //   4 FIN_O x += sum; x_g = x * g_mlp (bf16 hi/lo, blocked); per-row sum of squares
 //   5 GU    x_g W_gu^T -> partials          (gate / up interleaved in 64-row blocks)
@@ -74,8 +77,14 @@ __device__ constexpr int kGemmPhases[4] = {kPhQKV, kPhO, kPhGU, kPhDown};
 constexpr int kSmallPhaseUnits = 2;   // QKV / O: units per participating CTA
 constexpr int kCntStride = 16;        // phase counters 128 bytes apart (one L2 line each)
 constexpr uint32_t kTmemCols = 512;
-constexpr uint32_t kTmemS = 256;  // attention scores, 2 buffers x 16 columns
-constexpr uint32_t kTmemO = 288;  // attention output, 2 buffers x 16 columns
+// Attention P tiles (per warp group, two buffers): [8 heads][128 positions] fp16, rows padded
+// to 272 bytes so the eight rows of an ldmatrix fall in distinct banks.
+constexpr int kAttPRow = 272;
+constexpr int kAttPBytes = 8 * kAttPRow;
+// Attention probabilities are taken against a running maximum that is re-based only when a
+// score exceeds it by more than this (log2 units): P <= 2^8 in fp16, and most blocks skip the
+// block maximum and the rescale of the output.
+constexpr float kSoftmaxHeadroom = 8.f;
 
 struct MegaParams {
     int layers, d, H, KVH, hd, F, V, Gq, nqkv;
@@ -138,12 +147,13 @@ struct MegaParams {
 
 struct MegaSmem {
     uint64_t wfull[kWSlots], wempty[kWSlots];
+    uint64_t kvready[2][kWSlots];  // attention: ring slot s holds warp group g's next KV tile
     uint64_t xfull[kMaxXStages], xempty[kMaxXStages];
     uint64_t acc_full[2], acc_empty[2];
-    uint64_t q_ready[2], s_full[2], p_ready[2], o_full[2];
     uint64_t drain;
     unsigned long long target;  // counter value meaning "every CTA of this launch arrived"
     uint64_t wait_ns;           // bounded-wait limit of this launch
+    float p_headroom;           // attention: log2 of how far P may exceed 1 before re-basing
     int stall_idx;              // test hook: the phase counter whose waits never complete (-1: none)
     uint32_t tmem_base;
     int abort;
@@ -418,10 +428,10 @@ __device__ __forceinline__ void mega_w_producer(const MegaParams &p, MegaSmem &S
             MEGA_STAMP(1 + kPhasesPerLayer * l + k, 2);
             if (k == 0 && l < p.layers && ok) {
                 // the attention phase's KV blocks follow the QKV weights in ring order: unit
-                // pairs (one unit per compute warp group), block by block, K then V^T of the
-                // pair's first unit, then of its second; each one ring entry (K: d < 64 |
-                // d >= 64 halves, V^T: positions < 64 | >= 64).  The block holding a row's
-                // new position is copied once the q / k / v phase has appended it to the cache.
+                // pairs (one unit per compute warp group), block by block, the K of the pair's
+                // units, then their V^T; each one ring entry (K: d < 64 | d >= 64 halves, V^T:
+                // positions < 64 | >= 64).  The block holding a row's new position is copied
+                // once the q / k / v phase has appended it to the cache.
                 int64_t a0, a1;
                 att_range(p, S.n_items, a0, a1);
                 const int span = S.att_span;
@@ -432,33 +442,38 @@ __device__ __forceinline__ void mega_w_producer(const MegaParams &p, MegaSmem &S
                     const AttUnit ub = two ? att_unit(p, a + 1, span) : ua;
                     const int nbb = two ? ub.nb : 0;
                     for (int j = 0; j < max(ua.nb, nbb) && ok; ++j) {
-                        for (int w = 0; w < 2 && ok; ++w) {
-                            const AttUnit &u = w ? ub : ua;
-                            if (j >= (w ? nbb : ua.nb)) continue;
-                            if (u.last && j == u.nb - 1 && !finq_seen) {
-                                const int fq = 1 + kPhasesPerLayer * l + kPhFinQ;
-                                if (!spin_counter(&p.cnt[fq * kCntStride], phase_target(p, S, fq), err, ab, lim)) {
-                                    ok = false;
-                                    break;
+                        for (int kv = 0; kv < 2 && ok; ++kv) {
+                            for (int w = 0; w < 2 && ok; ++w) {
+                                const AttUnit &u = w ? ub : ua;
+                                if (j >= (w ? nbb : ua.nb)) continue;
+                                if (kv == 0 && u.last && j == u.nb - 1 && !finq_seen) {
+                                    const int fq = 1 + kPhasesPerLayer * l + kPhFinQ;
+                                    if (!spin_counter(&p.cnt[fq * kCntStride], phase_target(p, S, fq), err, ab, lim)) {
+                                        ok = false;
+                                        break;
+                                    }
+                                    fence_proxy_async_global();
+                                    finq_seen = true;
                                 }
-                                fence_proxy_async_global();
-                                finq_seen = true;
+                                const uint8_t *blk = kv_block(p, S, l, u, (int)(a - a0) + w, j);
+                                const int nj = min(kKVPos, u.n - j * kKVPos);
+                                if (!acquire(wi)) { ok = false; break; }
+                                const int s = (int)(wi % nws);
+                                if (kv == 0) {
+                                    const uint32_t kb = (uint32_t)(((nj + 7) & ~7) * 128);
+                                    mbar_arrive_expect_tx(&S.wfull[s], p.hd > 64 ? 2 * kb : kb);
+                                    bulk_load(sW + (size_t)s * kSlotBytes, blk, kb, &S.wfull[s], pol);
+                                    if (p.hd > 64)
+                                        bulk_load(sW + (size_t)s * kSlotBytes + 16384, blk + 16384, kb, &S.wfull[s], pol);
+                                } else {
+                                    const uint32_t vb = (uint32_t)(p.hd * 128);
+                                    mbar_arrive_expect_tx(&S.wfull[s], nj > 64 ? 2 * vb : vb);
+                                    bulk_load(sW + (size_t)s * kSlotBytes, blk + 32768, vb, &S.wfull[s], pol);
+                                    if (nj > 64)
+                                        bulk_load(sW + (size_t)s * kSlotBytes + 16384, blk + 49152, vb, &S.wfull[s], pol);
+                                }
+                                ++wi;
                             }
-                            const uint8_t *blk = kv_block(p, S, l, u, (int)(a - a0) + w, j);
-                            const int nj = min(kKVPos, u.n - j * kKVPos);
-                            const uint32_t kb = (uint32_t)(((nj + 7) & ~7) * 128), vb = (uint32_t)(p.hd * 128);
-                            if (!acquire(wi)) { ok = false; break; }
-                            int s = (int)(wi % nws);
-                            mbar_arrive_expect_tx(&S.wfull[s], p.hd > 64 ? 2 * kb : kb);
-                            bulk_load(sW + (size_t)s * kSlotBytes, blk, kb, &S.wfull[s], pol);
-                            if (p.hd > 64) bulk_load(sW + (size_t)s * kSlotBytes + 16384, blk + 16384, kb, &S.wfull[s], pol);
-                            ++wi;
-                            if (!acquire(wi)) { ok = false; break; }
-                            s = (int)(wi % nws);
-                            mbar_arrive_expect_tx(&S.wfull[s], nj > 64 ? 2 * vb : vb);
-                            bulk_load(sW + (size_t)s * kSlotBytes, blk + 32768, vb, &S.wfull[s], pol);
-                            if (nj > 64) bulk_load(sW + (size_t)s * kSlotBytes + 16384, blk + 49152, vb, &S.wfull[s], pol);
-                            ++wi;
                         }
                     }
                 }
@@ -524,13 +539,12 @@ __device__ __forceinline__ void mega_mma(const MegaParams &p, MegaSmem &S, uint8
     int *err = &p.c.v->err;
     const int NX = S.nx, R16 = S.rows16, nxl = S.nx_lg;
     const uint32_t stage = (uint32_t)R16 * 256;
-    const uint32_t ida = idesc_f16_f32(128, 16);
     // at most 64 live rows: one MMA per k-step over the stacked hi / lo groups (M = 2 R16
     // rounded up to 64 or 128: the rows past the stage only feed accumulator rows nobody
     // reads); more: the hi and the lo groups as two 128-row operands into one accumulator
     const bool stacked = R16 <= 64;
     uint32_t wi = 0, xi = 0;
-    int gi = 0, use0 = 0, use1 = 0, tseg = 0;  // accumulator buffer uses, GEMM tiles so far
+    int use0 = 0, use1 = 0, tseg = 0;  // accumulator buffer uses, GEMM tiles so far
     bool ok = true;
     constexpr uint32_t nws = kWSlots;
     auto wslot = [&](uint32_t i) -> uint32_t { return smem_u32(sW + (size_t)(i % nws) * kSlotBytes); };
@@ -578,64 +592,29 @@ __device__ __forceinline__ void mega_mma(const MegaParams &p, MegaSmem &S, uint8
             ++tseg;
         }
     };
-    // attention: unit pairs (one unit per compute warp group, group (gi + i) & 1), block by
-    // block in lockstep: S(a, j), S(b, j), PV(a, j), PV(b, j).  S(x, j > 0) may overwrite the
-    // score buffer once PV(x, j - 1) was issued (the group had read the scores before it
-    // released P); PV(x, j) waits for P(x, j), which the group publishes only after reading
-    // O(x, j - 1).  Per group: units (q_ready) and blocks (s_full / p_ready / o_full) counted
-    // for the barrier parities.
-    uint32_t aq0 = 0, aq1 = 0, ab0 = 0, ab1 = 0;
-    auto att = [&](int64_t a0, int64_t a1) {
+    // The attention phase's ring entries (its KV tiles) are read and released by the compute
+    // warp groups.  The issuer is the ring's one in-order observer: it waits for each entry to
+    // land and hands it to the group that runs its unit (an arrival on kvready[group][slot]).
+    // A group's consecutive uses of a slot are then at most one barrier phase apart (the slot
+    // is refilled only after the group released its previous tile there), which a group
+    // waiting on the shared wfull barriers directly could not rely on.
+    int gi = 0;  // attention units so far (unit i of a phase runs on group (gi + i) & 1)
+    auto att_fwd = [&](int64_t a0, int64_t a1) -> bool {
         const int n = (int)(a1 - a0), span = S.att_span;
-        uint32_t w = wi;
-        auto scores = [&](int b, uint32_t e, bool first_blk) -> bool {  // S = K q^T
-            uint32_t &cq = b ? aq1 : aq0;
-            if (first_blk) {
-                if (!mwait(&S.q_ready[b], cq & 1, err, ab, lim)) return false;
-                ++cq;
-            }
-            if (!wwait(e)) return false;
-            tc_fence_after();
-            const uint32_t dS = tmem + kTmemS + 16 * b, qb = smem_u32(sQ + 4096 * b), kb = wslot(e);
-            for (int ks = 0; ks < p.hd / 16; ++ks)
-                tc_mma_bf16(dS, sdesc_kmajor_sw128(kb + (ks >> 2) * 16384 + (ks & 3) * 32),
-                            sdesc_kmajor_sw128(qb + (ks >> 2) * 2048 + (ks & 3) * 32), ida, ks > 0 ? 1u : 0u);
-            tc_commit(&S.s_full[b]);
-            tc_commit(&S.wempty[e % nws]);
-            return true;
-        };
-        auto pv = [&](int b, uint32_t e, int nj) -> bool {  // O^T = V^T P^T
-            uint32_t &cb = b ? ab1 : ab0;
-            if (!mwait(&S.p_ready[b], cb & 1, err, ab, lim)) return false;
-            ++cb;
-            if (!wwait(e)) return false;
-            tc_fence_after();
-            const uint32_t dO = tmem + kTmemO + 16 * b, pb = smem_u32(sP + 4096 * b), vb = wslot(e);
-            const int ksteps = (nj + 15) >> 4;
-            for (int ks = 0; ks < ksteps; ++ks)
-                tc_mma_bf16(dO, sdesc_kmajor_sw128(vb + (ks >> 2) * 16384 + (ks & 3) * 32),
-                            sdesc_kmajor_sw128(pb + (ks >> 2) * 2048 + (ks & 3) * 32), ida, ks > 0 ? 1u : 0u);
-            tc_commit(&S.o_full[b]);
-            tc_commit(&S.wempty[e % nws]);
-            return true;
-        };
-        for (int i = 0; i < n && ok; i += 2) {
+        for (int i = 0; i < n; i += 2) {
             const bool two = i + 1 < n;
-            const AttUnit ua = att_unit(p, a0 + i, span);
-            const AttUnit ub = two ? att_unit(p, a0 + i + 1, span) : ua;
-            const int nba = ua.nb, nbb = two ? ub.nb : 0;
-            const int ba = (gi + i) & 1, bb = ba ^ 1;
-            for (int j = 0; j < max(nba, nbb) && ok; ++j) {
-                const uint32_t ea = w, eb = w + (j < nba ? 2u : 0u);
-                w += 2u * ((j < nba ? 1u : 0u) + (j < nbb ? 1u : 0u));
-                if (j < nba && !scores(ba, ea, j == 0)) ok = false;
-                if (ok && j < nbb && !scores(bb, eb, j == 0)) ok = false;
-                if (ok && j < nba && !pv(ba, ea + 1, min(kKVPos, ua.n - j * kKVPos))) ok = false;
-                if (ok && j < nbb && !pv(bb, eb + 1, min(kKVPos, ub.n - j * kKVPos))) ok = false;
-            }
+            const int nba = att_unit(p, a0 + i, span).nb, nbb = two ? att_unit(p, a0 + i + 1, span).nb : 0;
+            for (int j = 0; j < max(nba, nbb); ++j)
+                for (int kv = 0; kv < 2; ++kv)
+                    for (int x = 0; x < 2; ++x) {
+                        if (j >= (x ? nbb : nba)) continue;
+                        if (!wwait(wi)) return false;
+                        mbar_arrive(&S.kvready[(gi + i + x) & 1][wi % nws]);
+                        ++wi;
+                    }
         }
-        wi = w;
         gi += n;
+        return true;
     };
     for (int l = 0; l <= p.layers && ok; ++l) {
         for (int gp = 0; gp < 4 && ok; ++gp) {
@@ -649,7 +628,7 @@ __device__ __forceinline__ void mega_mma(const MegaParams &p, MegaSmem &S, uint8
             if (k == 0 && l < p.layers && ok) {
                 int64_t a0, a1;
                 att_range(p, S.n_items, a0, a1);
-                att(a0, a1);
+                if (!att_fwd(a0, a1)) ok = false;
                 MEGA_STAMP(1 + kPhasesPerLayer * l + kPhAtt, 3);
             }
         }
@@ -694,7 +673,13 @@ __device__ __forceinline__ void mega_compute(const MegaParams &p, MegaSmem &S, u
                        : pair      ? ((lane & 8) == 0 ? quarter * 16 + 8 * (lane >> 4) + (lane & 7) : 1 << 20)
                                    : quarter * 32 + lane;
     const bool quarter_live = (R16 <= 32 ? quarter * 8 : pair ? quarter * 16 : quarter * 32) < R;
-    uint32_t att_blk = 0;  // attention blocks this warp group ran (barrier parities)
+    uint32_t wring = 0;  // W ring entries of the phases before the current one (the producer's count)
+    uint32_t kvpar = 0;  // per ring slot (bit s): parity of this warp group's next kvready wait
+    auto kv_wait = [&](uint32_t e) {
+        const uint32_t sl = e % kWSlots;
+        mwait(&S.kvready[half][sl], (kvpar >> sl) & 1u, err, ab, lim);
+        kvpar ^= 1u << sl;
+    };
     int gi = 0, cuse0 = 0, cuse1 = 0, tseg = 0;  // accumulator buffer uses, GEMM tiles so far
 
     // phase arrival: the CTA's writes of this phase (made visible to thread 0 by the barrier)
@@ -833,6 +818,7 @@ __device__ __forceinline__ void mega_compute(const MegaParams &p, MegaSmem &S, u
                      gdn = gemm_phase(p, l, kPhDown);
         // ------------------------------------------------------------ QKV
         gemm_range(gq, u0, u1);
+        wring += (uint32_t)(u1 - u0);
         gemm_epi(gq, u0, u1);
         arrive(base + kPhQKV, false);
         // ------------------------------------------------------------ q, k, v (once per row)
@@ -924,112 +910,235 @@ __device__ __forceinline__ void mega_compute(const MegaParams &p, MegaSmem &S, u
             int i_unit = 0;
             DETAIL(0);
             // units alternate between the two warp groups: group h (warps 3..6 / 7..10, named
-            // barrier 2 + h) runs the units (gi + i) & 1 == h, each unit: q tile, then per KV
-            // block scores -> running max -> P -> rescaled output sum (online softmax over
-            // the unit's blocks), then output / split partial + merge, in order
+            // barrier 2 + h) runs the units (gi + i) & 1 == h, each unit: q in registers, then
+            // per KV block scores -> probabilities against the running max -> output sum
+            // (online softmax over the unit's blocks, warp-level MMAs on the ring's K and V^T
+            // tiles, which the group releases), then output / split partial + merge, in order
             const int hb = 2 + half;     // this group's named barrier
             const int ht = ctid & 127;   // thread index within the group
-            const int hq = ht >> 5;      // warp within the group (owns TMEM lanes 32 hq..)
+            const int hq = ht >> 5;      // warp within the group
             const int span = S.att_span;
-            for (int i = half ? 1 - (gi & 1) : (gi & 1); i < n; i += 2) {
-                const AttUnit u = att_unit(p, a0 + i, span);
-                const int b = half;
-                const uint16_t *qr = p.qkv16 + (int64_t)u.row * p.nqkv;
-                // ---- q tile rows 0..7 (score columns 8..15 are unused)
+            // ring entries of the phase's KV blocks: per unit pair, block by block, the K of
+            // the pair's units, then their V^T (the W producer's order)
+            uint32_t wpair = wring;
+            uint8_t *pbufs = sQ + half * 2 * kAttPBytes;  // this group's two P buffers
+            const int g8 = lane >> 2, t4 = lane & 3;     // mma fragment row / column pair
+            const int kst = hd >> 4;                      // k-steps of q.k (16 dims each)
+            for (int ip = 0; ip < n; ip += 2) {
+                const bool two = ip + 1 < n;
+                const AttUnit ua = att_unit(p, a0 + ip, span);
+                const int nba = ua.nb, nbb = two ? att_unit(p, a0 + ip + 1, span).nb : 0;
+                const int x = ((gi + ip) & 1) == half ? 0 : 1;  // our unit of the pair
+                const uint32_t w0 = wpair;
+                wpair += 2u * (uint32_t)(nba + nbb);
+                if (x == 1 && !two) continue;
+                const int i = ip + x;
+                const AttUnit u = x ? att_unit(p, a0 + i, span) : ua;
+                const int jm = min(nba, nbb);
+                auto ent = [&](int j, int kv) -> uint32_t {
+                    return j < jm ? w0 + 4u * j + 2u * kv + x : w0 + 4u * jm + 2u * (j - jm) + kv;
+                };
+                if (half == 0) { i_unit = i; DETAIL(1); }
+                // ---- q of the unit's heads as mma B fragments (q^T: k = dim, n = head g8)
+                uint32_t qf[8][2];
                 {
-                    const int g = ht >> 4, j = ht & 15;
-                    uint4 qv = make_uint4(0, 0, 0, 0);
-                    if (g < Gq && j * 8 < hd)
-                        qv = __ldcg(reinterpret_cast<const uint4 *>(qr + (u.kvh * Gq + g) * hd + j * 8));
-                    *reinterpret_cast<uint4 *>(sQ + 4096 * b + (j >> 3) * 2048 + g * 128 + (((j & 7) ^ (g & 7)) << 4)) = qv;
-                    fence_proxy_async_smem();
-                    named_bar_sync(hb, 128);
-                    if (half == 0) { i_unit = i; DETAIL(1); }
-                    if (ht == 0) mbar_arrive(&S.q_ready[b]);
-                }
-                // ---- per block: softmax with the running max, P, rescaled output sum
-                float mrun[8], lrun[8], oacc[8];
+                    const bool hv = g8 < Gq;
+                    const uint16_t *qh = p.qkv16 + (int64_t)u.row * p.nqkv + (u.kvh * Gq + (hv ? g8 : 0)) * hd + 2 * t4;
 #pragma unroll
-                for (int g = 0; g < 8; ++g) { mrun[g] = -INFINITY; lrun[g] = 0.f; oacc[g] = 0.f; }
-                const int pos = quarter * 32 + lane;  // score row (position in the block)
+                    for (int ks = 0; ks < 8; ++ks) {
+                        const bool ok = hv && ks < kst;
+                        qf[ks][0] = ok ? __ldcg(reinterpret_cast<const unsigned int *>(qh + 16 * ks)) : 0u;
+                        qf[ks][1] = ok ? __ldcg(reinterpret_cast<const unsigned int *>(qh + 16 * ks + 8)) : 0u;
+                    }
+                }
+                // ---- per block: S^T = K q^T (warp hq: positions 32 hq ..), probabilities
+                // against the running max, which is re-based only when a score exceeds it by
+                // more than the headroom; P to shared memory; O^T += V^T P^T (warp hq: dims
+                // 16 (hq + 4 m)).  Thread (g8, t4) holds heads 2 t4, 2 t4 + 1 throughout.
+                float mrun[2] = {-INFINITY, -INFINITY}, lthr[2] = {0.f, 0.f};
+                float o[2][4];
+#pragma unroll
+                for (int m = 0; m < 2; ++m)
+#pragma unroll
+                    for (int q = 0; q < 4; ++q) o[m][q] = 0.f;
                 for (int jb = 0; jb < u.nb; ++jb) {
-                    const uint32_t ph = att_blk & 1u;
-                    ++att_blk;
-                    const bool valid = pos < min(kKVPos, u.n - jb * kKVPos);
-                    mwait(&S.s_full[b], ph, err, ab, lim);
+                    const int nj = min(kKVPos, u.n - jb * kKVPos);
+                    const uint32_t ek = ent(jb, 0), ev = ent(jb, 1);
+                    kv_wait(ek);
                     if (half == 0 && jb == 0) DETAIL(2);
-                    tc_fence_after();
-                    float sv[8];
-                    tmem_ld_32x32b_x8(tmem + lane_base + kTmemS + 16 * b, sv);
+                    const uint32_t kbase = smem_u32(sW + (size_t)(ek % kWSlots) * kSlotBytes);
+                    float sc[2][4];
 #pragma unroll
-                    for (int g = 0; g < 8; ++g) {
-                        sv[g] = valid ? sv[g] : -INFINITY;
-                        const float m = warp_max_redux(sv[g]);
-                        if (lane == 0) S.red[half][quarter][g] = m;
-                    }
-                    tc_fence_before();
-                    named_bar_sync(hb, 128);
-                    float mnew[8];
-                    uint8_t *pb = sP + 4096 * b + (pos >> 6) * 2048;
-                    const int pc = pos & 63;
+                    for (int m = 0; m < 2; ++m) {
 #pragma unroll
-                    for (int g = 0; g < 8; ++g) {
-                        mnew[g] = fmaxf(mrun[g], fmaxf(fmaxf(S.red[half][0][g], S.red[half][1][g]),
-                                                       fmaxf(S.red[half][2][g], S.red[half][3][g])));
-                        const float e = valid ? exp2f(sv[g] - mnew[g]) : 0.f;
-                        *reinterpret_cast<uint16_t *>(pb + g * 128 + ((((pc >> 3) ^ (g & 7)) << 4) | ((pc & 7) << 1))) =
-                            f32_to_f16_sat(e);
-                        const float se = warp_sum_unit_redux(e);
-                        if (lane == 0) S.red2[half][quarter][g] = se;
-                    }
-                    fence_proxy_async_smem();
-                    named_bar_sync(hb, 128);
-                    if (half == 0 && jb == 0) DETAIL(3);
-                    if (ht == 0) mbar_arrive(&S.p_ready[b]);
-                    float alpha[8];
+                        for (int q = 0; q < 4; ++q) sc[m][q] = 0.f;
+                        const int pb0 = 32 * hq + 16 * m;
+                        if (pb0 < nj) {  // rows past the copied ones are never read
+                            const int pr = pb0 + (lane & 7) + ((lane >> 3) & 1) * 8;  // ldmatrix row of this lane
 #pragma unroll
-                    for (int g = 0; g < 8; ++g) {
-                        alpha[g] = exp2f(mrun[g] - mnew[g]);  // 0 on the first block
-                        lrun[g] = lrun[g] * alpha[g] + (S.red2[half][0][g] + S.red2[half][1][g]) +
-                                  (S.red2[half][2][g] + S.red2[half][3][g]);
-                        mrun[g] = mnew[g];
-                    }
-                    mwait(&S.o_full[b], ph, err, ab, lim);
-                    if (half == 0 && jb == 0) DETAIL(4);
-                    tc_fence_after();
-                    float ov[8];
-                    tmem_ld_32x32b_x8(tmem + lane_base + kTmemO + 16 * b, ov);
-#pragma unroll
-                    for (int g = 0; g < 8; ++g) oacc[g] = oacc[g] * alpha[g] + ov[g];
-                    tc_fence_before();
-                }
-                // ---- output (single split) or partial + split merge
-                {
-                    const int dd = quarter * 32 + lane;  // output dim of this thread
-                    if (u.nsplit == 1) {
-                        if (dd < hd) {
-#pragma unroll
-                            for (int g = 0; g < 8; ++g)
-                                if (g < Gq)
-                                    store_hilo(p.att, xblk_off(u.row, (u.kvh * Gq + g) * hd + dd, R16c),
-                                               oacc[g] / lrun[g]);
+                            for (int ks = 0; ks < 8; ++ks) {
+                                if (ks < kst) {
+                                    const int dim = 16 * ks + (lane >> 4) * 8;
+                                    uint32_t a[4];
+                                    ldsm_x4(kbase + (dim >> 6) * 16384 + pr * 128 + ((((dim & 63) >> 3) ^ (pr & 7)) << 4), a);
+                                    mma_f16_16816(sc[m], a, qf[ks][0], qf[ks][1]);
+                                }
+                            }
                         }
+                    }
+                    // scores: sc[m][q] = s(position 32 hq + 16 m + g8 + 8 (q >> 1), head 2 t4 + (q & 1))
+                    uint8_t *pbuf = pbufs + (jb & 1) * kAttPBytes;
+                    auto put_p = [&](float (&e)[2][4]) {
+#pragma unroll
+                        for (int m = 0; m < 2; ++m)
+#pragma unroll
+                            for (int q = 0; q < 4; ++q) {
+                                const int pos = 32 * hq + 16 * m + g8 + 8 * (q >> 1);
+                                *reinterpret_cast<uint16_t *>(pbuf + (2 * t4 + (q & 1)) * kAttPRow + 2 * pos) =
+                                    f32_to_f16_sat(e[m][q]);
+                            }
+                    };
+                    float e[2][4];
+                    bool rebase = jb == 0;
+                    if (!rebase) {
+                        bool over = false;
+#pragma unroll
+                        for (int m = 0; m < 2; ++m)
+#pragma unroll
+                            for (int q = 0; q < 4; ++q) {
+                                const bool valid = 32 * hq + 16 * m + g8 + 8 * (q >> 1) < nj;
+                                e[m][q] = valid ? exp2f(sc[m][q] - mrun[q & 1]) : 0.f;
+                                over |= valid && sc[m][q] - mrun[q & 1] > S.p_headroom;
+                            }
+                        put_p(e);
+                        rebase = named_bar_any(hb, 128, over);
+                    }
+                    if (rebase) {  // the block's maximum per head joins the running max
+                        float mx[2] = {-INFINITY, -INFINITY};
+#pragma unroll
+                        for (int m = 0; m < 2; ++m)
+#pragma unroll
+                            for (int q = 0; q < 4; ++q)
+                                if (32 * hq + 16 * m + g8 + 8 * (q >> 1) < nj) mx[q & 1] = fmaxf(mx[q & 1], sc[m][q]);
+#pragma unroll
+                        for (int k = 0; k < 2; ++k)
+#pragma unroll
+                            for (int o2 = 4; o2 < 32; o2 <<= 1) mx[k] = fmaxf(mx[k], __shfl_xor_sync(0xffffffffu, mx[k], o2));
+                        if (g8 == 0) {
+                            S.red[half][hq][2 * t4] = mx[0];
+                            S.red[half][hq][2 * t4 + 1] = mx[1];
+                        }
+                        named_bar_sync(hb, 128);
+                        float alpha[2];
+#pragma unroll
+                        for (int k = 0; k < 2; ++k) {
+                            const int h = 2 * t4 + k;
+                            const float mnew = fmaxf(mrun[k], fmaxf(fmaxf(S.red[half][0][h], S.red[half][1][h]),
+                                                                    fmaxf(S.red[half][2][h], S.red[half][3][h])));
+                            alpha[k] = exp2f(mrun[k] - mnew);  // 0 on the first block
+                            mrun[k] = mnew;
+                            lthr[k] *= alpha[k];
+                        }
+#pragma unroll
+                        for (int m = 0; m < 2; ++m)
+#pragma unroll
+                            for (int q = 0; q < 4; ++q) {
+                                o[m][q] *= alpha[q & 1];
+                                const bool valid = 32 * hq + 16 * m + g8 + 8 * (q >> 1) < nj;
+                                e[m][q] = valid ? exp2f(sc[m][q] - mrun[q & 1]) : 0.f;
+                            }
+                        put_p(e);
+                        named_bar_sync(hb, 128);
+                    }
+                    // every warp has read the K block: its ring slot goes back to the producer
+                    if (ht == 0) mbar_arrive(&S.wempty[ek % kWSlots]);
+#pragma unroll
+                    for (int m = 0; m < 2; ++m)
+#pragma unroll
+                        for (int q = 0; q < 4; ++q) lthr[q & 1] += e[m][q];
+                    if (half == 0 && jb == 0) DETAIL(3);
+                    // ---- O^T += V^T P^T over the block's positions (k-steps of 16)
+                    kv_wait(ev);
+                    const uint32_t vbase = smem_u32(sW + (size_t)(ev % kWSlots) * kSlotBytes);
+                    const uint32_t pbase = smem_u32(pbuf);
+                    const int kpv = (nj + 15) >> 4;
+#pragma unroll
+                    for (int ks = 0; ks < 8; ks += 2) {
+                        if (ks < kpv) {
+                            uint32_t bq[4];  // P^T fragments of k-steps ks, ks + 1 (rows: heads 0..7)
+                            ldsm_x4(pbase + (lane & 7) * kAttPRow + (16 * ks + 8 * (lane >> 3)) * 2, bq);
+#pragma unroll
+                            for (int m = 0; m < 2; ++m) {
+                                const int dr = 16 * (hq + 4 * m) + (lane & 7) + ((lane >> 3) & 1) * 8;  // V^T row (dim)
+                                if (16 * (hq + 4 * m) < hd) {
+#pragma unroll
+                                    for (int kk = 0; kk < 2; ++kk) {
+                                        if (ks + kk < kpv) {
+                                            const int pos = 16 * (ks + kk) + (lane >> 4) * 8;
+                                            uint32_t a[4];
+                                            ldsm_x4(vbase + (pos >> 6) * 16384 + dr * 128 + ((((pos & 63) >> 3) ^ (dr & 7)) << 4), a);
+                                            mma_f16_16816(o[m], a, bq[2 * kk], bq[2 * kk + 1]);
+                                        }
+                                    }
+                                }
+                            }
+                        }
+                    }
+                    named_bar_sync(hb, 128);  // every warp has read the V^T block
+                    if (ht == 0) mbar_arrive(&S.wempty[ev % kWSlots]);
+                }
+                if (half == 0) DETAIL(4);
+                // ---- row sums: heads 2 t4, 2 t4 + 1 over the warp (lanes of equal t4), then
+                // over the group's warps
+                float lrun[2];
+                {
+#pragma unroll
+                    for (int k = 0; k < 2; ++k)
+#pragma unroll
+                        for (int o2 = 4; o2 < 32; o2 <<= 1) lthr[k] += __shfl_xor_sync(0xffffffffu, lthr[k], o2);
+                    if (g8 == 0) {
+                        S.red2[half][hq][2 * t4] = lthr[0];
+                        S.red2[half][hq][2 * t4 + 1] = lthr[1];
+                    }
+                    named_bar_sync(hb, 128);
+#pragma unroll
+                    for (int k = 0; k < 2; ++k) {
+                        const int h = 2 * t4 + k;
+                        lrun[k] = (S.red2[half][0][h] + S.red2[half][1][h]) + (S.red2[half][2][h] + S.red2[half][3][h]);
+                    }
+                }
+                // ---- output (single split) or partial + split merge.  o[m][q]: O^T(dim
+                // 16 (hq + 4 m) + g8 + 8 (q >> 1), head 2 t4 + (q & 1))
+                {
+                    const int dd = quarter * 32 + lane;  // output dim of this thread in the merge
+                    if (u.nsplit == 1) {
+#pragma unroll
+                        for (int m = 0; m < 2; ++m)
+#pragma unroll
+                            for (int q = 0; q < 4; ++q) {
+                                const int dim = 16 * (hq + 4 * m) + g8 + 8 * (q >> 1), h = 2 * t4 + (q & 1);
+                                if (dim < hd && h < Gq)
+                                    store_hilo(p.att, xblk_off(u.row, (u.kvh * Gq + h) * hd + dim, R16c),
+                                               o[m][q] / lrun[q & 1]);
+                            }
                     } else {
                         float *mine = p.part + ((int64_t)u.item * p.KVH + u.kvh) * Gq * (hd + 2);
-                        if (dd < hd) {
 #pragma unroll
-                            for (int g = 0; g < 8; ++g)
-                                if (g < Gq) mine[g * (hd + 2) + 2 + dd] = oacc[g];
-                        }
-                        if (ht < Gq) {
-                            float mc = mrun[0], lc = lrun[0];
+                        for (int m = 0; m < 2; ++m)
 #pragma unroll
-                            for (int g = 1; g < 8; ++g) {
-                                mc = (ht == g) ? mrun[g] : mc;
-                                lc = (ht == g) ? lrun[g] : lc;
+                            for (int q = 0; q < 4; ++q) {
+                                const int dim = 16 * (hq + 4 * m) + g8 + 8 * (q >> 1), h = 2 * t4 + (q & 1);
+                                if (dim < hd && h < Gq) mine[h * (hd + 2) + 2 + dim] = o[m][q];
                             }
-                            mine[ht * (hd + 2)] = mc;
-                            mine[ht * (hd + 2) + 1] = lc;
+                        if (hq == 0 && g8 == 0) {
+#pragma unroll
+                            for (int k = 0; k < 2; ++k) {
+                                const int h = 2 * t4 + k;
+                                if (h < Gq) {
+                                    mine[h * (hd + 2)] = mrun[k];
+                                    mine[h * (hd + 2) + 1] = lrun[k];
+                                }
+                            }
                         }
                         named_bar_sync(hb, 128);
                         if (half == 0) DETAIL(5);
@@ -1094,6 +1203,7 @@ __device__ __forceinline__ void mega_compute(const MegaParams &p, MegaSmem &S, u
                     }
                 }
             }
+            wring = wpair;
             gi += n;
             i_unit = 0;
             DETAIL(8);
@@ -1103,6 +1213,7 @@ __device__ __forceinline__ void mega_compute(const MegaParams &p, MegaSmem &S, u
         }
         // ------------------------------------------------------------ O projection
         gemm_range(go, u0, u1);
+        wring += (uint32_t)(u1 - u0);
         gemm_epi(go, u0, u1);
         arrive(base + kPhO, false);
         // ------------------------------------------------------------ residual, MLP norm input
@@ -1114,6 +1225,7 @@ __device__ __forceinline__ void mega_compute(const MegaParams &p, MegaSmem &S, u
         if (l == min(2, p.layers - 1) && ctid == 0) MEGA_DETAIL(12);
         // ------------------------------------------------------------ gate / up
         gemm_range(gu, u0, u1);
+        wring += (uint32_t)(u1 - u0);
         gemm_epi(gu, u0, u1);
         arrive(base + kPhGU, false);
         // ------------------------------------------------------------ SwiGLU
@@ -1182,6 +1294,7 @@ __device__ __forceinline__ void mega_compute(const MegaParams &p, MegaSmem &S, u
         }
         // ------------------------------------------------------------ down
         gemm_range(gdn, u0, u1);
+        wring += (uint32_t)(u1 - u0);
         gemm_epi(gdn, u0, u1);
         arrive(base + kPhDown, false);
         // ------------------------------------------------------------ residual, next norm input
@@ -1294,15 +1407,16 @@ __global__ void __launch_bounds__(kMegaThreads, 1) decode_step_kernel(const __gr
     StepVars *V = p.c.v;
 
     if (threadIdx.x == 0) {
-        for (int s = 0; s < kWSlots; ++s) { mbar_init(&S.wfull[s], 1); mbar_init(&S.wempty[s], 1); }
+        for (int s = 0; s < kWSlots; ++s) {
+            mbar_init(&S.wfull[s], 1);
+            mbar_init(&S.wempty[s], 1);
+            mbar_init(&S.kvready[0][s], 1);
+            mbar_init(&S.kvready[1][s], 1);
+        }
         for (int s = 0; s < kMaxXStages; ++s) { mbar_init(&S.xfull[s], 1); mbar_init(&S.xempty[s], 1); }
         for (int a = 0; a < 2; ++a) {
             mbar_init(&S.acc_full[a], 1);
             mbar_init(&S.acc_empty[a], 8);
-            mbar_init(&S.q_ready[a], 1);
-            mbar_init(&S.s_full[a], 1);
-            mbar_init(&S.p_ready[a], 1);
-            mbar_init(&S.o_full[a], 1);
         }
         mbar_init(&S.drain, 1);
         const int live = *(volatile int *)&V->live;
@@ -1324,6 +1438,7 @@ __global__ void __launch_bounds__(kMegaThreads, 1) decode_step_kernel(const __gr
         const int64_t wl = p.c.kc->wait_ns;
         S.wait_ns = wl > 0 ? (uint64_t)wl : kWaitLimitNs;
         S.stall_idx = p.c.kc->stall_plus1 - 1;
+        S.p_headroom = p.c.kc->eager_softmax ? 0.f : kSoftmaxHeadroom;
         S.abort = (*(volatile int *)&V->err & ERR_WAIT_TIMEOUT) != 0;
         S.last_flag = 0;
         fence_mbar_init();

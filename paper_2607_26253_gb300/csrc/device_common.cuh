@@ -260,6 +260,25 @@ __device__ __forceinline__ void tmem_ld_32x32b_x8(uint32_t taddr, float (&v)[8])
     for (int i = 0; i < 8; ++i) v[i] = __uint_as_float(r[i]);
 }
 
+// Four 8x8 b16 matrices from shared memory (lane l gives the address of row l % 8 of matrix
+// l / 8); register i of every lane holds its fragment of matrix i.
+__device__ __forceinline__ void ldsm_x4(uint32_t addr, uint32_t (&r)[4]) {
+    asm volatile("ldmatrix.sync.aligned.m8n8.x4.shared.b16 {%0,%1,%2,%3}, [%4];"
+                 : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3])
+                 : "r"(addr)
+                 : "memory");
+}
+// Warp-level D += A B, A 16x16 (row-major fragments a), B 16x8 (column fragments b0, b1), fp16
+// inputs, fp32 accumulator (the register-resident tensor-core path: no tensor memory, no
+// asynchronous completion, for the attention's N = 8 head products).
+__device__ __forceinline__ void mma_f16_16816(float (&d)[4], const uint32_t (&a)[4], uint32_t b0, uint32_t b1) {
+    asm volatile(
+        "mma.sync.aligned.m16n8k16.row.col.f32.f16.f16.f32 {%0,%1,%2,%3}, {%4,%5,%6,%7}, {%8,%9}, "
+        "{%0,%1,%2,%3};"
+        : "+f"(d[0]), "+f"(d[1]), "+f"(d[2]), "+f"(d[3])
+        : "r"(a[0]), "r"(a[1]), "r"(a[2]), "r"(a[3]), "r"(b0), "r"(b1));
+}
+
 // Shared-memory matrix descriptor for a K-major bf16 tile written by TMA with 128-byte
 // swizzling: rows of 64 elements (128 B), 8-row atoms of 1024 B (stride-byte offset), the
 // tile base 1024-byte aligned.  Fields: start address >> 4 (bits 0-13), leading-byte offset
@@ -291,6 +310,20 @@ __host__ __device__ __forceinline__ uint32_t idesc_f16_f32(uint32_t M, uint32_t 
 // Named barrier among `nthreads` threads (multiple of 32) with id `id` (1..15).
 __device__ __forceinline__ void named_bar_sync(int id, int nthreads) {
     asm volatile("bar.sync %0, %1;" ::"r"(id), "r"(nthreads) : "memory");
+}
+
+// Named barrier that also returns whether any of its threads passed v = true.
+__device__ __forceinline__ bool named_bar_any(int id, int nthreads, bool v) {
+    uint32_t r;
+    asm volatile(
+        "{\n\t.reg .pred pi, po;\n\t"
+        "setp.ne.u32 pi, %1, 0;\n\t"
+        "bar.red.or.pred po, %2, %3, pi;\n\t"
+        "selp.u32 %0, 1, 0, po;\n\t}"
+        : "=r"(r)
+        : "r"((uint32_t)v), "r"(id), "r"(nthreads)
+        : "memory");
+    return r != 0;
 }
 
 // Warp maximum of a float in one redux.sync: floats mapped to order-preserving signed ints.

@@ -110,7 +110,7 @@ struct sara_handle {
     double *prior_next = nullptr;  // [2][max_prompts] warm-start priors of the next step
     // failure limits (sara_set_limits): bounded-wait limit, loop bound, stalled phase counter
     uint64_t wait_ns = 0;
-    int32_t max_iters = 0, stall_idx = -1;
+    int32_t max_iters = 0, stall_idx = -1, eager_softmax = 0;
     // graph
     cudaGraph_t graph = nullptr;
     cudaGraphExec_t exec = nullptr;
@@ -855,6 +855,7 @@ void collect_impl(sara_handle &h, const sara_prompts *pr, int64_t N, int32_t k, 
     K.max_iters = h.max_iters;
     K.stall_plus1 = h.stall_idx + 1;
     K.wait_ns = (int64_t)h.wait_ns;
+    K.eager_softmax = h.eager_softmax;
     K.tau_f = (double)t->tau_num / (double)t->tau_den;
     K.warm = warm ? 1 : 0;
     K.schedule = t->schedule;
@@ -1232,6 +1233,7 @@ int sara_profile(sara_handle *h, int32_t kernel, int32_t rows, int32_t ctx, int3
 int sara_set_limits(sara_handle *h, const sara_limits *lim) {
     if (!h || !lim) return SARA_EINVAL;
     if (lim->wait_limit_ns < 0 || lim->max_loop_iters < 0 || lim->stall_phase < -1 ||
+        (lim->eager_softmax != 0 && lim->eager_softmax != 1) || lim->reserved != 0 ||
         (h->has_model && lim->stall_phase >= h->n_phase_cnt)) {
         h->err = "limits out of range";
         return SARA_EINVAL;
@@ -1239,6 +1241,7 @@ int sara_set_limits(sara_handle *h, const sara_limits *lim) {
     h->wait_ns = (uint64_t)lim->wait_limit_ns;
     h->max_iters = lim->max_loop_iters;
     h->stall_idx = lim->stall_phase;
+    h->eager_softmax = lim->eager_softmax;
     return SARA_OK;
 }
 

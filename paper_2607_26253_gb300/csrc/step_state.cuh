@@ -27,6 +27,7 @@ struct StepConst {
     int32_t stall_plus1;  // test hook: 1 + the decode-step phase counter whose waits never
                           // complete (0: none)
     int64_t wait_ns;      // limit of the decode step's bounded waits (0: the built-in 2 s)
+    int32_t eager_softmax;  // 1: attention re-bases its running max at every block that raises it
     double tau_f;         // tau_num / tau_den (the warm-start predictor compares in fp64)
     int32_t warm;         // 1: per-prompt real priors q_pa / q_pb (warm-start) decide
     int32_t schedule;     // 0: synchronised rounds; 1 / 2: asynchronous per prompt (2: with the

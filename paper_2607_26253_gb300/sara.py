@@ -22,7 +22,7 @@ EXPORTED = ("sara_create", "sara_collect_step", "sara_teacher_force", "sara_last
             "sara_gemm_workspace_bytes", "sara_gemm_bf16", "sara_attention_workspace_bytes",
             "sara_attention_decode", "sara_sample", "sara_profile", "sara_gemm_bf16_static", "sara_set_limits",
             "sara_abi_version")
-ABI_VERSION = 2
+ABI_VERSION = 3
 
 c_p = ctypes.c_void_p
 
@@ -66,7 +66,7 @@ class Result(ctypes.Structure):
 
 class Limits(ctypes.Structure):
     _fields_ = [("wait_limit_ns", ctypes.c_int64), ("max_loop_iters", ctypes.c_int32),
-                ("stall_phase", ctypes.c_int32)]
+                ("stall_phase", ctypes.c_int32), ("eager_softmax", ctypes.c_int32), ("reserved", ctypes.c_int32)]
 
 
 class SaraError(RuntimeError):
@@ -276,9 +276,10 @@ class Handle:
         return StepOutput(status, n, s, rnd, toks, counters, float(res.device_ms), float(res.decode_kernel_ms),
                           int(res.kv_blocks_peak), (pan, pbn) if want_next_prior else None)
 
-    def set_limits(self, wait_limit_ns: int = 0, max_loop_iters: int = 0, stall_phase: int = -1):
+    def set_limits(self, wait_limit_ns: int = 0, max_loop_iters: int = 0, stall_phase: int = -1,
+                   eager_softmax: bool = False):
         """Failure limits of later calls (see sara_set_limits); no arguments restores the defaults."""
-        lim = Limits(wait_limit_ns, max_loop_iters, stall_phase)
+        lim = Limits(wait_limit_ns, max_loop_iters, stall_phase, int(eager_softmax), 0)
         _check(load().sara_set_limits(self._h, ctypes.byref(lim)), self._h)
 
     def profile(self, kernel: int, rows: int, ctx: int, iters: int = 20) -> float:

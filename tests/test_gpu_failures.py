@@ -92,7 +92,8 @@ def test_limits_out_of_range_rejected(pkg):
     w = synth.WORKLOADS["tiny"]
     weights = synth.model_weights(w.model, w.weight_seed)
     with pkg.Handle(handle_cfg(w, pkg), weights) as h:
-        for kw in ({"wait_limit_ns": -1}, {"max_loop_iters": -2}, {"stall_phase": -5}, {"stall_phase": 10 ** 6}):
+        for kw in ({"wait_limit_ns": -1}, {"max_loop_iters": -2}, {"stall_phase": -5}, {"stall_phase": 10 ** 6},
+                   {"eager_softmax": 2}):
             with pytest.raises(pkg.SaraError) as e:
                 h.set_limits(**kw)
             assert e.value.code == pkg.SARA_EINVAL

@@ -95,7 +95,8 @@ def test_tiny_other_seeds_and_configs(tiny):
             _assert_schedule(_run_step(h, w, si), oc.collect_workload(w, si))
 
 
-def test_tiny_teacher_forced_logits(tiny):
+@pytest.mark.parametrize("eager", [False, True])
+def test_tiny_teacher_forced_logits(tiny, eager):
     w, weights, h = tiny
     si = synth.step_inputs(w)
     rng = np.random.default_rng(1)
@@ -103,7 +104,11 @@ def test_tiny_teacher_forced_logits(tiny):
     prompts = si.tokens[:n]
     forced = rng.integers(0, w.model.vocab, size=(n, T)).astype(np.int32)
     uids = np.arange(n, dtype=np.int64) * 64 + 1
-    logits, sampled = h.teacher_force(prompts, forced, uids, w.sample_seed)
+    h.set_limits(eager_softmax=eager)
+    try:
+        logits, sampled = h.teacher_force(prompts, forced, uids, w.sample_seed)
+    finally:
+        h.set_limits()
     want = o2.teacher_forced_logits_batch(o2.Weights(w.model, weights), prompts, forced)
     err, rel = logit_errors(logits, want)
     assert err < LOGIT_MAX_ABS and rel < LOGIT_REL_L2, (err, rel)
@@ -187,13 +192,21 @@ def long_case(pkg, request):
     h.close()
 
 
+# eager: the attention re-bases its running maximum at every KV block that raises it, so the
+# rescale of the output accumulated in tensor memory runs on most blocks (by default it runs
+# only when a score exceeds the running maximum by more than 2^8, which these inputs never do)
+@pytest.mark.parametrize("eager", [False, True])
 @pytest.mark.parametrize("n", [26, LONG_ROWS])
-def test_full_shape_long_context_teacher_forced(long_case, n):
+def test_full_shape_long_context_teacher_forced(long_case, n, eager):
     w, h, prompts, forced, want = long_case
     uids = np.arange(n, dtype=np.int64) * 64 + 3
-    logits, sampled = h.teacher_force(prompts[:n], forced[:n], uids, w.sample_seed)
+    h.set_limits(eager_softmax=eager)
+    try:
+        logits, sampled = h.teacher_force(prompts[:n], forced[:n], uids, w.sample_seed)
+    finally:
+        h.set_limits()
     err, rel = logit_errors(logits, want[:n])
-    print(f"{w.model.name} rows {n} context {prompts.shape[1]}: max-abs {err:.2e} rel-L2 {rel:.2e}")
+    print(f"{w.model.name} rows {n} context {prompts.shape[1]} eager {eager}: max-abs {err:.2e} rel-L2 {rel:.2e}")
     assert err < LOGIT_MAX_ABS and rel < LOGIT_REL_L2, (err, rel)
     for i in range(n):
         for t in range(LONG_T):
