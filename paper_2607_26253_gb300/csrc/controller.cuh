@@ -256,7 +256,7 @@ static __device__ void ctl_round_setup(const StepConst &K, StepVars &V, const St
     if (R > c.max_seqs) { if (threadIdx.x == 0) report_error(&V.err, ERR_CAPACITY); return; }
     // first decode step: input = last prompt token at position Lp - 1
     const int nblk = (Lp + K.attn_chunk - 1) / K.attn_chunk;
-    const int span = att_span_for((int64_t)R * nblk, K.att_slots);
+    const int span = att_span_for((int64_t)R * nblk, K.att_slots, R);
     const int nsplit = (nblk + span - 1) / span;
     int maxL = 0;
     for (int r = threadIdx.x; r < R; r += kCtlThreads) {
@@ -688,7 +688,7 @@ static __device__ void ctl_async_join(const StepConst &K, StepVars &V, const Ste
         blk_excl_scan(i < live ? (c.row_pos[i] + K.attn_chunk) / K.attn_chunk : 0, tot, sh);
         blocks += tot;
     }
-    const int span = att_span_for(blocks, K.att_slots);
+    const int span = att_span_for(blocks, K.att_slots, live);
     int items = 0;
     for (int base = 0; base < live; base += kCtlThreads) {
         const int i = base + tid;

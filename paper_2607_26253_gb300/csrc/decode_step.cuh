@@ -1153,6 +1153,15 @@ __device__ __forceinline__ void mega_compute(const MegaParams &p, MegaSmem &S, u
                             const int ns = min(u.nsplit, kMegaMaxSplits);
                             const int64_t sp_stride = (int64_t)p.KVH * Gq * (hd + 2);
                             const float *pbase = p.part + ((int64_t)__ldg(&p.c.row_item0[u.row]) * p.KVH + u.kvh) * Gq * (hd + 2);
+                            // the first four splits' outputs (thread dd: dim dd of every head) load
+                            // together with the split weights' inputs: one round trip for both
+                            const float *src = pbase + 2 + dd;
+                            float vpre[4][8];
+#pragma unroll
+                            for (int q = 0; q < 4; ++q)
+#pragma unroll
+                                for (int g = 0; g < 8; ++g)
+                                    vpre[q][g] = (dd < hd && g < Gq && q < ns) ? __ldcg(src + q * sp_stride + g * (hd + 2)) : 0.f;
                             // split weights 2^(m_s - M) and the total weight L per head (warp hq: heads hq, hq + 4)
                             for (int g = hq; g < Gq; g += 4) {
                                 float ms[3], ls[3];
@@ -1182,14 +1191,22 @@ __device__ __forceinline__ void mega_compute(const MegaParams &p, MegaSmem &S, u
                                 float acc[8];
 #pragma unroll
                                 for (int g = 0; g < 8; ++g) acc[g] = 0.f;
-                                const float *src = pbase + 2 + dd;
-#pragma unroll 2
-                                for (int sp = 0; sp < ns; ++sp) {
-                                    float v[8];
 #pragma unroll
-                                    for (int g = 0; g < 8; ++g) v[g] = g < Gq ? __ldcg(src + sp * sp_stride + g * (hd + 2)) : 0.f;
+                                for (int q = 0; q < 4; ++q)
 #pragma unroll
-                                    for (int g = 0; g < 8; ++g) acc[g] += (g < Gq ? S.mw[half][g][sp] : 0.f) * v[g];
+                                    for (int g = 0; g < 8; ++g) acc[g] += (g < Gq && q < ns ? S.mw[half][g][q] : 0.f) * vpre[q][g];
+                                for (int s0 = 4; s0 < ns; s0 += 4) {  // the rest, four splits' loads in flight
+                                    float v[4][8];
+#pragma unroll
+                                    for (int q = 0; q < 4; ++q)
+#pragma unroll
+                                        for (int g = 0; g < 8; ++g)
+                                            v[q][g] = (g < Gq && s0 + q < ns) ? __ldcg(src + (s0 + q) * sp_stride + g * (hd + 2)) : 0.f;
+#pragma unroll
+                                    for (int q = 0; q < 4; ++q)
+#pragma unroll
+                                        for (int g = 0; g < 8; ++g)
+                                            acc[g] += (g < Gq && s0 + q < ns ? S.mw[half][g][s0 + q] : 0.f) * v[q][g];
                                 }
 #pragma unroll
                                 for (int g = 0; g < 8; ++g)

@@ -1085,7 +1085,7 @@ void profile_impl(sara_handle &h, int which, int rows, int ctx, int iters, doubl
     K.tau_num = 0; K.tau_den = 1; K.decode = 1; K.max_gen = m.max_gen_len; K.attn_chunk = kDecodeChunk;
     K.att_slots = att_slots(h);
     const int nblk = (ctx + kDecodeChunk - 1) / kDecodeChunk;
-    const int span = att_span_for((int64_t)rows * nblk, K.att_slots);
+    const int span = att_span_for((int64_t)rows * nblk, K.att_slots, rows);
     const int nsplit = (nblk + span - 1) / span;
     std::vector<int> slot(rows), pos(rows, ctx - 1), tok(rows, 0), item0(rows), zero(rows, 0), len(rows, m.max_gen_len);
     std::vector<uint64_t> seed(rows);

@@ -202,7 +202,7 @@ static __global__ void __launch_bounds__(256) sample_finish_kernel(StepPtrs c, i
         scan256(i < out ? (c.row_pos[i] + K.attn_chunk) / K.attn_chunk : 0, tot, warp_tot);
         blocks += tot;
     }
-    const int span = att_span_for(blocks, K.att_slots);
+    const int span = att_span_for(blocks, K.att_slots, out);
     int items = 0;
     for (int base = 0; base < out; base += 256) {
         const int i = base + tid;
@@ -238,7 +238,7 @@ static __global__ void __launch_bounds__(kCtlThreads, 1) teacher_setup_kernel(St
     StepVars &V = *c.v;
     const int Lp = K.Lp, Lpre = Lp - 1;
     const int nblk = (Lp + K.attn_chunk - 1) / K.attn_chunk;
-    const int span = att_span_for((int64_t)n * nblk, K.att_slots);
+    const int span = att_span_for((int64_t)n * nblk, K.att_slots, n);
     const int nsplit = (nblk + span - 1) / span;
     const int nsh = shared_blocks(Lp, K.attn_chunk);
     for (int i = threadIdx.x; i < c.n_priv; i += kCtlThreads) c.blk_free[i] = c.n_shared + c.n_priv - 1 - i;

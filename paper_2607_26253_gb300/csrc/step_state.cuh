@@ -66,10 +66,16 @@ struct StepVars {
 };
 
 // KV blocks per decode attention split: the smallest span that leaves at most `slots` split
-// units per kv head when `blocks` blocks (summed over the rows) are to be covered.
-__host__ __device__ inline int att_span_for(int64_t blocks, int slots) {
+// units per kv head when `blocks` blocks (summed over the `rows` rows) are to be covered, and
+// at least the rows' mean block count / kAttSplitsTarget, so that few long rows are not cut
+// into many one-block splits (each split adds partial stores and a share of the merge).
+constexpr int kAttSplitsTarget = 8;
+__host__ __device__ inline int att_span_for(int64_t blocks, int slots, int64_t rows) {
     if (slots < 1) slots = 1;
-    const int64_t s = (blocks + slots - 1) / slots;
+    if (rows < 1) rows = 1;
+    int64_t s = (blocks + slots - 1) / slots;
+    const int64_t by_len = (blocks + rows * kAttSplitsTarget - 1) / (rows * kAttSplitsTarget);
+    if (by_len > s) s = by_len;
     return s < 1 ? 1 : (int)s;
 }
 
