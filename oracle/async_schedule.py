@@ -27,6 +27,12 @@ the closed-form predictor of Prop. 1 / Eq. (peff) and the rule of Eq. (decide):
 
 With every rollout length equal, all prompts in flight finish in the same step, so this
 schedule reproduces the round-synchronous oracle exactly (decode steps = rounds x L).
+
+prior_a / prior_b (optional, float64 [P]): the history warm-start (App. D) on this schedule --
+each prompt's own real Beta prior in Eq. (peff) and Eq. (decide) and in the priority of
+continuing prompts, evaluated in float64 exactly as the warm-start oracle O1w does
+(oracle/warm_start.py); with equal lengths the schedule then reproduces O1w's round-synchronous
+step.
 """
 from __future__ import annotations
 
@@ -36,6 +42,7 @@ from dataclasses import dataclass
 import numpy as np
 
 from . import controller as oc
+from . import warm_start as ow
 
 COUNTER_NAMES = ("rollouts", "gen_tokens", "prefill_tokens", "decode_steps", "events",
                  "committed", "abandoned", "incomplete", "prompts_drawn")
@@ -59,7 +66,7 @@ class AsyncResult:
 
 def collect_step(thresholds: np.ndarray, lengths: np.ndarray, *, k: int, n0: int, tau, target_B: int,
                  N: int, reward_seed: int = 0, commit_min: int | None = None, prior=(1, 1),
-                 prompt_len: int = 1, reserve: bool = False) -> AsyncResult:
+                 prompt_len: int = 1, reserve: bool = False, prior_a=None, prior_b=None) -> AsyncResult:
     thr = np.ascontiguousarray(thresholds, dtype=np.uint64)
     P = thr.size
     L = np.ascontiguousarray(lengths, dtype=np.int64)
@@ -70,6 +77,23 @@ def collect_step(thresholds: np.ndarray, lengths: np.ndarray, *, k: int, n0: int
     cm = k if commit_min is None else commit_min
     a0, b0 = prior
     v = oc.verdicts(thr, k, reward_seed)  # uint8[P][k]: rollout j of prompt q
+    if (prior_a is None) != (prior_b is None):
+        raise ValueError("prior_a and prior_b go together")
+    if prior_a is not None:  # per-prompt real priors (warm-start): float64 predictor and rule
+        pa = np.asarray(prior_a, dtype=np.float64)
+        pb = np.asarray(prior_b, dtype=np.float64)
+
+        def decide(q, nn, ss):
+            return ow.decide(nn, ss, k, float(tau), cm, float(pa[q]), float(pb[q]))
+
+        def peff(q):
+            return ow.peff(int(n[q]), int(s[q]), k, float(pa[q]), float(pb[q]))
+    else:
+        def decide(q, nn, ss):
+            return oc.decide(nn, ss, k, tau, cm, a0, b0)
+
+        def peff(q):
+            return oc.peff(int(n[q]), int(s[q]), k, a0, b0)
 
     status = np.full(P, oc.UNDRAWN, np.uint8)
     n = np.zeros(P, np.int64)
@@ -120,7 +144,7 @@ def collect_step(thresholds: np.ndarray, lengths: np.ndarray, *, k: int, n0: int
             c = batch.pop(q)
             s[q] += int(v[q, n[q]:n[q] + c].sum())
             n[q] += c
-            d = oc.decide(int(n[q]), int(s[q]), k, tau, cm, a0, b0)
+            d = decide(q, int(n[q]), int(s[q]))
             if d == oc.COMMIT:
                 status[q] = oc.COMMITTED
                 decided[q] = t
@@ -137,7 +161,7 @@ def collect_step(thresholds: np.ndarray, lengths: np.ndarray, *, k: int, n0: int
             for q in cont:
                 status[q] = oc.INCOMPLETE
             continue
-        prio = sorted(cont, key=lambda q: (-oc.peff(int(n[q]), int(s[q]), k, a0, b0), q))
+        prio = sorted(cont, key=lambda q: (-peff(q), q))
         for q in prio:
             if used + 1 <= N:
                 issue(q, 1, t + 1)

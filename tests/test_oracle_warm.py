@@ -129,3 +129,81 @@ def test_history_reduces_rollouts_per_effective_group_on_recurring_prompts():
     # carrying the evidence lets saturated prompts be abandoned at the probe
     plain, warm = _multi_step(0.0), _multi_step(0.9)
     assert warm < 0.95 * plain, (plain, warm)
+
+
+# ---- the warm-start on the asynchronous schedule (oracle/async_schedule.py with prior_a / prior_b)
+from oracle import async_schedule as oa  # noqa: E402
+
+
+def _async_case(rng, it, equal_len=None):
+    k = int(rng.choice([4, 8, 16]))
+    tau = float(rng.choice([0.3, 0.45, 0.55]))
+    n0 = int(rng.integers(1, k + 1))
+    P = int(rng.integers(1, 300))
+    lengths = synth.Lengths("uniform", lo=1, hi=40) if equal_len is None else synth.Lengths("uniform", lo=equal_len,
+                                                                                         hi=equal_len)
+    return synth.Workload("warm-async", None, n_prompts=P, prompt_len=1, target_B=int(rng.integers(1, P + 1)), k=k,
+                          n0=n0, tau=tau, budget_N=int(rng.integers(0, 3 * P * k // 2 + 1)),
+                          commit_min=int(rng.integers(2, k + 1)), prior=(int(rng.integers(1, 4)), int(rng.integers(1, 4))),
+                          lengths=lengths, seed_latent=it, seed_lengths=it + 1, reward_seed=it + 2)
+
+
+@pytest.mark.parametrize("reserve", [False, True])
+def test_async_with_uniform_integer_priors_is_the_integer_async_oracle(reserve):
+    """Real priors all equal to the integer base prior: the float64 predictor takes the same
+    decisions and the same priority order as the exact one (cases with a tie excluded)."""
+    rng = np.random.default_rng(21)
+    checked = 0
+    for it in range(80):
+        w = _async_case(rng, it)
+        a0, b0 = w.prior
+        if not _tie_free(w.k, w.tau, a0, b0):
+            continue
+        si = synth.step_inputs(w)
+        kw = dict(k=w.k, n0=w.n0, tau=w.tau, target_B=w.target_B, N=w.budget_N, reward_seed=w.reward_seed,
+                  commit_min=w.commit_floor, prior=w.prior, reserve=reserve)
+        ref = oa.collect_step(si.thresholds, si.lengths, **kw)
+        got = oa.collect_step(si.thresholds, si.lengths, prior_a=np.full(w.n_prompts, float(a0)),
+                              prior_b=np.full(w.n_prompts, float(b0)), **kw)
+        assert np.array_equal(got.status, ref.status) and np.array_equal(got.n, ref.n), it
+        assert np.array_equal(got.s, ref.s) and np.array_equal(got.decided_step, ref.decided_step), it
+        assert got.counters == ref.counters, it
+        checked += 1
+    assert checked >= 40
+
+
+def test_async_with_real_priors_and_equal_lengths_is_the_round_synchronous_warm_oracle():
+    """Every rollout the same length: each step boundary with decisions is a round, so the
+    asynchronous schedule with per-prompt real priors equals O1w's round-synchronous step."""
+    rng = np.random.default_rng(22)
+    for it in range(60):
+        Lc = int(rng.integers(1, 30))
+        w = _async_case(rng, it, equal_len=Lc)
+        si = synth.step_inputs(w)
+        a = rng.uniform(0.5, 6.0, w.n_prompts)
+        b = rng.uniform(0.5, 6.0, w.n_prompts)
+        sync = ow.collect_step(si.thresholds, si.lengths, a, b, k=w.k, n0=w.n0, tau=w.tau, target_B=w.target_B,
+                               N=w.budget_N, reward_seed=w.reward_seed, commit_min=w.commit_floor)
+        asy = oa.collect_step(si.thresholds, si.lengths, k=w.k, n0=w.n0, tau=w.tau, target_B=w.target_B,
+                              N=w.budget_N, reward_seed=w.reward_seed, commit_min=w.commit_floor, prior_a=a,
+                              prior_b=b)
+        assert np.array_equal(asy.status, sync.status), it
+        assert np.array_equal(asy.n, sync.n) and np.array_equal(asy.s, sync.s), it
+        assert np.array_equal(asy.decided_event, sync.decided_round.astype(np.int32)), it
+        for key in ("rollouts", "gen_tokens", "committed", "abandoned", "incomplete", "prompts_drawn"):
+            assert asy.counters[key] == sync.counters[key], (it, key)
+        assert asy.counters["decode_steps"] == sync.counters["rounds"] * Lc
+
+
+def test_async_warm_start_abandons_a_prompt_seen_saturated_at_its_probe():
+    """The hand-worked case of the round schedule, on the asynchronous one: after a step of six
+    failures with lambda = 0.9 the prior is Beta(1, 6.4) and the all-fail probe of 2 has p_eff =
+    1 - 8.4 / 14.4 < 0.45, so the prompt is abandoned when its probe finishes; without the carried
+    prior it continues."""
+    thr = np.array([0], dtype=np.uint64)  # never solved
+    lengths = np.array([[3, 5, 2, 4, 6, 1, 7, 2]], dtype=np.int64)
+    kw = dict(k=8, n0=2, tau=0.45, target_B=1, N=16, reward_seed=0)
+    plain = oa.collect_step(thr, lengths, **kw)
+    warm = oa.collect_step(thr, lengths, prior_a=np.array([1.0]), prior_b=np.array([6.4]), **kw)
+    assert warm.status[0] == oc.ABANDONED and warm.n[0] == 2 and warm.decided_step[0] == 4  # probe ends at step 4
+    assert plain.status[0] == oc.ABANDONED and plain.n[0] == 4  # abandoned at n = 4 (4/9 < 0.45)
