@@ -134,10 +134,13 @@ typedef struct {
                                      rollouts finish and refill happens at the next decode step;
                                   2: as 1, drawing a fresh prompt only if the budget covers it
                                      and every prompt in flight running to k rollouts.
-                                  1 and 2 run on controller-only handles (layers == 0): decode
-                                  time comes from the length table (decode_steps), rounds
-                                  counts the step boundaries with decisions and decided_round
-                                  holds the index of the deciding one (capped at 32767). */
+                                  On controller-only handles (layers == 0) decode time comes
+                                  from the length table (decode_steps); on model handles the
+                                  decode engine decides and refills at every decode-step
+                                  boundary.  For 1 and 2, rounds counts the step boundaries
+                                  with decisions and decided_round holds the index of the
+                                  deciding one (capped at 32767).  Warm-start priors
+                                  (sara_prompts.prior_a / prior_b) apply to every schedule. */
     double decay;              /* warm-start decay lambda in [0, 1] of the carried priors that
                                   sara_result.prior_a_next / prior_b_next receive */
 } sara_thresholds;

@@ -946,7 +946,7 @@ static __global__ void __launch_bounds__(kCtlThreads, 1) ctl_async_kernel(StepPt
             c.q_n[q] = (uint8_t)n;
             c.q_s[q] = (uint8_t)s;
             if (reserve) resv -= k - n;
-            const int d = c.dec_tab[n * kTabDim + s];
+            const int d = K.warm ? decide_real(n, s, K, c.q_pa[q], c.q_pb[q]) : c.dec_tab[n * kTabDim + s];
             if (d == D_COMMIT) {
                 c.q_status[q] = ST_COMMITTED;
                 c.q_round[q] = (int16_t)min(ev, 32767);
@@ -963,15 +963,24 @@ static __global__ void __launch_bounds__(kCtlThreads, 1) ctl_async_kernel(StepPt
             for (int i = 0; i < ncont; ++i) c.q_status[c.act[i]] = ST_INCOMPLETE;
             continue;
         }
-        // continuing prompts by p_eff rank, then stream index (insertion sort: few per event)
+        // continuing prompts by p_eff (the exact rank; with warm-start priors the fp64 value),
+        // then stream index (insertion sort: few per event)
         for (int i = 1; i < ncont; ++i) {
             const int q = c.act[i];
-            const int rq = c.rank_tab[c.q_n[q] * kTabDim + c.q_s[q]];
+            const int rq = K.warm ? 0 : c.rank_tab[c.q_n[q] * kTabDim + c.q_s[q]];
+            const double pq = K.warm ? peff_real(c.q_n[q], c.q_s[q], k, c.q_pa[q], c.q_pb[q]) : 0.0;
             int j = i - 1;
             while (j >= 0) {
                 const int p2 = c.act[j];
-                const int rp = c.rank_tab[c.q_n[p2] * kTabDim + c.q_s[p2]];
-                if (rp < rq || (rp == rq && p2 < q)) break;
+                bool before;
+                if (K.warm) {
+                    const double pp = peff_real(c.q_n[p2], c.q_s[p2], k, c.q_pa[p2], c.q_pb[p2]);
+                    before = pp > pq || (pp == pq && p2 < q);
+                } else {
+                    const int rp = c.rank_tab[c.q_n[p2] * kTabDim + c.q_s[p2]];
+                    before = rp < rq || (rp == rq && p2 < q);
+                }
+                if (before) break;
                 c.act[j + 1] = p2;
                 --j;
             }

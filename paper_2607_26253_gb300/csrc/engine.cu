@@ -818,7 +818,6 @@ void collect_impl(sara_handle &h, const sara_prompts *pr, int64_t N, int32_t k, 
     if (t->schedule < 0 || t->schedule > 2) throw SaraError(SARA_EINVAL, "schedule must be 0, 1 or 2");
     const bool warm = pr->prior_a != nullptr || pr->prior_b != nullptr;
     if (warm && (!pr->prior_a || !pr->prior_b)) throw SaraError(SARA_EINVAL, "prior_a and prior_b go together");
-    if (warm && t->schedule != 0) throw SaraError(SARA_EINVAL, "warm-start priors run with the round schedule");
     if (!(t->decay >= 0.0 && t->decay <= 1.0)) throw SaraError(SARA_EINVAL, "decay must be in [0, 1]");
     if (warm && !pr->on_device) {
         for (int q = 0; q < P; ++q)

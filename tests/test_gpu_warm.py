@@ -13,6 +13,7 @@ import pytest
 
 import synth
 from gpu_util import handle_cfg
+from oracle import async_schedule as oa
 from oracle import controller as oc
 from oracle import warm_start as ow
 
@@ -97,7 +98,64 @@ def test_warm_start_arguments_rejected(pkg):
         kw = dict(thresholds=si.thresholds, lengths=si.lengths, N=w.budget_N, k=8, n0=2, tau=0.45, target_B=16,
                   reward_seed=1)
         for bad in ({"prior_a": np.ones(64)}, {"prior_a": np.ones(64), "prior_b": np.zeros(64)},
-                    {"decay": 1.5}, {"prior_a": np.ones(64), "prior_b": np.ones(64), "schedule": 1}):
+                    {"decay": 1.5}, {"prior_a": np.ones(64), "prior_b": np.full(64, np.inf)}):
             with pytest.raises(pkg.SaraError) as e:
                 h.collect_step(**kw, **bad)
             assert e.value.code == pkg.SARA_EINVAL
+
+
+@pytest.mark.parametrize("schedule", [1, 2])
+def test_warm_start_with_the_asynchronous_schedule(pkg, schedule):
+    """Controller-only handle, several steps with carried priors on the asynchronous schedule
+    (2: with the budget reserve); the budget binds, so continuing prompts at one boundary are
+    ranked by their fp64 p_eff.  Every prompt's outcome, n, s and deciding event, the counters
+    and the carried priors equal the oracle's."""
+    P, B, steps, lam = 1024, 96, 4, 0.9
+    base = synth.Workload("warm-async", None, n_prompts=P, prompt_len=1, target_B=B, k=8, n0=2, tau=0.45,
+                          budget_N=3 * B * 2, lengths=synth.Lengths("uniform", lo=1, hi=40))
+    cfg = pkg.model_cfg(None, max_prompts=P, max_active=B, max_seqs=1, max_prompt_len=1, max_gen_len=64, max_k=8)
+    si = synth.step_inputs(base)
+    a, b = np.ones(P), np.ones(P)
+    with pkg.Handle(cfg) as h:
+        for t in range(steps):
+            seed = 300 + t
+            ref = oa.collect_step(si.thresholds, si.lengths, k=8, n0=2, tau=0.45, target_B=B, N=base.budget_N,
+                                  reward_seed=seed, reserve=schedule == 2, prior_a=a, prior_b=b)
+            w = synth.Workload(base.name, None, n_prompts=P, prompt_len=1, target_B=B, k=8, n0=2, tau=0.45,
+                               budget_N=base.budget_N, lengths=base.lengths, reward_seed=seed)
+            assert _min_margin(si, a, b, w, ref) > 1e-9
+            out = h.collect_step(thresholds=si.thresholds, lengths=si.lengths, N=base.budget_N, k=8, n0=2, tau=0.45,
+                                 target_B=B, reward_seed=seed, prior_a=a, prior_b=b, decay=lam,
+                                 want_next_prior=True, schedule=schedule)
+            assert np.array_equal(out.status, ref.status), t
+            assert np.array_equal(out.n, ref.n) and np.array_equal(out.s, ref.s), t
+            assert np.array_equal(out.decided_round.astype(np.int32), np.minimum(ref.decided_event, 32767)), t
+            c = ref.counters
+            for key, v in (("rollouts", c["rollouts"]), ("gen_tokens", c["gen_tokens"]),
+                           ("decode_steps", c["decode_steps"]), ("rounds", c["events"]),
+                           ("committed", c["committed"]), ("incomplete", c["incomplete"])):
+                assert out.counters[key] == v, (t, key)
+            a, b = ow.carry(a, b, ref.n, ref.s, 1.0, 1.0, lam)
+            assert np.array_equal(out.prior_next[0], a) and np.array_equal(out.prior_next[1], b), t
+
+
+def test_warm_start_with_the_asynchronous_schedule_on_the_decode_engine(pkg):
+    """The tiny policy on the asynchronous schedule with carried priors: decisions at every
+    decode-step boundary take each prompt's own prior; the schedule equals the oracle's."""
+    w = synth.WORKLOADS["tiny"]
+    weights = synth.model_weights(w.model, w.weight_seed)
+    si = synth.step_inputs(w)
+    rng = np.random.default_rng(5)
+    a = 1.0 + 0.9 * rng.integers(0, 5, w.n_prompts)
+    b = 1.0 + 0.9 * rng.integers(0, 5, w.n_prompts)
+    ref = oa.collect_step(si.thresholds, si.lengths, k=w.k, n0=w.n0, tau=w.tau, target_B=w.target_B, N=w.budget_N,
+                          reward_seed=w.reward_seed, prompt_len=w.prompt_len, prior_a=a, prior_b=b)
+    assert _min_margin(si, a, b, w, ref) > 1e-9
+    with pkg.Handle(handle_cfg(w, pkg), weights) as h:
+        out = h.collect_step(thresholds=si.thresholds, lengths=si.lengths, tokens=si.tokens, N=w.budget_N, k=w.k,
+                             n0=w.n0, tau=w.tau, target_B=w.target_B, reward_seed=w.reward_seed,
+                             sample_seed=w.sample_seed, prior_a=a, prior_b=b, schedule=1)
+    assert np.array_equal(out.status, ref.status) and np.array_equal(out.n, ref.n)
+    assert np.array_equal(out.decided_round.astype(np.int32), np.minimum(ref.decided_event, 32767))
+    assert out.counters["decode_steps"] == ref.counters["decode_steps"]
+    assert out.counters["gen_tokens"] == ref.counters["gen_tokens"]
