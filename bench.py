@@ -61,6 +61,10 @@ def parse():
                          "eager decode step) on a reduced-capacity handle of the workload's shapes")
     ap.add_argument("--rows", type=int, default=25, help="live rows in --kernel-profile mode")
     ap.add_argument("--iters", type=int, default=5, help="launches in --kernel-profile mode")
+    ap.add_argument("--points", default=None, metavar="RxC,...",
+                    help="--kernel-profile mode: time the decode-step kernel (1) and the whole decode step (0) "
+                         "at each rows x context point with one handle, e.g. 1x384,26x758,128x300 "
+                         "(the comparison points of the design notes' A/B tables)")
     ap.add_argument("--ctx", type=int, default=None, help="context length in --kernel-profile mode "
                     "(default: prompt length + 128)")
     ap.add_argument("--controller", action="store_true",
@@ -482,6 +486,18 @@ def run_kernel_profile(args):
     gen = max(512, ctx - w.prompt_len + 2 * args.iters + 8)
     cfg = pkg.model_cfg(m, max_prompts=w.n_prompts, max_active=max(16, args.rows), max_seqs=max(32, args.rows),
                         max_prompt_len=w.prompt_len, max_gen_len=gen, max_k=w.k)
+    if args.points:
+        pts = [tuple(int(v) for v in p.split("x")) for p in args.points.split(",")]
+        rmax, cmax = max(r for r, _ in pts), max(c for _, c in pts)
+        cfg = pkg.model_cfg(m, max_prompts=w.n_prompts, max_active=max(16, rmax), max_seqs=max(32, rmax),
+                            max_prompt_len=w.prompt_len, max_gen_len=max(512, cmax - w.prompt_len + 2 * args.iters + 8),
+                            max_k=w.k)
+        with pkg.Handle(cfg, weights, stream=torch.cuda.current_stream()) as h:
+            for rows, c in pts:
+                k1 = h.profile(1, rows, c, iters=args.iters)
+                k0 = h.profile(0, rows, c, iters=args.iters)
+                print(json.dumps({"rows": rows, "ctx": c, "kernel_ms": round(k1, 4), "step_ms": round(k0, 4)}), flush=True)
+        return
     with pkg.Handle(cfg, weights, stream=torch.cuda.current_stream()) as h:
         ms = h.profile(args.kernel_profile, args.rows, ctx, iters=args.iters)
     print(json.dumps({"kernel": args.kernel_profile, "rows": args.rows, "ctx": ctx, "ms_per_launch": ms}))

@@ -755,6 +755,9 @@ __device__ __forceinline__ void mega_compute(const MegaParams &p, MegaSmem &S, u
         for (int u = gw; u < R * d64; u += nw) {
             const int r = u / d64, h64 = u - r * d64;
             const int f = h64 * 64 + lane * 2;
+            // the norm weights load with the residual and the partials (a layer's norm is not
+            // in L1, and after the residual's store the load could not move ahead of it)
+            const uint32_t gb = __ldg(reinterpret_cast<const unsigned int *>(gn + f));
             float2 x = __ldcg(reinterpret_cast<const float2 *>(p.x + (int64_t)r * d + f));
             if (g) {
                 const int gt = f / kTileN, col = f - gt * kTileN;
@@ -776,7 +779,6 @@ __device__ __forceinline__ void mega_compute(const MegaParams &p, MegaSmem &S, u
                 x.x += s.x; x.y += s.y;
                 *reinterpret_cast<float2 *>(p.x + (int64_t)r * d + f) = x;
             }
-            const uint32_t gb = *reinterpret_cast<const uint32_t *>(gn + f);
             uint16_t h0, l0, h1, l1;
             split_bf16(x.x * bf16_to_f32(gb & 0xffff), h0, l0);
             split_bf16(x.y * bf16_to_f32(gb >> 16), h1, l1);
@@ -842,8 +844,16 @@ __device__ __forceinline__ void mega_compute(const MegaParams &p, MegaSmem &S, u
                 const int col = f0 - t * kTileN, pcol = head * hd + pd0 - t * kTileN;
                 int ca, cb;
                 tile_ctas(gq, t, ca, cb);
-                // the row's sum-of-squares partials load with the first batch of QKV partials
+                // the row's sum-of-squares partials and rotation factors load with the first
+                // batch of QKV partials
                 const float sq = lane < d / 64 ? __ldcg(&p.ssqA[(int64_t)lane * p.rows_cap + r]) : 0.f;
+                const int pos = __ldg(&p.c.row_pos[r]);
+                float2 c0r = make_float2(1.f, 0.f), c1r = c0r;
+                if (isq || isk) {
+                    const int fr = d0 < half_hd ? d0 : pd0;
+                    c0r = __ldg(&p.rope[(int64_t)pos * half_hd + fr]);
+                    c1r = __ldg(&p.rope[(int64_t)pos * half_hd + fr + 1]);
+                }
                 float2 x = make_float2(0.f, 0.f), xp = x;
                 for (int c0 = ca; c0 <= cb; c0 += 16) {  // 16 contributors' loads in flight, CTA order
                     float2 a[16], b2[16];
@@ -861,14 +871,10 @@ __device__ __forceinline__ void mega_compute(const MegaParams &p, MegaSmem &S, u
                         xp.x += b2[k].x; xp.y += b2[k].y;
                     }
                 }
-                const int pos = __ldg(&p.c.row_pos[r]);
                 const float rs = rsqrtf(warp_sum(sq) / (float)d + p.eps) * (isq ? p.scale_log2 : 1.f);
                 if (!live) continue;
                 float y0 = x.x, y1 = x.y;
                 if (isq || isk) {  // rotate the pairs (i, i + hd/2)
-                    const int fr = d0 < half_hd ? d0 : pd0;
-                    const float2 c0r = __ldg(&p.rope[(int64_t)pos * half_hd + fr]);
-                    const float2 c1r = __ldg(&p.rope[(int64_t)pos * half_hd + fr + 1]);
                     if (d0 < half_hd) {
                         y0 = x.x * c0r.x - xp.x * c0r.y;
                         y1 = x.y * c1r.x - xp.y * c1r.y;
