@@ -247,19 +247,6 @@ __device__ __forceinline__ unsigned long long ld_acquire_u64(const unsigned long
     return v;
 }
 
-// 32 lanes x 8 consecutive fp32 columns.
-__device__ __forceinline__ void tmem_ld_32x32b_x8(uint32_t taddr, float (&v)[8]) {
-    uint32_t r[8];
-    __syncwarp();  // .aligned: the whole warp converged
-    asm volatile("tcgen05.ld.sync.aligned.32x32b.x8.b32 {%0,%1,%2,%3,%4,%5,%6,%7}, [%8];"
-                 : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]), "=r"(r[7])
-                 : "r"(taddr)
-                 : "memory");
-    asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
-#pragma unroll
-    for (int i = 0; i < 8; ++i) v[i] = __uint_as_float(r[i]);
-}
-
 // Four 8x8 b16 matrices from shared memory (lane l gives the address of row l % 8 of matrix
 // l / 8); register i of every lane holds its fragment of matrix i.
 __device__ __forceinline__ void ldsm_x4(uint32_t addr, uint32_t (&r)[4]) {
@@ -302,11 +289,6 @@ __host__ __device__ __forceinline__ uint32_t idesc_bf16_f32(uint32_t M, uint32_t
     return (1u << 4) | (1u << 7) | (1u << 10) | ((N >> 3) << 17) | ((M >> 4) << 24);
 }
 
-// Instruction descriptor, kind::f16 with fp16 A and B (format 0), fp32 accumulator.
-__host__ __device__ __forceinline__ uint32_t idesc_f16_f32(uint32_t M, uint32_t N) {
-    return (1u << 4) | ((N >> 3) << 17) | ((M >> 4) << 24);
-}
-
 // Named barrier among `nthreads` threads (multiple of 32) with id `id` (1..15).
 __device__ __forceinline__ void named_bar_sync(int id, int nthreads) {
     asm volatile("bar.sync %0, %1;" ::"r"(id), "r"(nthreads) : "memory");
@@ -324,23 +306,6 @@ __device__ __forceinline__ bool named_bar_any(int id, int nthreads, bool v) {
         : "r"((uint32_t)v), "r"(id), "r"(nthreads)
         : "memory");
     return r != 0;
-}
-
-// Warp maximum of a float in one redux.sync: floats mapped to order-preserving signed ints.
-__device__ __forceinline__ float warp_max_redux(float v) {
-    int k = __float_as_int(v);
-    k ^= (k >> 31) & 0x7fffffff;
-    int m;
-    asm volatile("redux.sync.max.s32 %0, %1, 0xffffffff;" : "=r"(m) : "r"(k));
-    m ^= (m >> 31) & 0x7fffffff;
-    return __int_as_float(m);
-}
-// Warp sum of values in [0, 1] in one redux.sync, as 2^-24 fixed point (exact for 32 lanes).
-__device__ __forceinline__ float warp_sum_unit_redux(float v) {
-    const unsigned q = (unsigned)__float2uint_rn(v * 16777216.0f);
-    unsigned s;
-    asm volatile("redux.sync.add.u32 %0, %1, 0xffffffff;" : "=r"(s) : "r"(q));
-    return (float)s * 5.9604644775390625e-08f;
 }
 
 __device__ __forceinline__ float warp_sum(float v) {
