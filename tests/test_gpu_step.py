@@ -168,7 +168,7 @@ def test_full_shape_step_schedule_1p5b(pkg):
 # Long contexts at the full shapes: many rows over a 2,000-token shared prefix, so that the
 # decode step runs the paths the benchmark runs -- 26 rows (one stacked hi/lo operand per
 # k-step) and 80 rows (above 64: hi and lo as separate 128-row operands), attention units of
-# several KV blocks and rows split over several units, merged by the O projection.  The
+# several KV blocks and rows split over several units, merged by the last split to finish.  The
 # oracle computes the prefix once (its keys and values are shared) and then every row's own
 # positions; rows differ in their last 4 prompt tokens and in their forced tokens.
 LONG_PREFIX, LONG_SUFFIX, LONG_T, LONG_ROWS = 2000, 4, 2, 80
@@ -193,7 +193,7 @@ def long_case(pkg, request):
 
 
 # eager: the attention re-bases its running maximum at every KV block that raises it, so the
-# rescale of the output accumulated in tensor memory runs on most blocks (by default it runs
+# rescale of the output accumulated in registers runs on most blocks (by default it runs
 # only when a score exceeds the running maximum by more than 2^8, which these inputs never do)
 @pytest.mark.parametrize("eager", [False, True])
 @pytest.mark.parametrize("n", [26, LONG_ROWS])
