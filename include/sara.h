@@ -241,13 +241,13 @@ SARA_API int sara_profile(sara_handle *h, int32_t kernel, int32_t rows, int32_t 
  *   stall_phase:    -1, or a phase-counter index of the decode-step kernel (0 = embedding,
  *                   1 + 9 l + j = phase j of layer l) whose waits are made to wait for a value
  *                   no launch reaches: they time out after wait_limit_ns.
- *   eager_softmax:  the decode attention's online softmax (Sec. 2's rollout model: causal
- *                   attention over the KV cache) takes each KV block's probabilities against
- *                   a running maximum.  0 (default): the maximum is re-based only when a score
- *                   exceeds it by more than 2^8, so probabilities stay <= 256 and most blocks
- *                   skip the block maximum and the output rescale.  1: re-based at every block
- *                   that raises it (probabilities <= 1).  The same softmax up to rounding; the
- *                   switch exists to test the rescale path.
+ *   eager_softmax:  the decode attention's online softmax takes each KV block's
+ *                   probabilities against a running maximum.  0 (default): the maximum is
+ *                   re-based only when a probability against it would exceed 2^8, so
+ *                   probabilities stay <= 256 and most blocks skip the block maximum and the
+ *                   output rescale.  1: re-based at every block that raises it
+ *                   (probabilities <= 1).  The same softmax up to rounding; the switch exists
+ *                   to test the rescale path.
  * The handle stays usable after a call that failed this way.  SARA_EINVAL if out of range.
  */
 typedef struct {
